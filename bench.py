@@ -1,0 +1,533 @@
+#!/usr/bin/env python3
+"""Benchmark of the FP8 linear training path on GB300.
+
+One step = one forward + backward pass of every linear layer of the
+workload through the library's C ABI, in the paper's recipe (section "FP8
+Mixed-Precision Training"; appendix "FP8 implementation pipeline"):
+
+  forward, layer 0 .. L-1, each linear: quantise W (128x128 blocks, with the
+      transposed copy), quantise X (1x128 groups, rowwise for Fprop and the
+      transposed copy kept for Wgrad), Fprop Y = X W^T
+  backward, layer L-1 .. 0, each linear in reverse: quantise dY (rowwise and
+      transposed), Dgrad dX = dY W, Wgrad dW = dY^T X
+
+Default workload: the 28-layer Qwen2-1.5B linear stack at M = 32768 tokens
+(qkv, o_proj, gate_up, down per layer), distinct seeded inputs per layer,
+all resident in HBM before timing; per-layer inputs (2.4 GB) exceed L2.
+
+Prints one JSON line (rank 0).  `value` is whole-step FP8 fwd+bwd TFLOP/s
+(3 GEMMs x 2MNK per linear, divided by the step time including all
+quantisation).  `roofline` is measured live with CUDA events around every
+launch of the dominant kernel inside the timed steps.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "FP8 linear fwd+bwd TFLOP/s and % of FP8 peak; quantise HBM GB/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+FP8_PER_BF16 = 2.0  # nominal dense ratio (4.5 / 2.25 PFLOP/s)
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", default="C5")
+    ap.add_argument("--scaling", choices=["block", "tensor"], default="block")
+    ap.add_argument("--layers", type=int, default=None, help="override layer count (profiling runs only)")
+    ap.add_argument("--tokens", type=int, default=None, help="override M (profiling runs only)")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-bf16", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    return ap.parse_args()
+
+
+# ----------------------------------------------------------------------------
+# clocks during the timed region
+# ----------------------------------------------------------------------------
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int, enabled: bool = True):
+        self.proc = None
+        self.path = None
+        self.gpu = gpu_index
+        if not enabled:
+            return
+        try:
+            fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+            os.close(fd)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={gpu_index}", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# ----------------------------------------------------------------------------
+# the stack of linears and one step through the C ABI
+# ----------------------------------------------------------------------------
+class LaunchTimer:
+    """CUDA events around launches, grouped by kernel category."""
+
+    def __init__(self, torch):
+        self.torch = torch
+        self.pending = []  # (category, units, start, end)
+        self.enabled = False
+
+    def run(self, cat: str, units: float, fn, *args, **kw):
+        if not self.enabled:
+            return fn(*args, **kw)
+        s = self.torch.cuda.Event(enable_timing=True)
+        e = self.torch.cuda.Event(enable_timing=True)
+        s.record()
+        fn(*args, **kw)
+        e.record()
+        self.pending.append((cat, units, s, e))
+
+    def totals(self):
+        out = {}
+        for cat, units, s, e in self.pending:
+            t = s.elapsed_time(e) * 1e-3
+            c = out.setdefault(cat, {"time_s": 0.0, "units": 0.0, "launches": 0})
+            c["time_s"] += t
+            c["units"] += units
+            c["launches"] += 1
+        return out
+
+
+class LinearStack:
+    def __init__(self, P, W, torch, wl, device, scaling, layers, M):
+        self.P, self.torch = P, torch
+        self.scaling = P.SCALE_BLOCK if scaling == "block" else P.SCALE_TENSOR
+        self.wl = wl
+        self.L = layers
+        self.M = M
+        self.device = device
+        self.timer = LaunchTimer(torch)
+        self.launches_per_step = 0
+        wl_eff = W.Workload(wl.key, wl.description, M, layers, wl.linears, wl.recipe, wl.scaling)
+        self.inputs = [[W.make_linear(wl_eff, l, j, device) for j in range(len(wl.linears))] for l in range(layers)]
+        u8, bf = torch.uint8, torch.bfloat16
+        sc = self.scaling
+        # persistent per layer: quantised weights (both copies) and the transposed X copy for Wgrad
+        self.wq, self.xqt = [], []
+        for l in range(layers):
+            wrow, xrow = [], []
+            for j, (_, N, K) in enumerate(wl.linears):
+                wrow.append(P.Quantized(
+                    P.FP8Operand(torch.empty((N, K), dtype=u8, device=device),
+                                 P.empty_scales(N, K, sc, P.ROLE_WEIGHT, device), scaling=sc, role=P.ROLE_WEIGHT),
+                    P.FP8Operand(torch.empty((K, N), dtype=u8, device=device),
+                                 P.empty_scales(K, N, sc, P.ROLE_WEIGHT, device), scaling=sc, role=P.ROLE_WEIGHT),
+                    torch.zeros(1, dtype=torch.int32, device=device) if sc == P.SCALE_TENSOR else None))
+                xrow.append(P.FP8Operand(torch.empty((K, M), dtype=u8, device=device),
+                                         P.empty_scales(K, M, sc, P.ROLE_ACT, device), scaling=sc))
+            self.wq.append(wrow)
+            self.xqt.append(xrow)
+        # shared across layers (consumed right after they are produced)
+        self.xq, self.dyq, self.y, self.dx, self.dw = [], [], [], [], []
+        for j, (_, N, K) in enumerate(wl.linears):
+            amax = torch.zeros(1, dtype=torch.int32, device=device) if sc == P.SCALE_TENSOR else None
+            self.xq.append(P.FP8Operand(torch.empty((M, K), dtype=u8, device=device),
+                                        P.empty_scales(M, K, sc, P.ROLE_ACT, device), scaling=sc))
+            self.dyq.append(P.Quantized(
+                P.FP8Operand(torch.empty((M, N), dtype=u8, device=device), P.empty_scales(M, N, sc, P.ROLE_ACT, device),
+                             scaling=sc),
+                P.FP8Operand(torch.empty((N, M), dtype=u8, device=device), P.empty_scales(N, M, sc, P.ROLE_ACT, device),
+                             scaling=sc), amax))
+            self.y.append(torch.empty((M, N), dtype=bf, device=device))
+            self.dx.append(torch.empty((M, K), dtype=bf, device=device))
+            self.dw.append(torch.empty((N, K), dtype=bf, device=device))
+        self.xamax = [torch.zeros(1, dtype=torch.int32, device=device) for _ in wl.linears]
+
+    # bytes each quantise launch moves by definition (read bf16, write both
+    # FP8 copies and their scales)
+    def _qbytes(self, rows, cols, role):
+        n = rows * cols
+        if self.scaling == self.P.SCALE_TENSOR:
+            return 4 * n + 8
+        if role == self.P.ROLE_WEIGHT:
+            return 4 * n + 2 * (rows // 128) * (cols // 128)
+        return 4 * n + 2 * n // 128
+
+    def _quant(self, x, role, q: "object"):
+        P, T = self.P, self.timer
+        rows, cols = x.shape
+        if self.scaling == P.SCALE_TENSOR:
+            T.run("amax", 2 * rows * cols, P.puro_fp8_amax, x, q.amax)
+            self.launches_per_step += 1
+        T.run("quantize", self._qbytes(rows, cols, role), P.puro_fp8_quantize, x, P.E4M3, self.scaling, role,
+              q.amax if self.scaling == P.SCALE_TENSOR else None, q.rowwise.data, q.rowwise.scale,
+              q.colwise.data, q.colwise.scale)
+        self.launches_per_step += 1
+
+    def step(self):
+        P, T = self.P, self.timer
+        self.launches_per_step = 0
+        for l in range(self.L):
+            for j, (_, N, K) in enumerate(self.wl.linears):
+                li = self.inputs[l][j]
+                self._quant(li.w, P.ROLE_WEIGHT, self.wq[l][j])
+                xq = P.Quantized(self.xq[j], self.xqt[l][j], self.xamax[j])
+                self._quant(li.x, P.ROLE_ACT, xq)
+                T.run("gemm", 2.0 * self.M * N * K, P.puro_fp8_linear_fprop, self.xq[j], self.wq[l][j].rowwise,
+                      self.y[j])
+                self.launches_per_step += 1
+        for l in reversed(range(self.L)):
+            for j in reversed(range(len(self.wl.linears))):
+                _, N, K = self.wl.linears[j]
+                li = self.inputs[l][j]
+                self._quant(li.dy, P.ROLE_ACT, self.dyq[j])
+                T.run("gemm", 2.0 * self.M * N * K, P.puro_fp8_linear_dgrad, self.dyq[j].rowwise,
+                      self.wq[l][j].colwise, self.dx[j])
+                T.run("gemm", 2.0 * self.M * N * K, P.puro_fp8_linear_wgrad, self.dyq[j].colwise, self.xqt[l][j],
+                      self.dw[j])
+                self.launches_per_step += 2
+
+    def flops_per_step(self):
+        return self.L * sum(6.0 * self.M * N * K for _, N, K in self.wl.linears)
+
+
+def bf16_layer_speedup(P, torch, stack):
+    """Same three GEMMs of layer 0's linears in BF16 (tcgen05 kind::f16) vs
+    FP8 (blockwise, kind::mxf8f6f4), GEMM time only, operands already in
+    the layout each GEMM reads."""
+    dev = stack.device
+    M = stack.M
+    li0 = stack.inputs[0]
+    bufs = []
+    for j, (_, N, K) in enumerate(stack.wl.linears):
+        li = li0[j]
+        bufs.append((li.x, li.w, li.dy, li.w.t().contiguous(), li.dy.t().contiguous(), li.x.t().contiguous(), N, K))
+
+    def run_bf16():
+        for j, (x, w, dy, wt, dyt, xt, N, K) in enumerate(bufs):
+            P.puro_bf16_linear_fprop(x, w, stack.y[j], M, N, K)
+        for j, (x, w, dy, wt, dyt, xt, N, K) in enumerate(bufs):
+            P.puro_bf16_linear_dgrad(dy, wt, stack.dx[j], M, N, K)
+            P.puro_bf16_linear_wgrad(dyt, xt, stack.dw[j], M, N, K)
+
+    def run_fp8():
+        for j, (_, N, K) in enumerate(stack.wl.linears):
+            P.puro_fp8_linear_fprop(stack.xq[j], stack.wq[0][j].rowwise, stack.y[j])
+        for j, (_, N, K) in enumerate(stack.wl.linears):
+            P.puro_fp8_linear_dgrad(stack.dyq[j].rowwise, stack.wq[0][j].colwise, stack.dx[j])
+            P.puro_fp8_linear_wgrad(stack.dyq[j].colwise, stack.xqt[0][j], stack.dw[j])
+
+    def timeit(fn, reps=5):
+        for _ in range(2):
+            fn()
+        torch.cuda.synchronize()
+        s = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        s.record()
+        for _ in range(reps):
+            fn()
+        e.record()
+        torch.cuda.synchronize()
+        return s.elapsed_time(e) * 1e-3 / reps
+
+    # fill the FP8 operands of layer 0 (quantise once, outside the timing)
+    for j, (_, N, K) in enumerate(stack.wl.linears):
+        li = li0[j]
+        P.quantize(li.w, P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT, out=stack.wq[0][j])
+        P.quantize(li.x, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT, out=P.Quantized(stack.xq[j], stack.xqt[0][j]))
+        P.quantize(li.dy, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT, out=stack.dyq[j])
+    t_bf16 = timeit(run_bf16)
+    t_fp8 = timeit(run_fp8)
+    flops = sum(6.0 * M * N * K for _, N, K in stack.wl.linears)
+    del bufs
+    torch.cuda.empty_cache()
+    return {"layer": 0, "bf16_gemm_tflops": flops / t_bf16 / 1e12, "fp8_gemm_tflops": flops / t_fp8 / 1e12,
+            "fp8_over_bf16": t_bf16 / t_fp8, "paper_fp8_over_bf16_whole_model_rtx5090": 1.36}
+
+
+def e2e_measure(P, torch, stack, steps):
+    """Same step with host-resident inputs: every layer's X and dY are copied
+    from pinned host memory into the device buffers before use, and every
+    layer's dW is read back to pinned host memory; copies are inside the
+    timed region.  The pinned source holds layer 0's inputs and serves
+    every layer."""
+    dev = stack.device
+    hx = [li.x.cpu().pin_memory() for li in stack.inputs[0]]
+    hdy = [li.dy.cpu().pin_memory() for li in stack.inputs[0]]
+    hdw = [torch.empty(d.shape, dtype=d.dtype).pin_memory() for d in stack.dw]
+    h2d = 0
+    d2h = 0
+
+    def one_step():
+        nonlocal h2d, d2h
+        h2d = d2h = 0
+        P_ = P
+        for l in range(stack.L):
+            for j, (_, N, K) in enumerate(stack.wl.linears):
+                li = stack.inputs[l][j]
+                li.x.copy_(hx[j], non_blocking=True)
+                h2d += hx[j].numel() * 2
+                stack._quant(li.w, P_.ROLE_WEIGHT, stack.wq[l][j])
+                xq = P_.Quantized(stack.xq[j], stack.xqt[l][j], stack.xamax[j])
+                stack._quant(li.x, P_.ROLE_ACT, xq)
+                P_.puro_fp8_linear_fprop(stack.xq[j], stack.wq[l][j].rowwise, stack.y[j])
+        for l in reversed(range(stack.L)):
+            for j in reversed(range(len(stack.wl.linears))):
+                li = stack.inputs[l][j]
+                li.dy.copy_(hdy[j], non_blocking=True)
+                h2d += hdy[j].numel() * 2
+                stack._quant(li.dy, P_.ROLE_ACT, stack.dyq[j])
+                P_.puro_fp8_linear_dgrad(stack.dyq[j].rowwise, stack.wq[l][j].colwise, stack.dx[j])
+                P_.puro_fp8_linear_wgrad(stack.dyq[j].colwise, stack.xqt[l][j], stack.dw[j])
+                hdw[j].copy_(stack.dw[j], non_blocking=True)
+                d2h += stack.dw[j].numel() * 2
+
+    stack.timer.enabled = False
+    one_step()
+    torch.cuda.synchronize()
+    s = torch.cuda.Event(enable_timing=True)
+    e = torch.cuda.Event(enable_timing=True)
+    s.record()
+    for _ in range(steps):
+        one_step()
+    e.record()
+    torch.cuda.synchronize()
+    t = s.elapsed_time(e) * 1e-3 / steps
+    return {"value": stack.flops_per_step() / t / 1e12, "unit": "TFLOP/s", "ms_per_step": t * 1e3,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "note": "inputs copied from pinned host memory (layer 0's bytes serve every layer), dW read back"}
+
+
+def cpu_baseline(torch, stack, seconds_hint=True):
+    """The oracle, as it stands, on the host cores: quantise + Fprop/Dgrad/Wgrad
+    in fp64 for the first M_s tokens of layer 0's o_proj linear."""
+    import numpy as np
+
+    import oracle as O
+
+    M_s = 2048
+    li = stack.inputs[0][1]  # o_proj [1536, 1536]
+    N, K = li.w.shape
+
+    def b(t):
+        return t.contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+
+    x, w, dy = b(li.x[:M_s]), b(li.w), b(li.dy[:M_s])
+    threads = os.cpu_count() or 1
+    t0 = time.perf_counter()
+    O.linear_block(x, w, dy, nthreads=threads)
+    t = time.perf_counter() - t0
+    flops = 6.0 * M_s * N * K
+    return {"value": flops / t / 1e12, "unit": "TFLOP/s", "cores": threads, "kind": "oracle",
+            "seconds": t, "sample": f"layer 0 o_proj [{N},{K}], first {M_s} of {stack.M} tokens: blockwise "
+                                    f"quantise + Fprop/Dgrad/Wgrad in fp64 ({flops / 1e9:.1f} GFLOP)"}
+
+
+# ----------------------------------------------------------------------------
+def reference_arm(args):
+    """The oracle timed on host cores, same metric/unit/config."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import numpy as np
+    import torch
+
+    import oracle as O
+    from paper_2608_27370_gb300 import workloads as W
+
+    wl = W.WORKLOADS[args.config]
+    M_s = 256
+    _, N, K = wl.linears[1] if len(wl.linears) > 1 else wl.linears[0]
+    g = lambda shape, std, seed: W.normal_bf16(shape, std, "cpu", seed).view(torch.int16).numpy().view(np.uint16)  # noqa
+    x, w, dy = g((M_s, K), 1.0, 1), g((N, K), 0.02, 2), g((M_s, N), 1e-3, 3)
+    threads = os.cpu_count() or 1
+    flops = 6.0 * M_s * N * K
+    for _ in range(args.warmup):
+        O.linear_block(x, w, dy, nthreads=threads)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        O.linear_block(x, w, dy, nthreads=threads)
+    t = (time.perf_counter() - t0) / max(args.steps, 1)
+    v = flops / t / 1e12
+    sample = f"one [{N},{K}] linear of {args.config}, {M_s} tokens per step: blockwise quantise + 3 GEMMs in fp64"
+    line = {"metric": METRIC, "value": v, "unit": "TFLOP/s", "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": t * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": wl.description, "tokens_per_step": M_s},
+            "cpu_baseline": {"value": v, "unit": "TFLOP/s", "cores": threads, "kind": "oracle", "sample": sample},
+            "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return reference_arm(args)
+
+    import torch
+    import torch.distributed as dist
+
+    import paper_2608_27370_gb300 as P
+    from paper_2608_27370_gb300 import workloads as W
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    device = f"cuda:{local}"
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device(device))
+    P.load_library()
+    peaks, peak_src = load_peaks()
+
+    wl = W.WORKLOADS[args.config]
+    layers = args.layers or wl.layers
+    M = args.tokens or wl.M
+    stack = LinearStack(P, W, torch, wl, device, args.scaling, layers, M)
+    torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        stack.step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = ClockSampler(local, enabled=not args.no_clocks)
+    stack.timer.pending.clear()
+    stack.timer.enabled = True
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record()
+    for _ in range(args.steps):
+        stack.step()
+    t_end.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    stack.timer.enabled = False
+    elapsed = t_start.elapsed_time(t_end) * 1e-3
+    if world > 1:
+        t = torch.tensor([elapsed], device=device, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed = float(t.item())
+        dist.barrier()
+    per_kernel = stack.timer.totals()
+    step_s = elapsed / args.steps
+    flops = stack.flops_per_step()
+    value = world * flops / step_s / 1e12
+
+    fp8_peak_burst = peaks["bf16_tflops"] * FP8_PER_BF16
+    fp8_peak_sust = peaks["bf16_tflops_sustained"] * FP8_PER_BF16
+    g = per_kernel.get("gemm", {"time_s": 1.0, "units": 0.0, "launches": 1})
+    q = per_kernel.get("quantize", {"time_s": 1.0, "units": 0.0, "launches": 1})
+    gemm_tflops = g["units"] / g["time_s"] / 1e12
+    quant_gbs = q["units"] / q["time_s"] / 1e9
+    total_kernel_time = sum(c["time_s"] for c in per_kernel.values())
+    shares = {k: c["time_s"] / total_kernel_time for k, c in per_kernel.items()}
+
+    result = {
+        "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "fp8_e4m3" + ("+e8m0_block_scales" if args.scaling == "block" else "+fp32_tensor_scale"),
+        "data": "synthetic",
+        "config": {"workload": f"{wl.key}: " + wl.description if layers == wl.layers and M == wl.M else
+                   f"{wl.key} profile subset: {layers} layers, M={M}",
+                   "tokens_per_step": M, "layers": layers, "linears_per_layer": len(wl.linears),
+                   "scaling": args.scaling, "l2": "inputs larger than L2 (>=2.4 GB per layer)",
+                   "parallelism": f"replicas x{world} (weak scaling, no collective on the path)"},
+        "pct_fp8_peak": 100.0 * value / world / fp8_peak_sust,
+        "tokens_per_s": world * M / step_s,
+        "gemm_only_tflops": gemm_tflops,
+        "quantize_gbs": quant_gbs,
+        "kernel_time_share": shares,
+        "gpu_launches": stack.launches_per_step * args.steps,
+        "roofline": {"bound": "tensor", "kernel": "gemm_tn_kernel<FP8 block-scaled>", "achieved": gemm_tflops,
+                     "peak": fp8_peak_sust, "unit": "TFLOP/s", "frac": gemm_tflops / fp8_peak_sust,
+                     "peak_source": f"2 x bf16_tflops_sustained ({peak_src}); kernel timed inside a long step",
+                     "traffic": None},
+        "roofline_quantize": {"bound": "hbm", "kernel": "quant_tile_kernel", "achieved": quant_gbs,
+                              "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": quant_gbs / peaks["hbm_gbs"],
+                              "peak_source": f"hbm_gbs ({peak_src})", "traffic": None},
+    }
+    if args.scaling == "tensor":
+        result["roofline"]["kernel"] = "gemm_tn_kernel<FP8 per-tensor>"
+    if clk:
+        result["clocks"] = clk
+    if rank == 0 and world == 1 and not args.no_bf16 and args.scaling == "block":
+        try:
+            result["bf16_comparison"] = bf16_layer_speedup(P, torch, stack)
+        except (RuntimeError, torch.cuda.OutOfMemoryError) as exc:  # report, do not hide
+            result["bf16_comparison"] = {"error": str(exc)}
+    if not args.no_e2e:
+        result["e2e"] = e2e_measure(P, torch, stack, max(1, min(args.steps, 3)))
+        if world > 1:
+            t = torch.tensor([result["e2e"]["ms_per_step"]], device=device, dtype=torch.float64)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            result["e2e"]["ms_per_step"] = float(t.item())
+            result["e2e"]["value"] = world * flops / (float(t.item()) * 1e-3) / 1e12
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(torch, stack)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

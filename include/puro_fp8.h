@@ -1,0 +1,210 @@
+/*
+ * puro_fp8.h -- C ABI of the GB300 (sm_103a) FP8 linear-layer training path.
+ *
+ * The method (Puro-2B, section "FP8 Mixed-Precision Training"; appendix
+ * "Production Training Details", paragraph "FP8 implementation pipeline"
+ * and its precision-flow figure):
+ *   - every Transformer linear layer runs its three GEMMs -- Fprop
+ *     Y = X W^T, Dgrad dX = dY W, Wgrad dW = dY^T X -- from FP8 operands,
+ *     accumulates in FP32 and writes a BF16 output;
+ *   - operands are E4M3; inputs and weights are quantised from BF16
+ *     immediately before the GEMM, with scales computed online per local
+ *     group: 1x128 groups along the GEMM reduction dimension for activations
+ *     and activation gradients, 128x128 blocks for weights;
+ *   - each group scale is a power of two (E8M0 expressiveness);
+ *   - the quantised input is kept for Wgrad.
+ * A per-tensor ("one scale for an entire tensor", the contrast drawn in the
+ * same section) mode and the E5M2 format are provided as well.
+ *
+ * Conventions for every entry point
+ *   - Ownership: the caller allocates and owns every buffer.  The library
+ *     allocates no memory, never synchronises the stream (except
+ *     puro_fp8_get_status, which says so) and keeps no state between calls.
+ *   - Ordering: all work is enqueued on `stream` (a cudaStream_t passed as
+ *     void*; NULL is the legacy default stream) in call order.
+ *   - Pointers: device pointers unless marked "host".  Every tensor pointer
+ *     must be 16-byte aligned.
+ *   - Errors: argument violations are detected on the host before anything
+ *     is enqueued and return PURO_ERR_INVALID_ARG or PURO_ERR_UNSUPPORTED;
+ *     a failed launch returns PURO_ERR_CUDA.  No entry point traps or
+ *     asserts on the device.  Non-finite data is carried in-band (NaN codes,
+ *     E8M0 0xFF, NaN scale_inv).  A GEMM whose pipeline wait exceeds its
+ *     internal iteration bound exits cleanly and stores PURO_ERR_TIMEOUT in
+ *     *dev_status when dev_status is non-NULL.
+ *   - Layout: every tensor is row-major and dense.  A quantised GEMM operand
+ *     is stored [rows, red] with the reduction dimension `red` contiguous;
+ *     all three GEMMs read both operands this way ("TN"), which is why the
+ *     quantiser can emit a transposed copy.
+ *
+ * Scale layouts
+ *   PURO_SCALE_TENSOR : `scale` is one float, the dequantisation factor
+ *                       scale_inv = fp32(1 / fp32(fmt_max / amax)).
+ *   PURO_SCALE_BLOCK, role ACT (1x128 groups along `red`):
+ *                       uint8 E8M0 exponents g (value 2^(g-127)), stored
+ *                       group-major: s[(c / 128) * rows + r] is the scale of
+ *                       elements (r, c .. c+127).  Shape [red/128][rows].
+ *   PURO_SCALE_BLOCK, role WEIGHT (128x128 blocks):
+ *                       uint8 E8M0 exponents, s[(r/128) * (red/128) + c/128],
+ *                       shape [rows/128][red/128] (plain row-major grid).
+ *   g = 0xFF marks a group that held Inf or NaN; its codes are NaN.
+ */
+#ifndef PURO_FP8_H
+#define PURO_FP8_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    PURO_OK = 0,
+    PURO_ERR_INVALID_ARG = 1,  /* null/misaligned pointer, bad shape, bad enum */
+    PURO_ERR_UNSUPPORTED = 2,  /* valid request this build does not implement */
+    PURO_ERR_CUDA = 3,         /* a CUDA runtime/driver call failed */
+    PURO_ERR_TIMEOUT = 4       /* device-side bounded wait expired (see dev_status) */
+} puro_status_t;
+
+typedef enum { PURO_E4M3 = 0, PURO_E5M2 = 1 } puro_fp8_format_t;
+typedef enum { PURO_SCALE_TENSOR = 0, PURO_SCALE_BLOCK = 1 } puro_scaling_t;
+typedef enum { PURO_ROLE_ACT = 0, PURO_ROLE_WEIGHT = 1 } puro_role_t;
+
+/* One quantised GEMM operand, as produced by puro_fp8_quantize. */
+typedef struct {
+    const uint8_t *data;  /* device, [rows, red] FP8 codes, row-major        */
+    const void *scale;    /* device, layout per `scaling` and `role` above   */
+    int64_t rows;         /* non-reduction extent                            */
+    int64_t red;          /* reduction extent (contiguous)                   */
+    int32_t fmt;          /* puro_fp8_format_t                               */
+    int32_t scaling;      /* puro_scaling_t                                  */
+    int32_t role;         /* puro_role_t (BLOCK only; ignored for TENSOR)    */
+    int32_t reserved;     /* must be 0                                       */
+} puro_fp8_tensor_t;
+
+/*
+ * amax: max |x| over a BF16 tensor -- the online scale statistic of the
+ * section "FP8 Mixed-Precision Training" ("compute scales online").
+ *   x         : device, [rows, cols] bf16, 16-byte aligned.
+ *   amax_bits : device, one uint32.  The call zeroes it (stream-ordered)
+ *               and then writes the bf16 bit pattern of max |x| (sign
+ *               cleared) into its low 16 bits.  Computed as an integer max
+ *               of (bits & 0x7FFF): exact, order independent, and NaN
+ *               propagating (any NaN gives a value > 0x7F80).
+ * rows == 0 or cols == 0 is valid and yields 0.
+ */
+puro_status_t puro_fp8_amax(const void *x, int64_t rows, int64_t cols,
+                            uint32_t *amax_bits, void *stream);
+
+/*
+ * quantize: BF16 -> FP8 with online scales (section "FP8 Mixed-Precision
+ * Training"), optionally emitting the transposed copy that Wgrad consumes
+ * (same section: "its quantized input is retained for Wgrad").
+ *   x        : device [rows, cols] bf16.
+ *   fmt      : PURO_E4M3 or PURO_E5M2.
+ *   scaling  : PURO_SCALE_BLOCK (the paper's recipe) or PURO_SCALE_TENSOR.
+ *   role     : BLOCK only.  ACT: 1x128 groups along cols for q and along
+ *              rows for q_t.  WEIGHT: 128x128 blocks; q_t holds exactly the
+ *              transposed codes and scale_t the transposed grid.
+ *   amax_bits: TENSOR only: device uint32 written by puro_fp8_amax on this
+ *              same x; NULL in BLOCK mode.
+ *   q, scale : rowwise copy [rows, cols] and its scales (layouts above).
+ *   q_t, scale_t : optional transposed copy [cols, rows] and its scales.
+ *              BLOCK: both NULL or both non-NULL.  TENSOR: scale_t may be
+ *              NULL; when given it receives the same scale_inv.
+ * Codes: code = RNE_satfinite(x * 2^(127-g)) in BLOCK mode, where g is the
+ * smallest exponent with amax <= fmt_max * 2^(g-127) (clamped to [0,254]);
+ * code = RNE_satfinite(fp32(x * scale)) in TENSOR mode, scale =
+ * fp32(fmt_max / amax) (1 if amax == 0, FLT_MAX if the quotient overflows).
+ * Negative values that round to zero give -0 (0x80).
+ * Shapes: BLOCK needs rows % 128 == 0 and cols % 128 == 0.  TENSOR needs
+ * cols % 16 == 0, and rows % 16 == 0 when q_t is requested.  An empty
+ * tensor (rows or cols 0) writes no codes, so x, q and q_t may be NULL;
+ * in TENSOR mode it still writes scale_inv = 1 (amax of nothing is 0).
+ */
+puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t cols,
+                                int32_t fmt, int32_t scaling, int32_t role,
+                                const uint32_t *amax_bits,
+                                uint8_t *q, void *scale,
+                                uint8_t *q_t, void *scale_t,
+                                void *stream);
+
+/*
+ * The three FP8 GEMMs of a linear layer with weight W [N, K], input X [M, K]
+ * and output gradient dY [M, N] (appendix "FP8 implementation pipeline":
+ * Fprop, Dgrad and Wgrad all use blockwise E4M3 operands).  Each computes
+ *     D[i, j] = sum_r sA(i, r) sB(j, r) qA[i, r] qB[j, r]
+ * with FP32 accumulation on the tensor cores and BF16 (RNE) output, where
+ * the scales are the E8M0 group scales (BLOCK) or the two scale_inv values
+ * (TENSOR, applied in the epilogue).
+ *   fprop: A = x   (Xq   [M, K], ACT)    B = w   (Wq   [N, K], WEIGHT)  -> y  [M, N]
+ *   dgrad: A = dy  (dYq  [M, N], ACT)    B = w_t (Wq^T [K, N], WEIGHT)  -> dx [M, K]
+ *   wgrad: A = dy_t(dYq^T[N, M], ACT)    B = x_t (Xq^T [K, M], ACT)     -> dw [N, K]
+ * Both operands must use the same `scaling`.  BLOCK: all extents multiples
+ * of 128.  TENSOR: extents multiples of 16.  A zero reduction extent writes
+ * zeros; a zero output extent is a no-op.
+ *   workspace, workspace_bytes: optional scratch (may be NULL/0).  When at
+ *     least puro_fp8_workspace_size(...) bytes are given, small-output
+ *     GEMMs may split the reduction across CTAs; results are the same
+ *     within the output tolerance either way.
+ *   dev_status: optional device int32, written only on a device-side
+ *     timeout (PURO_ERR_TIMEOUT).  The caller zeroes it.
+ */
+puro_status_t puro_fp8_linear_fprop(const puro_fp8_tensor_t *x, const puro_fp8_tensor_t *w,
+                                    void *y, void *workspace, size_t workspace_bytes,
+                                    int32_t *dev_status, void *stream);
+puro_status_t puro_fp8_linear_dgrad(const puro_fp8_tensor_t *dy, const puro_fp8_tensor_t *w_t,
+                                    void *dx, void *workspace, size_t workspace_bytes,
+                                    int32_t *dev_status, void *stream);
+puro_status_t puro_fp8_linear_wgrad(const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t,
+                                    void *dw, void *workspace, size_t workspace_bytes,
+                                    int32_t *dev_status, void *stream);
+
+/*
+ * Scratch bytes that let a GEMM with output [rows_out, cols_out] and
+ * reduction extent `red` use its split-reduction schedule (0 if it never
+ * would).  Host-only, no CUDA call.
+ */
+size_t puro_fp8_workspace_size(int64_t rows_out, int64_t cols_out, int64_t red);
+
+/*
+ * Copy *dev_status to *host_out (host pointer).  Synchronises `stream`.
+ */
+puro_status_t puro_fp8_get_status(const int32_t *dev_status, int32_t *host_out, void *stream);
+
+/*
+ * BF16 build of the same three GEMMs on the same tensor cores, for the
+ * FP8-versus-BF16 comparison the paper reports (appendix "MuonH
+ * Scaling-Ladder Analysis", "Precision and throughput decomposition").
+ * Operands are BF16, row-major, reduction dimension contiguous (the same
+ * TN forms as above; the caller supplies W^T, dY^T, X^T for dgrad/wgrad).
+ *   fprop: x [M,K], w [N,K]      -> y  [M,N]
+ *   dgrad: dy [M,N], w_t [K,N]   -> dx [M,K]
+ *   wgrad: dy_t [N,M], x_t [K,M] -> dw [N,K]
+ * Extents must be multiples of 8.
+ */
+puro_status_t puro_bf16_linear_fprop(const void *x, const void *w, void *y,
+                                     int64_t M, int64_t N, int64_t K,
+                                     int32_t *dev_status, void *stream);
+puro_status_t puro_bf16_linear_dgrad(const void *dy, const void *w_t, void *dx,
+                                     int64_t M, int64_t N, int64_t K,
+                                     int32_t *dev_status, void *stream);
+puro_status_t puro_bf16_linear_wgrad(const void *dy_t, const void *x_t, void *dw,
+                                     int64_t M, int64_t N, int64_t K,
+                                     int32_t *dev_status, void *stream);
+
+/*
+ * Wall-time bound (nanoseconds, process-wide, default 2e9) of every
+ * device-side pipeline wait in the GEMM kernels.  Fault-detection tests
+ * lower it to force the PURO_ERR_TIMEOUT path without hanging the GPU.
+ */
+void puro_set_wait_timeout_ns(uint64_t ns);
+
+/* Human-readable name of a status code (static string). */
+const char *puro_status_string(puro_status_t s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PURO_FP8_H */

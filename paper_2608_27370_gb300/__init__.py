@@ -1,0 +1,285 @@
+"""GB300 (sm_103a) FP8 linear-layer training path of Puro-2B.
+
+Python binding of ``libpuro_fp8.so`` (C ABI in ``include/puro_fp8.h``).
+Every function here is argument marshalling only: it checks that the torch
+tensors it is handed are CUDA, contiguous and of the right dtype, and passes
+their device pointers, the sizes and the current CUDA stream to the library
+entry point of the same name.  All arithmetic runs in the library's CUDA
+kernels.  There is no fallback: if the library is missing, every call raises
+:class:`PuroError`.
+
+The method (paper section "FP8 Mixed-Precision Training"; appendix
+"Production Training Details", paragraph "FP8 implementation pipeline"):
+E4M3 operands for all three GEMMs of every linear layer, power-of-two scales
+computed online for 1x128 groups along the reduction dimension (activations
+and activation gradients) or 128x128 blocks (weights), FP32 accumulation and
+BF16 output.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import Optional
+
+import torch
+
+from . import _build
+
+E4M3, E5M2 = 0, 1
+SCALE_TENSOR, SCALE_BLOCK = 0, 1
+ROLE_ACT, ROLE_WEIGHT = 0, 1
+
+PURO_OK = 0
+PURO_ERR_INVALID_ARG = 1
+PURO_ERR_UNSUPPORTED = 2
+PURO_ERR_CUDA = 3
+PURO_ERR_TIMEOUT = 4
+
+LIB_PATH = _build.LIB
+HEADER_PATH = os.path.join(_build.INCLUDE, "puro_fp8.h")
+
+
+class PuroError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        self.status = status
+        names = {1: "PURO_ERR_INVALID_ARG", 2: "PURO_ERR_UNSUPPORTED", 3: "PURO_ERR_CUDA", 4: "PURO_ERR_TIMEOUT"}
+        super().__init__(f"{fn} returned {names.get(status, status)}")
+
+
+class puro_fp8_tensor_t(ctypes.Structure):
+    """Mirror of the C struct puro_fp8_tensor_t."""
+    _fields_ = [
+        ("data", ctypes.c_void_p),
+        ("scale", ctypes.c_void_p),
+        ("rows", ctypes.c_int64),
+        ("red", ctypes.c_int64),
+        ("fmt", ctypes.c_int32),
+        ("scaling", ctypes.c_int32),
+        ("role", ctypes.c_int32),
+        ("reserved", ctypes.c_int32),
+    ]
+
+
+_P = ctypes.c_void_p
+_I64 = ctypes.c_int64
+_I32 = ctypes.c_int32
+_SIGNATURES = {
+    "puro_fp8_amax": (_I32, [_P, _I64, _I64, _P, _P]),
+    "puro_fp8_quantize": (_I32, [_P, _I64, _I64, _I32, _I32, _I32, _P, _P, _P, _P, _P, _P]),
+    "puro_fp8_linear_fprop": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
+    "puro_fp8_linear_dgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
+    "puro_fp8_linear_wgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
+    "puro_fp8_workspace_size": (ctypes.c_size_t, [_I64, _I64, _I64]),
+    "puro_fp8_get_status": (_I32, [_P, _P, _P]),
+    "puro_bf16_linear_fprop": (_I32, [_P, _P, _P, _I64, _I64, _I64, _P, _P]),
+    "puro_bf16_linear_dgrad": (_I32, [_P, _P, _P, _I64, _I64, _I64, _P, _P]),
+    "puro_bf16_linear_wgrad": (_I32, [_P, _P, _P, _I64, _I64, _I64, _P, _P]),
+    "puro_set_wait_timeout_ns": (None, [ctypes.c_uint64]),
+    "puro_status_string": (ctypes.c_char_p, [_I32]),
+}
+
+_lib = None
+
+
+def load_library(path: Optional[str] = None):
+    """Load libpuro_fp8.so (built by ``__graft_entry__.build()``); raises if absent."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise RuntimeError(
+            f"libpuro_fp8.so not found at {p}: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = ctypes.CDLL(p)
+    for name, (res, args) in _SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    if path is None:
+        _lib = lib
+    return lib
+
+
+def _check(fn: str, status: int) -> None:
+    if status != PURO_OK:
+        raise PuroError(fn, status)
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, torch.cuda.Stream):
+        return stream.cuda_stream
+    return int(stream)
+
+
+def _ptr(t: Optional[torch.Tensor], dtype=None, name: str = "tensor") -> Optional[int]:
+    if t is None:
+        return None
+    if t.numel() == 0:
+        return t.data_ptr() or None
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype not in (dtype if isinstance(dtype, tuple) else (dtype,)):
+        raise ValueError(f"{name} has dtype {t.dtype}, expected {dtype}")
+    return t.data_ptr()
+
+
+# --------------------------------------------------------------------------
+# Entry points (same names as the C ABI)
+# --------------------------------------------------------------------------
+def puro_fp8_amax(x: torch.Tensor, amax_bits: torch.Tensor, stream=None) -> None:
+    rows, cols = (x.shape[0], x.shape[1]) if x.dim() == 2 else (1, x.numel())
+    st = load_library().puro_fp8_amax(_ptr(x, torch.bfloat16, "x"), rows, cols,
+                                      _ptr(amax_bits, (torch.int32, torch.uint32), "amax_bits"), _stream(stream))
+    _check("puro_fp8_amax", st)
+
+
+def puro_fp8_quantize(x: torch.Tensor, fmt: int, scaling: int, role: int, amax_bits: Optional[torch.Tensor],
+                      q: torch.Tensor, scale: torch.Tensor, q_t: Optional[torch.Tensor] = None,
+                      scale_t: Optional[torch.Tensor] = None, stream=None) -> None:
+    rows, cols = x.shape
+    u8 = torch.uint8
+    sdt = u8 if scaling == SCALE_BLOCK else torch.float32
+    st = load_library().puro_fp8_quantize(
+        _ptr(x, torch.bfloat16, "x"), rows, cols, fmt, scaling, role,
+        _ptr(amax_bits, (torch.int32, torch.uint32), "amax_bits"), _ptr(q, u8, "q"), _ptr(scale, sdt, "scale"),
+        _ptr(q_t, u8, "q_t"), _ptr(scale_t, sdt, "scale_t"), _stream(stream))
+    _check("puro_fp8_quantize", st)
+
+
+@dataclass
+class FP8Operand:
+    """A quantised GEMM operand: codes [rows, red] plus scales (torch tensors kept alive here)."""
+    data: torch.Tensor
+    scale: torch.Tensor
+    fmt: int = E4M3
+    scaling: int = SCALE_BLOCK
+    role: int = ROLE_ACT
+
+    @property
+    def rows(self) -> int:
+        return self.data.shape[0]
+
+    @property
+    def red(self) -> int:
+        return self.data.shape[1]
+
+    def as_c(self) -> puro_fp8_tensor_t:
+        return puro_fp8_tensor_t(_ptr(self.data, torch.uint8, "data"), _ptr(self.scale, None, "scale"),
+                                 self.data.shape[0], self.data.shape[1], self.fmt, self.scaling, self.role, 0)
+
+
+def _gemm(name: str, a: FP8Operand, b: FP8Operand, out: torch.Tensor, workspace, dev_status, stream) -> None:
+    ca, cb = a.as_c(), b.as_c()
+    ws_ptr = _ptr(workspace, None, "workspace")
+    ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    fn = getattr(load_library(), name)
+    st = fn(ctypes.byref(ca), ctypes.byref(cb), _ptr(out, torch.bfloat16, "out"), ws_ptr, ws_bytes,
+            _ptr(dev_status, torch.int32, "dev_status"), _stream(stream))
+    _check(name, st)
+
+
+def puro_fp8_linear_fprop(x: FP8Operand, w: FP8Operand, y: torch.Tensor, workspace=None, dev_status=None,
+                          stream=None) -> None:
+    """Y [M,N] = X [M,K] . W [N,K]^T."""
+    _gemm("puro_fp8_linear_fprop", x, w, y, workspace, dev_status, stream)
+
+
+def puro_fp8_linear_dgrad(dy: FP8Operand, w_t: FP8Operand, dx: torch.Tensor, workspace=None, dev_status=None,
+                          stream=None) -> None:
+    """dX [M,K] = dY [M,N] . W [N,K] (B operand = W^T [K,N])."""
+    _gemm("puro_fp8_linear_dgrad", dy, w_t, dx, workspace, dev_status, stream)
+
+
+def puro_fp8_linear_wgrad(dy_t: FP8Operand, x_t: FP8Operand, dw: torch.Tensor, workspace=None, dev_status=None,
+                          stream=None) -> None:
+    """dW [N,K] = dY^T [N,M] . X [M,K] (operands dY^T [N,M], X^T [K,M])."""
+    _gemm("puro_fp8_linear_wgrad", dy_t, x_t, dw, workspace, dev_status, stream)
+
+
+def puro_fp8_workspace_size(rows_out: int, cols_out: int, red: int) -> int:
+    return int(load_library().puro_fp8_workspace_size(rows_out, cols_out, red))
+
+
+def puro_fp8_get_status(dev_status: torch.Tensor, stream=None) -> int:
+    out = ctypes.c_int32(0)
+    st = load_library().puro_fp8_get_status(_ptr(dev_status, torch.int32, "dev_status"), ctypes.byref(out),
+                                            _stream(stream))
+    _check("puro_fp8_get_status", st)
+    return out.value
+
+
+def _bf16(name, a, b, out, M, N, K, dev_status, stream):
+    fn = getattr(load_library(), name)
+    st = fn(_ptr(a, torch.bfloat16, "a"), _ptr(b, torch.bfloat16, "b"), _ptr(out, torch.bfloat16, "out"), M, N, K,
+            _ptr(dev_status, torch.int32, "dev_status"), _stream(stream))
+    _check(name, st)
+
+
+def puro_bf16_linear_fprop(x, w, y, M, N, K, dev_status=None, stream=None) -> None:
+    _bf16("puro_bf16_linear_fprop", x, w, y, M, N, K, dev_status, stream)
+
+
+def puro_bf16_linear_dgrad(dy, w_t, dx, M, N, K, dev_status=None, stream=None) -> None:
+    _bf16("puro_bf16_linear_dgrad", dy, w_t, dx, M, N, K, dev_status, stream)
+
+
+def puro_bf16_linear_wgrad(dy_t, x_t, dw, M, N, K, dev_status=None, stream=None) -> None:
+    _bf16("puro_bf16_linear_wgrad", dy_t, x_t, dw, M, N, K, dev_status, stream)
+
+
+def puro_set_wait_timeout_ns(ns: int) -> None:
+    load_library().puro_set_wait_timeout_ns(int(ns))
+
+
+# --------------------------------------------------------------------------
+# Allocation helpers (torch allocates; the library computes)
+# --------------------------------------------------------------------------
+@dataclass
+class Quantized:
+    """Both copies produced by one quantise call."""
+    rowwise: FP8Operand
+    colwise: Optional[FP8Operand]
+    amax: Optional[torch.Tensor] = None
+
+
+def empty_scales(rows: int, red: int, scaling: int, role: int, device) -> torch.Tensor:
+    if scaling == SCALE_TENSOR:
+        return torch.empty(1, dtype=torch.float32, device=device)
+    if role == ROLE_ACT:
+        return torch.empty((red // 128, rows), dtype=torch.uint8, device=device)
+    return torch.empty((rows // 128, red // 128), dtype=torch.uint8, device=device)
+
+
+def quantize(x: torch.Tensor, fmt: int = E4M3, scaling: int = SCALE_BLOCK, role: int = ROLE_ACT,
+             transpose: bool = True, out: Optional[Quantized] = None, stream=None) -> Quantized:
+    """Quantise x [rows, cols] (bf16) into a rowwise operand [rows, cols] and,
+    if ``transpose``, a columnwise operand [cols, rows]; per-tensor mode runs
+    the amax kernel first."""
+    rows, cols = x.shape
+    dev = x.device
+    if out is None:
+        q = torch.empty((rows, cols), dtype=torch.uint8, device=dev)
+        s = empty_scales(rows, cols, scaling, role, dev)
+        colwise = None
+        if transpose:
+            colwise = FP8Operand(torch.empty((cols, rows), dtype=torch.uint8, device=dev),
+                                 empty_scales(cols, rows, scaling, role, dev), fmt, scaling, role)
+        amax = torch.zeros(1, dtype=torch.int32, device=dev) if scaling == SCALE_TENSOR else None
+        out = Quantized(FP8Operand(q, s, fmt, scaling, role), colwise, amax)
+    if scaling == SCALE_TENSOR:
+        puro_fp8_amax(x, out.amax, stream)
+    puro_fp8_quantize(x, fmt, scaling, role, out.amax if scaling == SCALE_TENSOR else None, out.rowwise.data,
+                      out.rowwise.scale, out.colwise.data if out.colwise else None,
+                      out.colwise.scale if out.colwise else None, stream)
+    return out
+
+
+__all__ = [n for n in dir() if n.startswith("puro_")] + [
+    "E4M3", "E5M2", "SCALE_TENSOR", "SCALE_BLOCK", "ROLE_ACT", "ROLE_WEIGHT", "PuroError", "FP8Operand",
+    "Quantized", "quantize", "load_library", "empty_scales", "LIB_PATH", "HEADER_PATH",
+]

@@ -1,0 +1,292 @@
+// api.cu -- the C ABI declared in include/puro_fp8.h: argument validation
+// (entirely on the host, before anything is enqueued), TMA descriptor
+// encoding and kernel launch.  See the header for the contract of every
+// entry point.
+#include <atomic>
+#include <mutex>
+
+#include "internal.h"
+#include "puro_fp8.h"
+
+#define PURO_API extern "C" __attribute__((visibility("default")))
+
+namespace puro {
+namespace {
+
+std::atomic<uint64_t> g_wait_timeout_ns{2000000000ull};  // 2 s
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *,
+                                   CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                   CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// 2-D tensor map over a row-major [outer, inner] matrix.
+bool make_map(CUtensorMap *m, CUtensorMapDataType dt, const void *base, uint64_t inner, uint64_t outer,
+              uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle sw) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {inner, outer};
+    const cuuint64_t strides[1] = {row_bytes};
+    const cuuint32_t box[2] = {box_inner, box_outer};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(m, dt, 2, const_cast<void *>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int sm_count() {
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (dev >= 0 && dev < 64 && cache[dev]) return cache[dev];
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    if (dev >= 0 && dev < 64) cache[dev] = n;
+    return n;
+}
+
+puro_status_t cuda_status(cudaError_t e) { return e == cudaSuccess ? PURO_OK : PURO_ERR_CUDA; }
+
+bool valid_fmt(int32_t f) { return f == PURO_E4M3 || f == PURO_E5M2; }
+
+// Shape/pointer checks shared by the FP8 GEMM entry points.
+puro_status_t check_operand(const puro_fp8_tensor_t *t, bool must_be_act) {
+    if (!t || !t->data || !t->scale) return PURO_ERR_INVALID_ARG;
+    if (!aligned16(t->data) || !aligned16(t->scale)) return PURO_ERR_INVALID_ARG;
+    if (t->rows < 0 || t->red < 0 || !valid_fmt(t->fmt) || t->reserved != 0) return PURO_ERR_INVALID_ARG;
+    if (t->rows > INT32_MAX || t->red > INT32_MAX) return PURO_ERR_UNSUPPORTED;
+    if (t->scaling == PURO_SCALE_BLOCK) {
+        if (t->role != PURO_ROLE_ACT && t->role != PURO_ROLE_WEIGHT) return PURO_ERR_INVALID_ARG;
+        if (must_be_act && t->role != PURO_ROLE_ACT) return PURO_ERR_INVALID_ARG;
+        if (t->rows % 128 || t->red % 128) return PURO_ERR_INVALID_ARG;
+    } else if (t->scaling == PURO_SCALE_TENSOR) {
+        if (t->rows % 16 || t->red % 16) return PURO_ERR_INVALID_ARG;
+    } else {
+        return PURO_ERR_INVALID_ARG;
+    }
+    return PURO_OK;
+}
+
+// D[M,N] = A[M,K] * B[N,K]^T over quantised operands.
+puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, void *d, int32_t *dev_status,
+                       void *stream) {
+    puro_status_t st = check_operand(a, /*must_be_act=*/true);
+    if (st != PURO_OK) return st;
+    st = check_operand(b, /*must_be_act=*/false);
+    if (st != PURO_OK) return st;
+    if (a->red != b->red || a->scaling != b->scaling) return PURO_ERR_INVALID_ARG;
+    if (!d || !aligned16(d)) return PURO_ERR_INVALID_ARG;
+    const int64_t M = a->rows, N = b->rows, K = a->red;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (M == 0 || N == 0) return PURO_OK;
+    if (K == 0) return cuda_status(cudaMemsetAsync(d, 0, static_cast<size_t>(M * N) * 2, s));
+    const bool block = a->scaling == PURO_SCALE_BLOCK;
+    if (block && b->role == PURO_ROLE_WEIGHT && K / 128 > 256) return PURO_ERR_UNSUPPORTED;
+
+    CUtensorMap tm_a, tm_b, tm_d;
+    if (!make_map(&tm_a, CU_TENSOR_MAP_DATA_TYPE_UINT8, a->data, K, M, K, 128, kGemmBM,
+                  CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&tm_b, CU_TENSOR_MAP_DATA_TYPE_UINT8, b->data, K, N, K, 128, kGemmBN,
+                  CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&tm_d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B))
+        return PURO_ERR_CUDA;
+    GemmArgs g{};
+    g.kind = block ? kGemmFP8Block : kGemmFP8Tensor;
+    g.a_fmt = a->fmt;
+    g.b_fmt = b->fmt;
+    g.M = M;
+    g.N = N;
+    g.K = K;
+    if (block) {
+        g.sfa = static_cast<const uint8_t *>(a->scale);
+        g.sfb = static_cast<const uint8_t *>(b->scale);
+        g.sfb_blk = b->role == PURO_ROLE_WEIGHT ? 1 : 0;
+    } else {
+        g.sia = static_cast<const float *>(a->scale);
+        g.sib = static_cast<const float *>(b->scale);
+    }
+    g.status = dev_status;
+    g.wait_timeout_ns = g_wait_timeout_ns.load();
+    g.num_sms = sm_count();
+    if (g.num_sms <= 0) return PURO_ERR_CUDA;
+    return cuda_status(launch_gemm(g, tm_a, tm_b, tm_d, s));
+}
+
+puro_status_t bf16_gemm(const void *a, const void *b, void *d, int64_t M, int64_t N, int64_t K,
+                        int32_t *dev_status, void *stream) {
+    if (!a || !b || !d || !aligned16(a) || !aligned16(b) || !aligned16(d)) return PURO_ERR_INVALID_ARG;
+    if (M < 0 || N < 0 || K < 0 || M % 8 || N % 8 || K % 8) return PURO_ERR_INVALID_ARG;
+    if (M > INT32_MAX || N > INT32_MAX || K > INT32_MAX) return PURO_ERR_UNSUPPORTED;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (M == 0 || N == 0) return PURO_OK;
+    if (K == 0) return cuda_status(cudaMemsetAsync(d, 0, static_cast<size_t>(M * N) * 2, s));
+    CUtensorMap tm_a, tm_b, tm_d;
+    if (!make_map(&tm_a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a, K, M, K * 2, 64, kGemmBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, b, K, N, K * 2, 64, kGemmBN, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&tm_d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B))
+        return PURO_ERR_CUDA;
+    GemmArgs g{};
+    g.kind = kGemmBF16;
+    g.M = M;
+    g.N = N;
+    g.K = K;
+    g.status = dev_status;
+    g.wait_timeout_ns = g_wait_timeout_ns.load();
+    g.num_sms = sm_count();
+    if (g.num_sms <= 0) return PURO_ERR_CUDA;
+    return cuda_status(launch_gemm(g, tm_a, tm_b, tm_d, s));
+}
+
+}  // namespace
+}  // namespace puro
+
+using namespace puro;
+
+PURO_API puro_status_t puro_fp8_amax(const void *x, int64_t rows, int64_t cols, uint32_t *amax_bits, void *stream) {
+    if (!amax_bits || rows < 0 || cols < 0) return PURO_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(amax_bits) & 3u) != 0) return PURO_ERR_INVALID_ARG;
+    const int64_t n = rows * cols;
+    if (n > 0 && (!x || !aligned16(x))) return PURO_ERR_INVALID_ARG;
+    return cuda_status(launch_amax(static_cast<const uint16_t *>(x), n, amax_bits, static_cast<cudaStream_t>(stream)));
+}
+
+PURO_API puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t cols, int32_t fmt, int32_t scaling,
+                                         int32_t role, const uint32_t *amax_bits, uint8_t *q, void *scale,
+                                         uint8_t *q_t, void *scale_t, void *stream) {
+    if (!valid_fmt(fmt) || rows < 0 || cols < 0) return PURO_ERR_INVALID_ARG;
+    if ((q_t == nullptr) != (scale_t == nullptr) && scaling == PURO_SCALE_BLOCK) return PURO_ERR_INVALID_ARG;
+    const bool has_t = q_t != nullptr;
+    QuantArgs a{};
+    a.fmt = fmt;
+    a.rows = rows;
+    a.cols = cols;
+    a.has_t = has_t;
+    if (scaling == PURO_SCALE_BLOCK) {
+        if (role != PURO_ROLE_ACT && role != PURO_ROLE_WEIGHT) return PURO_ERR_INVALID_ARG;
+        if (amax_bits != nullptr) return PURO_ERR_INVALID_ARG;
+        if (rows % 128 || cols % 128) return PURO_ERR_INVALID_ARG;
+        a.kind = role == PURO_ROLE_ACT ? kQuantBlockAct : kQuantBlockWeight;
+        a.scale_u8 = static_cast<uint8_t *>(scale);
+        a.scale_t_u8 = static_cast<uint8_t *>(scale_t);
+    } else if (scaling == PURO_SCALE_TENSOR) {
+        if (!amax_bits || (reinterpret_cast<uintptr_t>(amax_bits) & 3u)) return PURO_ERR_INVALID_ARG;
+        if (cols % 16 || (has_t && rows % 16)) return PURO_ERR_INVALID_ARG;
+        a.kind = kQuantTensor;
+        a.scale_f = static_cast<float *>(scale);
+        a.scale_t_f = static_cast<float *>(scale_t);
+        if ((reinterpret_cast<uintptr_t>(scale) & 3u) || (reinterpret_cast<uintptr_t>(scale_t) & 3u))
+            return PURO_ERR_INVALID_ARG;
+    } else {
+        return PURO_ERR_INVALID_ARG;
+    }
+    const bool empty = rows == 0 || cols == 0;
+    // Empty tensors write no codes (their buffers may be NULL); per-tensor
+    // mode still writes scale_inv.
+    if (!aligned16(q) || !aligned16(scale) || !aligned16(q_t) || !aligned16(scale_t)) return PURO_ERR_INVALID_ARG;
+    if (!empty && (!q || !scale)) return PURO_ERR_INVALID_ARG;
+    if (empty && scaling == PURO_SCALE_TENSOR && !scale) return PURO_ERR_INVALID_ARG;
+    if (rows > INT32_MAX || cols > INT32_MAX) return PURO_ERR_UNSUPPORTED;
+    if (!empty && (!x || !aligned16(x))) return PURO_ERR_INVALID_ARG;
+    a.amax = amax_bits;
+    if (empty) {
+        if (scaling == PURO_SCALE_TENSOR)  // empty tensor: amax is 0, scale_inv is 1
+            return cuda_status(launch_tensor_scale_only(a, static_cast<cudaStream_t>(stream)));
+        return PURO_OK;
+    }
+    a.x = static_cast<const uint16_t *>(x);
+    CUtensorMap tm_q, tm_qt;
+    if (!make_map(&tm_q, CU_TENSOR_MAP_DATA_TYPE_UINT8, q, cols, rows, cols, 128, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
+        return PURO_ERR_CUDA;
+    if (has_t) {
+        if (!make_map(&tm_qt, CU_TENSOR_MAP_DATA_TYPE_UINT8, q_t, rows, cols, rows, 128, 128,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
+            return PURO_ERR_CUDA;
+    } else {
+        tm_qt = tm_q;
+    }
+    return cuda_status(launch_quantize(a, tm_q, tm_qt, static_cast<cudaStream_t>(stream)));
+}
+
+PURO_API puro_status_t puro_fp8_linear_fprop(const puro_fp8_tensor_t *x, const puro_fp8_tensor_t *w, void *y,
+                                             void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                                             void *stream) {
+    (void)workspace;
+    (void)workspace_bytes;
+    return fp8_gemm(x, w, y, dev_status, stream);
+}
+
+PURO_API puro_status_t puro_fp8_linear_dgrad(const puro_fp8_tensor_t *dy, const puro_fp8_tensor_t *w_t, void *dx,
+                                             void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                                             void *stream) {
+    (void)workspace;
+    (void)workspace_bytes;
+    return fp8_gemm(dy, w_t, dx, dev_status, stream);
+}
+
+PURO_API puro_status_t puro_fp8_linear_wgrad(const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t, void *dw,
+                                             void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                                             void *stream) {
+    (void)workspace;
+    (void)workspace_bytes;
+    return fp8_gemm(dy_t, x_t, dw, dev_status, stream);
+}
+
+PURO_API size_t puro_fp8_workspace_size(int64_t rows_out, int64_t cols_out, int64_t red) {
+    (void)rows_out;
+    (void)cols_out;
+    (void)red;
+    return 0;
+}
+
+PURO_API puro_status_t puro_fp8_get_status(const int32_t *dev_status, int32_t *host_out, void *stream) {
+    if (!dev_status || !host_out || (reinterpret_cast<uintptr_t>(dev_status) & 3u)) return PURO_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemcpyAsync(host_out, dev_status, sizeof(int32_t), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    return cuda_status(e);
+}
+
+PURO_API puro_status_t puro_bf16_linear_fprop(const void *x, const void *w, void *y, int64_t M, int64_t N,
+                                              int64_t K, int32_t *dev_status, void *stream) {
+    return bf16_gemm(x, w, y, M, N, K, dev_status, stream);
+}
+
+PURO_API puro_status_t puro_bf16_linear_dgrad(const void *dy, const void *w_t, void *dx, int64_t M, int64_t N,
+                                              int64_t K, int32_t *dev_status, void *stream) {
+    // dX [M, K] = dY [M, N] * (W^T [K, N])^T
+    return bf16_gemm(dy, w_t, dx, M, K, N, dev_status, stream);
+}
+
+PURO_API puro_status_t puro_bf16_linear_wgrad(const void *dy_t, const void *x_t, void *dw, int64_t M, int64_t N,
+                                              int64_t K, int32_t *dev_status, void *stream) {
+    // dW [N, K] = dY^T [N, M] * (X^T [K, M])^T
+    return bf16_gemm(dy_t, x_t, dw, N, K, M, dev_status, stream);
+}
+
+PURO_API void puro_set_wait_timeout_ns(uint64_t ns) { g_wait_timeout_ns.store(ns); }
+
+PURO_API const char *puro_status_string(puro_status_t s) {
+    switch (s) {
+        case PURO_OK: return "PURO_OK";
+        case PURO_ERR_INVALID_ARG: return "PURO_ERR_INVALID_ARG";
+        case PURO_ERR_UNSUPPORTED: return "PURO_ERR_UNSUPPORTED";
+        case PURO_ERR_CUDA: return "PURO_ERR_CUDA";
+        case PURO_ERR_TIMEOUT: return "PURO_ERR_TIMEOUT";
+        default: return "PURO_ERR_UNKNOWN";
+    }
+}

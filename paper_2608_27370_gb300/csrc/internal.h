@@ -1,0 +1,75 @@
+// internal.h -- declarations shared by the CUDA translation units of the
+// FP8 linear-path library (not part of the public C ABI).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cstddef>
+#include <cstdint>
+
+namespace puro {
+
+// How a quantiser groups values (section "FP8 Mixed-Precision Training").
+enum QuantKind : int {
+    kQuantBlockAct = 0,     // 1x128 groups along cols (q) and along rows (q_t)
+    kQuantBlockWeight = 1,  // 128x128 blocks; q_t = transposed codes
+    kQuantTensor = 2,       // one scale for the whole tensor
+};
+
+struct QuantArgs {
+    const uint16_t *x;        // bf16 [rows, cols]
+    int64_t rows, cols;
+    int fmt;                  // 0 = E4M3, 1 = E5M2
+    QuantKind kind;
+    const uint32_t *amax;     // kQuantTensor only
+    uint8_t *scale_u8;        // block scales of q
+    uint8_t *scale_t_u8;      // block scales of q_t
+    float *scale_f;           // tensor scale_inv for q
+    float *scale_t_f;         // tensor scale_inv for q_t (may be null)
+    bool has_t;
+};
+
+cudaError_t launch_amax(const uint16_t *x, int64_t n, uint32_t *amax, cudaStream_t s);
+
+// tm_q: u8 [rows, cols], box {128, 128}, no swizzle.
+// tm_qt: u8 [cols, rows], box {128, 128}, 128-byte swizzle (only if has_t).
+cudaError_t launch_quantize(const QuantArgs &a, const CUtensorMap &tm_q, const CUtensorMap &tm_qt,
+                            cudaStream_t s);
+
+// Writes only the per-tensor scale_inv (used for empty tensors).
+cudaError_t launch_tensor_scale_only(const QuantArgs &a, cudaStream_t s);
+
+// Operand kinds of the tensor-core GEMM D[M,N] = A[M,K] * B[N,K]^T.
+enum GemmKind : int {
+    kGemmBF16 = 0,       // kind::f16, bf16 operands
+    kGemmFP8Tensor = 1,  // kind::f8f6f4, per-tensor scale_inv product in the epilogue
+    kGemmFP8Block = 2,   // kind::mxf8f6f4 with E8M0 group scales
+};
+
+struct GemmArgs {
+    GemmKind kind;
+    int a_fmt, b_fmt;            // FP8 formats (0 = E4M3, 1 = E5M2)
+    int64_t M, N, K;
+    // kGemmFP8Block: A scales are 1x128 groups, group-major [K/128][M].
+    const uint8_t *sfa;
+    // B scales: group-major [K/128][N] (sfb_blk = 0) or 128x128 grid
+    // [N/128][K/128] (sfb_blk = 1).
+    const uint8_t *sfb;
+    int sfb_blk;
+    // kGemmFP8Tensor: dequantisation factors of A and B.
+    const float *sia, *sib;
+    int32_t *status;             // optional device status word
+    uint64_t wait_timeout_ns;
+    int num_sms;
+};
+
+// tm_a: A [M, K], tm_b: B [N, K] (128-byte swizzle, box {128 bytes, rows}),
+// tm_d: D [M, N] bf16 (128-byte swizzle, box {64, 32}).
+cudaError_t launch_gemm(const GemmArgs &g, const CUtensorMap &tm_a, const CUtensorMap &tm_b,
+                        const CUtensorMap &tm_d, cudaStream_t s);
+
+// Tile shape of the GEMM kernel (rows of A per CTA tile, rows of B).
+constexpr int kGemmBM = 128;
+constexpr int kGemmBN = 256;
+
+}  // namespace puro

@@ -1,0 +1,169 @@
+"""Helpers shared by the GPU parity tests: run one linear layer through the
+C ABI, rebuild the oracle's view of the same bytes, compare.
+
+The oracle never sees a byte produced by the CUDA path: it quantises the
+same BF16 inputs itself and forms its own fp64 products.  Layout
+conversions between the oracle's natural scale grids and the library's
+group-major ones are plain transposes.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle as O
+import paper_2608_27370_gb300 as P
+
+
+def bits(t: torch.Tensor) -> np.ndarray:
+    """bf16 tensor -> uint16 numpy array of its bit patterns (host copy)."""
+    return t.detach().contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+
+
+def host(t: torch.Tensor) -> np.ndarray:
+    return t.detach().cpu().numpy()
+
+
+def bf16_values(t: torch.Tensor) -> np.ndarray:
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+# --------------------------------------------------------------------------
+# Running the path
+# --------------------------------------------------------------------------
+def run_linear(x, w, dy, scaling=P.SCALE_BLOCK, fmt_x=P.E4M3, fmt_w=P.E4M3, fmt_g=P.E4M3):
+    """Quantise X, W, dY (rowwise + transposed copies) and run the three GEMMs."""
+    M, K = x.shape
+    N = w.shape[0]
+    dev = x.device
+    xq = P.quantize(x, fmt_x, scaling, P.ROLE_ACT)
+    wq = P.quantize(w, fmt_w, scaling, P.ROLE_WEIGHT)
+    dyq = P.quantize(dy, fmt_g, scaling, P.ROLE_ACT)
+    y = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
+    dx = torch.empty((M, K), dtype=torch.bfloat16, device=dev)
+    dw = torch.empty((N, K), dtype=torch.bfloat16, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    P.puro_fp8_linear_fprop(xq.rowwise, wq.rowwise, y, dev_status=status)
+    P.puro_fp8_linear_dgrad(dyq.rowwise, wq.colwise, dx, dev_status=status)
+    P.puro_fp8_linear_wgrad(dyq.colwise, xq.colwise, dw, dev_status=status)
+    torch.cuda.synchronize()
+    assert P.puro_fp8_get_status(status) == 0
+    return dict(xq=xq, wq=wq, dyq=dyq, y=y, dx=dx, dw=dw)
+
+
+# --------------------------------------------------------------------------
+# Comparisons
+# --------------------------------------------------------------------------
+def assert_close(gpu: torch.Tensor, ref: np.ndarray, what: str):
+    g = bf16_values(gpu)
+    ok, ratio = O.within_tolerance(g, ref)
+    if not ok:
+        rms = float(np.sqrt(np.mean(ref * ref)))
+        bound = 2.0 ** -7 * np.abs(ref) + 1e-3 * rms
+        bad = np.argwhere(np.abs(g - ref) > bound)
+        i = tuple(bad[0])
+        raise AssertionError(f"{what}: {len(bad)} of {ref.size} outside tolerance (worst ratio {ratio:.3g}); "
+                             f"first at {i}: gpu {g[i]!r} ref {ref[i]!r}")
+
+
+def assert_bytes(gpu: torch.Tensor, ref: np.ndarray, what: str):
+    g = host(gpu)
+    assert g.shape == ref.shape, (what, g.shape, ref.shape)
+    if not np.array_equal(g, ref):
+        bad = np.argwhere(g != ref)
+        i = tuple(bad[0])
+        raise AssertionError(f"{what}: {len(bad)} of {ref.size} bytes differ; first at {i}: "
+                             f"gpu {g[i]:#04x} ref {ref[i]:#04x}")
+
+
+def check_block_act_quant(x: torch.Tensor, q: P.Quantized, fmt: int, rows=None, cols=None):
+    """Bit-exact check of a 1x128 quantisation (rowwise + transposed copy).
+    rows/cols: optional index subsets (full-size sampling)."""
+    xb = bits(x if rows is None else x[rows])
+    q_ref, s_ref = O.quantize_rows_1x128(xb, fmt)
+    qr = q.rowwise.data if rows is None else q.rowwise.data[rows]
+    sr = q.rowwise.scale if rows is None else q.rowwise.scale[:, rows]
+    assert_bytes(qr, q_ref, "rowwise codes")
+    assert_bytes(sr, np.ascontiguousarray(s_ref.T), "rowwise scales")
+    if q.colwise is None:
+        return
+    xc = bits(x if cols is None else x[:, cols])
+    qt_ref, st_ref = O.quantize_cols_128x1(xc, fmt)
+    qc = q.colwise.data if cols is None else q.colwise.data[cols]
+    sc = q.colwise.scale if cols is None else q.colwise.scale[:, cols]
+    assert_bytes(qc, qt_ref, "transposed codes")
+    assert_bytes(sc, np.ascontiguousarray(st_ref.T), "transposed scales")
+
+
+def check_block_weight_quant(w: torch.Tensor, q: P.Quantized, fmt: int):
+    q_ref, s_ref = O.quantize_blocks_128x128(bits(w), fmt)
+    assert_bytes(q.rowwise.data, q_ref, "weight codes")
+    assert_bytes(q.rowwise.scale, s_ref, "weight block scales")
+    if q.colwise is not None:
+        assert_bytes(q.colwise.data, np.ascontiguousarray(q_ref.T), "transposed weight codes")
+        assert_bytes(q.colwise.scale, np.ascontiguousarray(s_ref.T), "transposed weight scales")
+
+
+def check_tensor_quant(x: torch.Tensor, q: P.Quantized, fmt: int):
+    amax, q_ref, si_ref = O.quantize_tensor(bits(x), fmt)
+    got_amax = int(host(q.amax)[0]) & 0xFFFF
+    assert got_amax == amax, f"amax {got_amax:#06x} != {amax:#06x}"
+    assert_bytes(q.rowwise.data, q_ref, "tensor-scaled codes")
+    got_si = host(q.rowwise.scale)[0]
+    assert np.float32(got_si).tobytes() == np.float32(si_ref).tobytes(), (got_si, si_ref)
+    if q.colwise is not None:
+        assert_bytes(q.colwise.data, np.ascontiguousarray(q_ref.T), "transposed tensor-scaled codes")
+        assert np.float32(host(q.colwise.scale)[0]).tobytes() == np.float32(si_ref).tobytes()
+
+
+def oracle_linear(x, w, dy, scaling, fmt_x=P.E4M3, fmt_w=P.E4M3, fmt_g=P.E4M3, nthreads=8):
+    xb, wb, dyb = bits(x), bits(w), bits(dy)
+    if scaling == P.SCALE_BLOCK:
+        return O.linear_block(xb, wb, dyb, fmt_x, fmt_w, fmt_g, nthreads)
+    return O.linear_tensor(xb, wb, dyb, fmt_x, fmt_w, fmt_g, nthreads)
+
+
+# --------------------------------------------------------------------------
+# Full-size sampling (blockwise recipe)
+# --------------------------------------------------------------------------
+def sample_index(n: int, k_rand: int, rng: np.random.Generator) -> np.ndarray:
+    """First 128, last 128 and k_rand random indices of range(n), sorted, unique."""
+    edge = min(128, n)
+    idx = np.concatenate([np.arange(edge), np.arange(n - edge, n), rng.choice(n, size=min(k_rand, n), replace=False)])
+    return np.unique(idx)
+
+
+def check_linear_sampled(x, w, dy, out, rng, k_rand=64, fmt=P.E4M3, nthreads=16):
+    """Blockwise recipe at full size: quantised bytes on sampled rows/columns,
+    GEMM outputs on the cross product of sampled rows and columns (which
+    contains the four corner 128x128 tiles)."""
+    M, K = x.shape
+    N = w.shape[0]
+    Ms = sample_index(M, k_rand, rng)
+    Ns = sample_index(N, k_rand, rng)
+    Ks = sample_index(K, k_rand, rng)
+    Ms_t, Ns_t, Ks_t = (torch.from_numpy(a).to(x.device) for a in (Ms, Ns, Ks))
+
+    # quantised operands: X rows Ms / columns Ks, dY rows Ms / columns Ns, all of W
+    check_block_act_quant(x, out["xq"], fmt, rows=Ms_t, cols=Ks_t)
+    check_block_act_quant(dy, out["dyq"], fmt, rows=Ms_t, cols=Ns_t)
+    check_block_weight_quant(w, out["wq"], fmt)
+
+    # oracle operands for the sampled products
+    xr_q, xr_s = O.quantize_rows_1x128(bits(x[Ms_t]), fmt)            # X rows (groups along K)
+    X_rows = O.dequant_rows_1x128(xr_q, xr_s, fmt)
+    dyr_q, dyr_s = O.quantize_rows_1x128(bits(dy[Ms_t]), fmt)         # dY rows (groups along N)
+    dY_rows = O.dequant_rows_1x128(dyr_q, dyr_s, fmt)
+    wq, ws = O.quantize_blocks_128x128(bits(w), fmt)                  # W blocks
+    W = O.dequant_blocks_128x128(wq, ws, fmt)
+    xc_q, xc_s = O.quantize_cols_128x1(bits(x[:, Ks_t]), fmt)         # X columns (groups along M)
+    Xt_rows = O.dequant_rows_1x128(xc_q, xc_s, fmt)
+    dyc_q, dyc_s = O.quantize_cols_128x1(bits(dy[:, Ns_t]), fmt)      # dY columns (groups along M)
+    dYt_rows = O.dequant_rows_1x128(dyc_q, dyc_s, fmt)
+
+    y_ref = O.gemm_tn(X_rows, W[Ns], nthreads)                         # Y[Ms, Ns]
+    dx_ref = O.gemm_tn(dY_rows, np.ascontiguousarray(W.T[Ks]), nthreads)  # dX[Ms, Ks]
+    dw_ref = O.gemm_tn(dYt_rows, Xt_rows, nthreads)                    # dW[Ns, Ks]
+    assert_close(out["y"][Ms_t][:, Ns_t], y_ref, "fprop (sampled)")
+    assert_close(out["dx"][Ms_t][:, Ks_t], dx_ref, "dgrad (sampled)")
+    assert_close(out["dw"][Ns_t][:, Ks_t], dw_ref, "wgrad (sampled)")

@@ -1,0 +1,117 @@
+"""GPU parity of the three GEMMs of a linear layer (Fprop, Dgrad, Wgrad)
+against the oracle's fp64 products, element by element, within
+|gpu - ref| <= 2^-7 |ref| + 1e-3 rms(ref).
+
+Shapes span several output tiles (128 x 256) with ragged last tiles; the
+per-tensor and BF16 cases also have ragged reduction tails.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import paper_2608_27370_gb300 as P
+from paper_2608_27370_gb300 import workloads as W
+from _parity import assert_close, bits, host, oracle_linear, run_linear
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    P.load_library()
+
+
+def _inputs(M, N, K, seed, t3=False):
+    x = (W.student_t3_f32((M, K), DEV, seed) if t3 else W.normal_f32((M, K), 1.0, DEV, seed)).to(torch.bfloat16)
+    w = W.normal_bf16((N, K), 0.02, DEV, seed + 1)
+    dy = W.normal_bf16((M, N), 1e-3, DEV, seed + 2)
+    return x, w, dy
+
+
+@pytest.mark.parametrize("M,N,K", [(128, 128, 128), (384, 640, 384), (256, 1536, 1536), (512, 256, 1024)])
+def test_block_linear(M, N, K):
+    x, w, dy = _inputs(M, N, K, 1000 + M + N + K, t3=True)
+    out = run_linear(x, w, dy, P.SCALE_BLOCK)
+    ref = oracle_linear(x, w, dy, P.SCALE_BLOCK)
+    assert_close(out["y"], ref["y"], "fprop")
+    assert_close(out["dx"], ref["dx"], "dgrad")
+    assert_close(out["dw"], ref["dw"], "wgrad")
+
+
+@pytest.mark.parametrize("fmts", [(P.E4M3, P.E4M3, P.E5M2), (P.E5M2, P.E5M2, P.E5M2)])
+def test_block_linear_e5m2(fmts):
+    M, N, K = 256, 384, 256
+    x, w, dy = _inputs(M, N, K, 77)
+    out = run_linear(x, w, dy, P.SCALE_BLOCK, *fmts)
+    ref = oracle_linear(x, w, dy, P.SCALE_BLOCK, *fmts)
+    for k in ("y", "dx", "dw"):
+        assert_close(out[k], ref[k], k)
+
+
+@pytest.mark.parametrize("M,N,K", [(256, 1536, 1536), (272, 400, 208), (16, 16, 16), (144, 528, 272)])
+def test_tensor_linear(M, N, K):
+    x, w, dy = _inputs(M, N, K, 2000 + M + N + K)
+    out = run_linear(x, w, dy, P.SCALE_TENSOR)
+    ref = oracle_linear(x, w, dy, P.SCALE_TENSOR)
+    assert_close(out["y"], ref["y"], "fprop")
+    assert_close(out["dx"], ref["dx"], "dgrad")
+    assert_close(out["dw"], ref["dw"], "wgrad")
+
+
+@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (264, 392, 200), (512, 1536, 1536)])
+def test_bf16_linear(M, N, K):
+    x, w, dy = _inputs(M, N, K, 3000 + M)
+    y = torch.empty((M, N), dtype=torch.bfloat16, device=DEV)
+    dx = torch.empty((M, K), dtype=torch.bfloat16, device=DEV)
+    dw = torch.empty((N, K), dtype=torch.bfloat16, device=DEV)
+    P.puro_bf16_linear_fprop(x, w, y, M, N, K)
+    P.puro_bf16_linear_dgrad(dy, w.t().contiguous(), dx, M, N, K)
+    P.puro_bf16_linear_wgrad(dy.t().contiguous(), x.t().contiguous(), dw, M, N, K)
+    torch.cuda.synchronize()
+    X, Wd, dY = (O.bf16_to_double(bits(t)) for t in (x, w, dy))
+    assert_close(y, O.gemm_tn(X, Wd, 8), "bf16 fprop")
+    assert_close(dx, O.gemm_tn(dY, np.ascontiguousarray(Wd.T), 8), "bf16 dgrad")
+    assert_close(dw, O.gemm_tn(np.ascontiguousarray(dY.T), np.ascontiguousarray(X.T), 8), "bf16 wgrad")
+
+
+def test_fprop_of_transposed_weight_equals_dgrad_bitwise():
+    """Dgrad is Fprop of the linear whose weight is W^T: same kernel, same
+    operand bytes, so the outputs are identical bit for bit."""
+    M, N, K = 256, 512, 384
+    x, w, dy = _inputs(M, N, K, 55)
+    out = run_linear(x, w, dy, P.SCALE_BLOCK)
+    y2 = torch.empty((M, K), dtype=torch.bfloat16, device=DEV)
+    P.puro_fp8_linear_fprop(out["dyq"].rowwise, out["wq"].colwise, y2)
+    torch.cuda.synchronize()
+    assert torch.equal(y2.view(torch.int16), out["dx"].view(torch.int16))
+
+
+def test_zero_reduction_writes_zeros_and_empty_output_is_noop():
+    import ctypes
+    lib = P.load_library()
+    stream = torch.cuda.current_stream().cuda_stream
+    buf = torch.zeros(4096, dtype=torch.uint8, device=DEV)
+    p = buf.data_ptr()
+    a = P.puro_fp8_tensor_t(p, p, 256, 0, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT, 0)
+    b = P.puro_fp8_tensor_t(p, p, 128, 0, P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT, 0)
+    y = torch.full((256, 128), 7.0, dtype=torch.bfloat16, device=DEV)
+    assert lib.puro_fp8_linear_fprop(ctypes.byref(a), ctypes.byref(b), y.data_ptr(), None, 0, None, stream) == 0
+    torch.cuda.synchronize()
+    assert torch.all(y == 0)
+    a0 = P.puro_fp8_tensor_t(p, p, 0, 128, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT, 0)
+    b1 = P.puro_fp8_tensor_t(p, p, 128, 128, P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT, 0)
+    y.fill_(3.0)
+    assert lib.puro_fp8_linear_fprop(ctypes.byref(a0), ctypes.byref(b1), y.data_ptr(), None, 0, None, stream) == 0
+    torch.cuda.synchronize()
+    assert torch.all(y == 3.0)
+
+
+def test_gemm_status_word_stays_clear_on_success():
+    M, N, K = 256, 256, 256
+    x, w, dy = _inputs(M, N, K, 91)
+    out = run_linear(x, w, dy, P.SCALE_BLOCK)  # asserts the status word is 0
+    assert torch.isfinite(out["y"].float()).all()

@@ -1,0 +1,178 @@
+"""GPU parity of amax and the quantisers against the oracle: every amax,
+every scale and every FP8 byte must match bit for bit.
+
+Sizes span several 128x128 tiles; per-tensor cases include ragged tails
+(extents that are multiples of 16 but not of 128).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import paper_2608_27370_gb300 as P
+from paper_2608_27370_gb300 import workloads as W
+from _parity import bits, check_block_act_quant, check_block_weight_quant, check_tensor_quant, host
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+FMTS = [P.E4M3, P.E5M2]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    P.load_library()
+
+
+def _t3(shape, seed, scale=1.0):
+    return (W.student_t3_f32(shape, DEV, seed) * scale).to(torch.bfloat16)
+
+
+# ------------------------------------------------------------------ amax
+@pytest.mark.parametrize("n", [0, 1, 7, 8, 9, 1000, 4096 * 33 + 5, 3_000_001])
+def test_amax_bit_exact(n):
+    x = _t3((n,), 100 + n, 3.0)
+    a = torch.full((1,), -1, dtype=torch.int32, device=DEV)
+    P.puro_fp8_amax(x, a)
+    torch.cuda.synchronize()
+    want = O.amax_bf16(bits(x)) if n else 0
+    assert int(host(a)[0]) == want
+
+
+def test_amax_nonfinite_and_sign():
+    x = torch.randn(50_000, device=DEV).to(torch.bfloat16)
+    x[123] = -300.0
+    a = torch.zeros(1, dtype=torch.int32, device=DEV)
+    P.puro_fp8_amax(x, a)
+    torch.cuda.synchronize()
+    assert int(host(a)[0]) == O.amax_bf16(bits(x)) == 0x4396  # |-300| = 0x4396 in bf16
+    x[40_000] = float("-inf")
+    P.puro_fp8_amax(x, a)
+    torch.cuda.synchronize()
+    assert int(host(a)[0]) == 0x7F80
+    x.view(torch.int16)[7] = 0x7FC1  # a NaN
+    P.puro_fp8_amax(x, a)
+    torch.cuda.synchronize()
+    assert int(host(a)[0]) == O.amax_bf16(bits(x)) > 0x7F80
+
+
+# ------------------------------------------------- 1x128 groups (activations)
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("shape", [(128, 128), (384, 640), (256, 1536), (1024, 256)])
+def test_block_act_quantize(shape, fmt):
+    x = _t3(shape, 7 + shape[0] + shape[1])
+    x[:, 5] *= 50.0  # an outlier channel
+    q = P.quantize(x, fmt, P.SCALE_BLOCK, P.ROLE_ACT)
+    torch.cuda.synchronize()
+    check_block_act_quant(x, q, fmt)
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+def test_block_act_quantize_rowwise_only(fmt):
+    x = _t3((256, 384), 9)
+    q = P.quantize(x, fmt, P.SCALE_BLOCK, P.ROLE_ACT, transpose=False)
+    torch.cuda.synchronize()
+    assert q.colwise is None
+    check_block_act_quant(x, q, fmt)
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+def test_block_act_special_values(fmt):
+    """Zero groups, non-finite groups, bf16 subnormals, huge values, values
+    that round to -0, and exact FP8 values."""
+    x = _t3((256, 512), 11)
+    xv = x.view(torch.int16)
+    x[0:128, 0:128] = 0.0                                  # all-zero tile (row and column groups)
+    x[3, 130] = float("inf")                               # one inf: its row group and column group
+    xv[200, 300] = 0x7FC0                                  # +NaN
+    xv[201, 301] = -1                                      # 0xFFFF: -NaN
+    x[130, 384:512] = torch.tensor(1e-40).to(torch.bfloat16)   # bf16 subnormals (scale exponent clamps at 0)
+    x[131, 384:512] = 3.0e38                                # near the bf16 max
+    x[132, 384:400] = -1e-30                                # tiny negatives in a group with a large max
+    x[132, 400] = 200.0
+    q = P.quantize(x, fmt, P.SCALE_BLOCK, P.ROLE_ACT)
+    torch.cuda.synchronize()
+    check_block_act_quant(x, q, fmt)
+    s = host(q.rowwise.scale)
+    assert s[1, 3] == 0xFF and s[0, 0] == 127 and s[3, 130] == 0  # non-finite / zero / clamped
+
+
+def test_block_act_canaries():
+    """Guard bands around every output buffer stay untouched."""
+    R, C, pad = 384, 256, 64
+    x = _t3((R, C), 12)
+
+    def guarded(n):
+        buf = torch.full((n + 2 * pad,), 0xA5, dtype=torch.uint8, device=DEV)
+        return buf, buf[pad:pad + n]
+
+    bq, q = guarded(R * C)
+    bs, s = guarded(R * C // 128)
+    bqt, qt = guarded(R * C)
+    bst, st = guarded(R * C // 128)
+    P.puro_fp8_quantize(x, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT, None, q.view(R, C), s.view(C // 128, R),
+                        qt.view(C, R), st.view(R // 128, C))
+    torch.cuda.synchronize()
+    for b in (bq, bs, bqt, bst):
+        h = host(b)
+        assert np.all(h[:pad] == 0xA5) and np.all(h[-pad:] == 0xA5)
+    out = P.Quantized(P.FP8Operand(q.view(R, C), s.view(C // 128, R)), P.FP8Operand(qt.view(C, R), st.view(R // 128, C)))
+    check_block_act_quant(x, out, P.E4M3)
+
+
+# ----------------------------------------------- 128x128 blocks (weights)
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("shape", [(128, 128), (256, 384), (1536, 1536), (2048, 1536)])
+def test_block_weight_quantize(shape, fmt):
+    w = W.normal_bf16(shape, 0.02, DEV, 31 + shape[0])
+    w[7, 9] = -1.5
+    q = P.quantize(w, fmt, P.SCALE_BLOCK, P.ROLE_WEIGHT)
+    torch.cuda.synchronize()
+    check_block_weight_quant(w, q, fmt)
+
+
+def test_block_weight_nonfinite_block():
+    w = W.normal_bf16((256, 256), 0.02, DEV, 5)
+    w[130, 3] = float("nan")
+    q = P.quantize(w, P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT)
+    torch.cuda.synchronize()
+    check_block_weight_quant(w, q, P.E4M3)
+    assert host(q.rowwise.scale)[1, 0] == 0xFF
+
+
+# ------------------------------------------------------- per-tensor scaling
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("shape", [(256, 1536), (272, 400), (16, 16), (128, 2064)])
+def test_tensor_quantize(shape, fmt):
+    x = _t3(shape, 41 + shape[1], 0.01)
+    q = P.quantize(x, fmt, P.SCALE_TENSOR, P.ROLE_ACT)
+    torch.cuda.synchronize()
+    check_tensor_quant(x, q, fmt)
+
+
+def test_tensor_quantize_edge_cases():
+    z = torch.zeros((32, 64), dtype=torch.bfloat16, device=DEV)
+    q = P.quantize(z, P.E4M3, P.SCALE_TENSOR, P.ROLE_ACT)
+    torch.cuda.synchronize()
+    check_tensor_quant(z, q, P.E4M3)
+    assert host(q.rowwise.scale)[0] == 1.0
+    tiny = torch.zeros((16, 32), dtype=torch.bfloat16, device=DEV)
+    tiny.view(torch.int16)[0, 0] = 1          # smallest bf16 subnormal: 448/amax overflows -> FLT_MAX
+    tiny.view(torch.int16)[5, 5] = -32767     # 0x8001
+    q = P.quantize(tiny, P.E4M3, P.SCALE_TENSOR, P.ROLE_ACT)
+    torch.cuda.synchronize()
+    check_tensor_quant(tiny, q, P.E4M3)
+    bad = torch.ones((16, 32), dtype=torch.bfloat16, device=DEV)
+    bad[3, 3] = float("-inf")
+    q = P.quantize(bad, P.E4M3, P.SCALE_TENSOR, P.ROLE_ACT)
+    torch.cuda.synchronize()
+    check_tensor_quant(bad, q, P.E4M3)
+    assert np.isnan(host(q.rowwise.scale)[0])
+
+
+def test_tensor_quantize_empty():
+    x = torch.empty((0, 64), dtype=torch.bfloat16, device=DEV)
+    q = P.quantize(x, P.E4M3, P.SCALE_TENSOR, P.ROLE_ACT, transpose=False)
+    torch.cuda.synchronize()
+    assert int(host(q.amax)[0]) == 0 and host(q.rowwise.scale)[0] == 1.0

@@ -1,0 +1,149 @@
+"""Host-side checks of the C ABI (no GPU needed): the library builds and
+loads, exports every entry point the header declares, the ctypes mirror of
+puro_fp8_tensor_t has the C layout, and argument validation rejects bad
+calls synchronously, before any CUDA work is enqueued."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+import torch
+
+import paper_2608_27370_gb300 as P
+from paper_2608_27370_gb300 import _build
+
+BAD = P.PURO_ERR_INVALID_ARG
+A = 0x100000  # a 16-byte aligned fake device address (never dereferenced)
+
+
+@pytest.fixture(scope="module")
+def lib():
+    _build.build()
+    return P.load_library()
+
+
+def _declared_functions():
+    text = open(P.HEADER_PATH).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(puro_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared_functions()
+    for required in ("puro_fp8_amax", "puro_fp8_quantize", "puro_fp8_linear_fprop", "puro_fp8_linear_dgrad",
+                     "puro_fp8_linear_wgrad", "puro_fp8_workspace_size", "puro_fp8_get_status",
+                     "puro_bf16_linear_fprop", "puro_bf16_linear_dgrad", "puro_bf16_linear_wgrad"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in _declared_functions():
+        assert hasattr(lib, name), name
+        assert name in P._SIGNATURES, f"binding lacks {name}"
+
+
+def test_struct_layout_matches_c(tmp_path):
+    """Compile a probe against the header with the C compiler and compare."""
+    src = tmp_path / "probe.c"
+    src.write_text(
+        '#include <stddef.h>\n#include <stdio.h>\n#include "puro_fp8.h"\n'
+        "int main(void){printf(\"%zu %zu %zu %zu %zu %zu %zu %zu %zu\\n\", sizeof(puro_fp8_tensor_t),"
+        "offsetof(puro_fp8_tensor_t,data),offsetof(puro_fp8_tensor_t,scale),offsetof(puro_fp8_tensor_t,rows),"
+        "offsetof(puro_fp8_tensor_t,red),offsetof(puro_fp8_tensor_t,fmt),offsetof(puro_fp8_tensor_t,scaling),"
+        "offsetof(puro_fp8_tensor_t,role),offsetof(puro_fp8_tensor_t,reserved));return 0;}\n")
+    exe = tmp_path / "probe"
+    subprocess.run(["gcc", "-std=c11", "-I", os.path.dirname(P.HEADER_PATH), str(src), "-o", str(exe)], check=True)
+    got = [int(v) for v in subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()]
+    T = P.puro_fp8_tensor_t
+    want = [ctypes.sizeof(T)] + [getattr(T, f).offset for f in
+                                 ("data", "scale", "rows", "red", "fmt", "scaling", "role", "reserved")]
+    assert got == want
+
+
+def test_status_strings(lib):
+    assert lib.puro_status_string(0) == b"PURO_OK"
+    assert lib.puro_status_string(4) == b"PURO_ERR_TIMEOUT"
+
+
+def test_amax_validation(lib):
+    assert lib.puro_fp8_amax(A, 4, 8, None, None) == BAD           # no output word
+    assert lib.puro_fp8_amax(A, -1, 8, A, None) == BAD             # negative extent
+    assert lib.puro_fp8_amax(A + 2, 4, 8, A, None) == BAD          # misaligned input
+    assert lib.puro_fp8_amax(None, 4, 8, A, None) == BAD           # null input
+    assert lib.puro_fp8_amax(A, 4, 8, A + 2, None) == BAD          # misaligned output word
+
+
+def test_quantize_validation(lib):
+    q = lib.puro_fp8_quantize
+    BLK, TEN, ACT, WGT = P.SCALE_BLOCK, P.SCALE_TENSOR, P.ROLE_ACT, P.ROLE_WEIGHT
+    assert q(A, 128, 128, 7, BLK, ACT, None, A, A, A, A, None) == BAD       # bad format
+    assert q(A, 128, 128, 0, 9, ACT, None, A, A, A, A, None) == BAD         # bad scaling
+    assert q(A, 128, 128, 0, BLK, 5, None, A, A, A, A, None) == BAD         # bad role
+    assert q(A, 130, 128, 0, BLK, ACT, None, A, A, A, A, None) == BAD       # ragged rows in BLOCK
+    assert q(A, 128, 200, 0, BLK, WGT, None, A, A, A, A, None) == BAD       # ragged cols in BLOCK
+    assert q(A, 128, 128, 0, BLK, ACT, A, A, A, A, A, None) == BAD          # amax given in BLOCK
+    assert q(A, 128, 128, 0, BLK, ACT, None, A, A, A, None, None) == BAD    # q_t without scale_t
+    assert q(A, 128, 128, 0, BLK, ACT, None, A + 8, A, None, None, None) == BAD  # misaligned q
+    assert q(A, 128, 128, 0, TEN, ACT, None, A, A, None, None, None) == BAD  # TENSOR needs amax
+    assert q(A, 128, 120, 0, TEN, ACT, A, A, A, None, None, None) == BAD     # TENSOR cols % 16
+    assert q(A, 120, 128, 0, TEN, ACT, A, A, A, A, None, None) == BAD        # TENSOR rows % 16 with q_t
+    assert q(None, 128, 128, 0, BLK, ACT, None, A, A, A, A, None) == BAD     # null input
+    assert q(A, 128, 128, 0, BLK, ACT, None, None, A, None, None, None) == BAD  # null q
+    # empty BLOCK tensors are a valid no-op that touches nothing
+    assert q(None, 0, 128, 0, BLK, ACT, None, A, A, A, A, None) == P.PURO_OK
+
+
+def _op(rows, red, scaling=P.SCALE_BLOCK, role=P.ROLE_ACT, fmt=0, data=A, scale=A, reserved=0):
+    return P.puro_fp8_tensor_t(data, scale, rows, red, fmt, scaling, role, reserved)
+
+
+def test_gemm_validation(lib):
+    f = lib.puro_fp8_linear_fprop
+    r = ctypes.byref
+    x, w = _op(256, 384), _op(512, 384, role=P.ROLE_WEIGHT)
+    assert f(r(x), r(w), None, None, 0, None, None) == BAD                       # no output
+    assert f(r(x), r(w), A + 4, None, 0, None, None) == BAD                      # misaligned output
+    assert f(r(x), r(_op(512, 256, role=P.ROLE_WEIGHT)), A, None, 0, None, None) == BAD  # K mismatch
+    assert f(r(_op(256, 384, role=P.ROLE_WEIGHT)), r(w), A, None, 0, None, None) == BAD  # A must be ACT
+    assert f(r(x), r(_op(512, 384, scaling=P.SCALE_TENSOR)), A, None, 0, None, None) == BAD  # mixed scaling
+    assert f(r(_op(200, 384)), r(w), A, None, 0, None, None) == BAD              # ragged BLOCK
+    assert f(r(_op(256, 384, fmt=3)), r(w), A, None, 0, None, None) == BAD       # bad format
+    assert f(r(_op(256, 384, reserved=1)), r(w), A, None, 0, None, None) == BAD  # reserved field
+    assert f(r(_op(256, 384, data=0)), r(w), A, None, 0, None, None) == BAD      # null data
+    assert f(r(_op(256, 384, scale=A + 1)), r(w), A, None, 0, None, None) == BAD  # misaligned scale
+    assert f(r(_op(24, 40, scaling=P.SCALE_TENSOR)), r(_op(16, 40, scaling=P.SCALE_TENSOR)), A, None, 0, None,
+             None) == BAD                                                         # TENSOR extents % 16
+    assert f(None, r(w), A, None, 0, None, None) == BAD
+    # empty output extent: valid no-op
+    assert f(r(_op(0, 384)), r(w), A, None, 0, None, None) == P.PURO_OK
+    # 128x128 weight grids longer than 256 blocks along K are not implemented
+    big = 128 * 257
+    assert f(r(_op(128, big)), r(_op(128, big, role=P.ROLE_WEIGHT)), A, None, 0, None, None) == P.PURO_ERR_UNSUPPORTED
+
+
+def test_bf16_gemm_validation(lib):
+    assert lib.puro_bf16_linear_fprop(A, A, A, 12, 16, 16, None, None) == BAD   # M % 8
+    assert lib.puro_bf16_linear_fprop(A, A + 2, A, 16, 16, 16, None, None) == BAD
+    assert lib.puro_bf16_linear_dgrad(None, A, A, 16, 16, 16, None, None) == BAD
+    assert lib.puro_bf16_linear_wgrad(A, A, A, 16, -8, 16, None, None) == BAD
+    assert lib.puro_bf16_linear_fprop(A, A, A, 0, 16, 16, None, None) == P.PURO_OK
+
+
+def test_get_status_validation(lib):
+    out = ctypes.c_int32(0)
+    assert lib.puro_fp8_get_status(None, ctypes.byref(out), None) == BAD
+    assert lib.puro_fp8_get_status(A, None, None) == BAD
+
+
+@pytest.mark.skipif(torch.cuda.is_available(), reason="checks the no-GPU failure mode")
+def test_valid_call_without_gpu_fails_loudly(lib):
+    x, w = _op(256, 384), _op(512, 384, role=P.ROLE_WEIGHT)
+    st = lib.puro_fp8_linear_fprop(ctypes.byref(x), ctypes.byref(w), A, None, 0, None, None)
+    assert st == P.PURO_ERR_CUDA
+
+
+def test_binding_refuses_host_tensors():
+    x = torch.zeros(128, 128, dtype=torch.bfloat16)
+    with pytest.raises(ValueError):
+        P.puro_fp8_amax(x, torch.zeros(1, dtype=torch.int32))
