@@ -358,7 +358,7 @@ def cpu_baseline(torch, stack, seconds_hint=True):
 
     import oracle as O
 
-    M_s = 2048
+    M_s = min(8192, stack.M)
     li = stack.inputs[0][1]  # o_proj [1536, 1536]
     N, K = li.w.shape
 
