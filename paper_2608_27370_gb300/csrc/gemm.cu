@@ -8,10 +8,14 @@
 //   warp 0      TMA producer: A/B tiles (128-byte swizzle) and, for the
 //               block-scaled kind, the raw E8M0 row scales, into a
 //               STAGES-deep shared-memory ring gated by mbarriers;
-//   warp 1      MMA issuer: allocates tensor memory, stages the block
-//               scales into tensor memory (tcgen05.cp), issues tcgen05.mma
-//               (kind::f16 / kind::f8f6f4 / kind::mxf8f6f4.block_scale) and
-//               commits stage releases and accumulator hand-offs;
+//   warp 1      MMA issuer: allocates tensor memory, copies the staged
+//               block scales into tensor memory (tcgen05.cp), issues
+//               tcgen05.mma (kind::f16 / kind::f8f6f4 /
+//               kind::mxf8f6f4.block_scale) and commits stage releases and
+//               accumulator hand-offs;
+//   warp 2      (block-scaled kind) scale staging: rearranges each stage's
+//               E8M0 exponents into the tcgen05.cp source layout, off the
+//               MMA issuer's critical path;
 //   warps 4..7  epilogue: tcgen05.ld the 128x256 FP32 accumulator (one
 //               32-lane quarter per warp), release it, convert to BF16
 //               (times scale_inv_a * scale_inv_b for the per-tensor kind)
@@ -45,6 +49,7 @@ struct GemmSmem {
     alignas(16) uint8_t sf_raw_a[kStages][kBM];
     alignas(16) uint8_t sf_raw_b[kStages][kBN];
     uint64_t full[kStages];
+    uint64_t sf_ready[kStages];  // block-scaled kind: scale vectors staged for tcgen05.cp
     uint64_t empty[kStages];
     uint64_t tfull[2];
     uint64_t tempty[2];
@@ -108,6 +113,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(&sm.full[s], 1);
+            mbar_init(&sm.sf_ready[s], 1);
             mbar_init(&sm.empty[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -134,9 +140,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------ TMA producer
         if (lane == 0) {
             uint32_t stage = 0, phase = 0;
-            uint32_t fills[kStages];  // times each stage was filled
-#pragma unroll
-            for (int s = 0; s < kStages; ++s) fills[s] = 0;
+            uint32_t issued = 0;  // stage fills started by this thread
             bool aborted = false;
             for (int tile = blockIdx.x; tile < p.num_tiles && !aborted; tile += gridDim.x) {
                 const int m0 = (tile / p.num_n) * kBM;
@@ -160,54 +164,28 @@ __global__ void __launch_bounds__(kThreads, 1)
                             bulk_load(sm.sf_raw_b[stage], p.sfb + static_cast<int64_t>(kb) * p.N + n0, sfb_bytes,
                                       &sm.full[stage]);
                     }
-                    ++fills[stage];
+                    ++issued;
                     if (++stage == kStages) {
                         stage = 0;
                         phase ^= 1u;
                     }
                 }
             }
-            // Every copy this thread started must land before the CTA exits.
-            for (int s = 0; s < kStages; ++s)
-                if (fills[s] > 0) mbar_wait_bounded(&sm.full[s], (fills[s] - 1u) & 1u, kDrainTimeoutNs);
+            // Every copy this thread started must land before the CTA exits:
+            // wait for the latest fill of each stage (fills go round-robin).
+            for (uint32_t s = 0; s < kStages; ++s) {
+                const uint32_t fills = issued / kStages + (s < issued % kStages ? 1u : 0u);
+                if (fills > 0) mbar_wait_bounded(&sm.full[s], (fills - 1u) & 1u, kDrainTimeoutNs);
+            }
         }
     } else if (warp == 1) {
         // ------------------------------------------------ MMA issuer
         uint32_t stage = 0, phase = 0;
         bool aborted = false;
         int local = 0;
-        // 128x128 weight-block scales of the current / next tile: lane j
-        // holds k-blocks 8j .. 8j+7 of n-block 0 (words 0,1) and 1 (2,3).
-        uint32_t blk_cur[4] = {0, 0, 0, 0}, blk_nxt[4] = {0, 0, 0, 0};
-        auto load_blk = [&](int tile, uint32_t (&r)[4]) {
-            const int nb0 = (tile % p.num_n) * (kBN / 128);
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int nb = nb0 + h;
-                const bool nb_ok = nb * 128 < p.N;
-#pragma unroll
-                for (int w = 0; w < 2; ++w) {
-                    uint32_t word = 0;
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        const int kb = 8 * lane + 4 * w + i;
-                        uint32_t v = 127u;
-                        if (nb_ok && kb < p.sfb_kb) v = p.sfb[static_cast<int64_t>(nb) * p.sfb_kb + kb];
-                        word |= v << (8 * i);
-                    }
-                    r[2 * h + w] = word;
-                }
-            }
-        };
-        if (kMX && p.sfb_blk && static_cast<int>(blockIdx.x) < p.num_tiles) load_blk(blockIdx.x, blk_cur);
-
         for (int tile = blockIdx.x; tile < p.num_tiles && !aborted; tile += gridDim.x, ++local) {
-            const int n0 = (tile % p.num_n) * kBN;
             const int buf = local % kAccBufs;
             const uint32_t acc_phase = static_cast<uint32_t>(local / kAccBufs) & 1u;
-            if (kMX && p.sfb_blk && tile + static_cast<int>(gridDim.x) < p.num_tiles)
-                load_blk(tile + gridDim.x, blk_nxt);
-
             bool ok = (sm.abort_flag == 0) && mbar_wait_bounded(&sm.tempty[buf], acc_phase ^ 1u, p.wait_ns);
             if (!__all_sync(0xFFFFFFFFu, ok)) {
                 if (lane == 0) record_timeout(sm, p.status);
@@ -218,55 +196,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t d_tmem = tmem + static_cast<uint32_t>(buf * kBN);
 
             for (int kb = 0; kb < p.num_kb; ++kb) {
-                ok = (sm.abort_flag == 0) && mbar_wait_bounded(&sm.full[stage], phase, p.wait_ns);
+                // block-scaled: the scale warp has staged this stage's scale
+                // vectors (and has itself seen the operands land)
+                ok = (sm.abort_flag == 0) &&
+                     mbar_wait_bounded(kMX ? &sm.sf_ready[stage] : &sm.full[stage], phase, p.wait_ns) &&
+                     (!kMX || mbar_wait_bounded(&sm.full[stage], phase, p.wait_ns));
                 if (!__all_sync(0xFFFFFFFFu, ok)) {
                     if (lane == 0) record_timeout(sm, p.status);
                     aborted = true;
                     break;
                 }
                 tc_fence_after_sync();
-                uint32_t sfa_col = 0, sfb_col = 0;
-                if constexpr (kMX) {
-                    // Scale factors in tensor memory: row r of a 128-row
-                    // operand block sits in lane r % 32 (of every quarter),
-                    // column r / 32; the byte chosen by the scale id (0) --
-                    // all four bytes carry the same exponent.
-                    sfa_col = kSfBase + stage * kSfColsPerStage;
-                    sfb_col = sfa_col + 4;
-                    const uint8_t *ra = sm.sf_raw_a[stage];
-                    uint4 la;
-                    la.x = ra[lane] * 0x01010101u;
-                    la.y = ra[lane + 32] * 0x01010101u;
-                    la.z = ra[lane + 64] * 0x01010101u;
-                    la.w = ra[lane + 96] * 0x01010101u;
-                    *reinterpret_cast<uint4 *>(sm.sf_utccp_a[stage] + 16 * lane) = la;
-                    uint32_t wb[8];
-                    if (p.sfb_blk) {
-                        const int src = kb >> 3, wsel = (kb >> 2) & 1, sh = 8 * (kb & 3);
-                        const uint32_t w00 = __shfl_sync(0xFFFFFFFFu, blk_cur[0], src);
-                        const uint32_t w01 = __shfl_sync(0xFFFFFFFFu, blk_cur[1], src);
-                        const uint32_t w10 = __shfl_sync(0xFFFFFFFFu, blk_cur[2], src);
-                        const uint32_t w11 = __shfl_sync(0xFFFFFFFFu, blk_cur[3], src);
-                        const uint32_t s0 = ((wsel ? w01 : w00) >> sh) & 0xFFu;
-                        const uint32_t s1 = ((wsel ? w11 : w10) >> sh) & 0xFFu;
-#pragma unroll
-                        for (int j = 0; j < 8; ++j) wb[j] = (j < 4 ? s0 : s1) * 0x01010101u;
-                    } else {
-                        const uint8_t *rb = sm.sf_raw_b[stage];
-                        const int valid = p.N - n0;
-#pragma unroll
-                        for (int j = 0; j < 8; ++j) {
-                            const int r = lane + 32 * j;
-                            wb[j] = (r < valid ? static_cast<uint32_t>(rb[r]) : 127u) * 0x01010101u;
-                        }
-                    }
-                    *reinterpret_cast<uint4 *>(sm.sf_utccp_b[stage] + 16 * lane) = make_uint4(wb[0], wb[1], wb[2], wb[3]);
-                    *reinterpret_cast<uint4 *>(sm.sf_utccp_b[stage] + 512 + 16 * lane) =
-                        make_uint4(wb[4], wb[5], wb[6], wb[7]);
-                    fence_proxy_async_smem();
-                    __syncwarp();
-                }
                 if (lane == 0) {
+                    const uint32_t sfa_col = kSfBase + stage * kSfColsPerStage;
+                    const uint32_t sfb_col = sfa_col + 4;
                     if constexpr (kMX) {
                         tmem_cp_32x128b_warpx4(tmem + sfa_col, smem_desc_plain_16B_rows(smem_u32(sm.sf_utccp_a[stage])));
                         tmem_cp_32x128b_warpx4(tmem + sfb_col, smem_desc_plain_16B_rows(smem_u32(sm.sf_utccp_b[stage])));
@@ -298,10 +241,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (aborted) break;
             if (lane == 0) tc_commit(&sm.tfull[buf]);  // accumulator complete
             __syncwarp();
-            if (kMX && p.sfb_blk) {
-#pragma unroll
-                for (int i = 0; i < 4; ++i) blk_cur[i] = blk_nxt[i];
-            }
         }
         // All MMAs and copies issued by this warp complete before teardown.
         if (lane == 0) {
@@ -309,6 +248,91 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_wait_bounded(&sm.drain, 0, kDrainTimeoutNs);
         }
         __syncwarp();
+    } else if (kMX && warp == 2) {
+        // ------------------------------------------------ scale staging
+        // Turns each stage's raw E8M0 exponents into the tcgen05.cp source
+        // layout: row r of a 128-row operand block goes to line r % 32, word
+        // r / 32, all four bytes of the word carrying the exponent (one 1x128
+        // group spans four K=32 MMAs, each reading one scale per row).
+        uint32_t stage = 0, phase = 0;
+        bool aborted = false;
+        // 128x128 weight-block scales of the current / next tile: lane j
+        // holds k-blocks 8j .. 8j+7 of n-block 0 (words 0,1) and 1 (2,3).
+        uint32_t blk_cur[4] = {0, 0, 0, 0}, blk_nxt[4] = {0, 0, 0, 0};
+        auto load_blk = [&](int tile, uint32_t (&r)[4]) {
+            const int nb0 = (tile % p.num_n) * (kBN / 128);
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int nb = nb0 + h;
+                const bool nb_ok = nb * 128 < p.N;
+#pragma unroll
+                for (int w = 0; w < 2; ++w) {
+                    uint32_t word = 0;
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const int kb = 8 * lane + 4 * w + i;
+                        uint32_t v = 127u;
+                        if (nb_ok && kb < p.sfb_kb) v = p.sfb[static_cast<int64_t>(nb) * p.sfb_kb + kb];
+                        word |= v << (8 * i);
+                    }
+                    r[2 * h + w] = word;
+                }
+            }
+        };
+        if (p.sfb_blk && static_cast<int>(blockIdx.x) < p.num_tiles) load_blk(blockIdx.x, blk_cur);
+        for (int tile = blockIdx.x; tile < p.num_tiles && !aborted; tile += gridDim.x) {
+            const int n0 = (tile % p.num_n) * kBN;
+            if (p.sfb_blk && tile + static_cast<int>(gridDim.x) < p.num_tiles) load_blk(tile + gridDim.x, blk_nxt);
+            for (int kb = 0; kb < p.num_kb; ++kb) {
+                bool ok = (sm.abort_flag == 0) && mbar_wait_bounded(&sm.full[stage], phase, p.wait_ns);
+                if (!__all_sync(0xFFFFFFFFu, ok)) {
+                    if (lane == 0) record_timeout(sm, p.status);
+                    aborted = true;
+                    break;
+                }
+                const uint8_t *ra = sm.sf_raw_a[stage];
+                uint4 la;
+                la.x = ra[lane] * 0x01010101u;
+                la.y = ra[lane + 32] * 0x01010101u;
+                la.z = ra[lane + 64] * 0x01010101u;
+                la.w = ra[lane + 96] * 0x01010101u;
+                *reinterpret_cast<uint4 *>(sm.sf_utccp_a[stage] + 16 * lane) = la;
+                uint32_t wb[8];
+                if (p.sfb_blk) {
+                    const int src = kb >> 3, wsel = (kb >> 2) & 1, sh = 8 * (kb & 3);
+                    const uint32_t w00 = __shfl_sync(0xFFFFFFFFu, blk_cur[0], src);
+                    const uint32_t w01 = __shfl_sync(0xFFFFFFFFu, blk_cur[1], src);
+                    const uint32_t w10 = __shfl_sync(0xFFFFFFFFu, blk_cur[2], src);
+                    const uint32_t w11 = __shfl_sync(0xFFFFFFFFu, blk_cur[3], src);
+                    const uint32_t s0 = ((wsel ? w01 : w00) >> sh) & 0xFFu;
+                    const uint32_t s1 = ((wsel ? w11 : w10) >> sh) & 0xFFu;
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) wb[j] = (j < 4 ? s0 : s1) * 0x01010101u;
+                } else {
+                    const uint8_t *rb = sm.sf_raw_b[stage];
+                    const int valid = p.N - n0;
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        const int r = lane + 32 * j;
+                        wb[j] = (r < valid ? static_cast<uint32_t>(rb[r]) : 127u) * 0x01010101u;
+                    }
+                }
+                *reinterpret_cast<uint4 *>(sm.sf_utccp_b[stage] + 16 * lane) = make_uint4(wb[0], wb[1], wb[2], wb[3]);
+                *reinterpret_cast<uint4 *>(sm.sf_utccp_b[stage] + 512 + 16 * lane) =
+                    make_uint4(wb[4], wb[5], wb[6], wb[7]);
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sm.sf_ready[stage]);
+                if (++stage == kStages) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            if (p.sfb_blk) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) blk_cur[i] = blk_nxt[i];
+            }
+        }
     } else if (warp >= 4) {
         // ------------------------------------------------ epilogue
         const int q = warp & 3;  // TMEM lane quarter of this warp
@@ -330,19 +354,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t t_row = tmem + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(buf * kBN);
             uint32_t packed[kBN / 2];  // the whole 256-column row as bf16 pairs
 #pragma unroll
-            for (int c = 0; c < kBN / 32; ++c) {
-                uint32_t r[32];
-                tmem_ld_32x32b_x32(t_row + 32 * c, r);
+            for (int h = 0; h < kBN / 128; ++h) {
+                uint32_t r[4][32];
+#pragma unroll
+                for (int c = 0; c < 4; ++c) tmem_ld_32x32b_x32(t_row + 128 * h + 32 * c, r[c]);
                 tmem_ld_wait();
 #pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    float lo = __uint_as_float(r[2 * i]), hi = __uint_as_float(r[2 * i + 1]);
-                    if constexpr (KIND == kGemmFP8Tensor) {
-                        lo = __fmul_rn(lo, sab);
-                        hi = __fmul_rn(hi, sab);
+                for (int c = 0; c < 4; ++c) {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        float lo = __uint_as_float(r[c][2 * i]), hi = __uint_as_float(r[c][2 * i + 1]);
+                        if constexpr (KIND == kGemmFP8Tensor) {
+                            lo = __fmul_rn(lo, sab);
+                            hi = __fmul_rn(hi, sab);
+                        }
+                        __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+                        packed[64 * h + 16 * c + i] = *reinterpret_cast<uint32_t *>(&v);
                     }
-                    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-                    packed[16 * c + i] = *reinterpret_cast<uint32_t *>(&v);
                 }
             }
             tc_fence_before_sync();
