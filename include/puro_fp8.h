@@ -39,13 +39,21 @@
  * Scale layouts
  *   PURO_SCALE_TENSOR : `scale` is one float, the dequantisation factor
  *                       scale_inv = fp32(1 / fp32(fmt_max / amax)).
- *   PURO_SCALE_BLOCK, role ACT (1x128 groups along `red`):
- *                       uint8 E8M0 exponents g (value 2^(g-127)), stored
- *                       group-major: s[(c / 128) * rows + r] is the scale of
- *                       elements (r, c .. c+127).  Shape [red/128][rows].
- *   PURO_SCALE_BLOCK, role WEIGHT (128x128 blocks):
- *                       uint8 E8M0 exponents, s[(r/128) * (red/128) + c/128],
- *                       shape [rows/128][red/128] (plain row-major grid).
+ *   PURO_SCALE_BLOCK  : uint8 E8M0 exponents g (scale 2^(g-127)) stored as
+ *                       the tensor cores read them ("scale vectors"): for an
+ *                       operand [rows, red], KB = red/128 k-blocks in
+ *                       KG = ceil(KB/4) groups, the buffer is
+ *                       [rows/128][KG][512] bytes and byte
+ *                           16*l + 4*j + b   of chunk (rb, kg)
+ *                       holds g of row 128*rb + 32*j + l, k-block 4*kg + b
+ *                       (l < 32, j < 4, b < 4); bytes of k-blocks >= KB are
+ *                       127.  One 512-byte chunk is exactly the 32-line x
+ *                       16-byte image tcgen05.cp loads for 128 rows, and b is
+ *                       the MMA scale id.
+ *                       role ACT: g of the 1x128 group (row, k-block).
+ *                       role WEIGHT: g of the 128x128 block (row/128,
+ *                       k-block), i.e. repeated over the block's rows.
+ *                       Size: rows * KG * 4 bytes (puro_fp8_scale_bytes).
  *   g = 0xFF marks a group that held Inf or NaN; its codes are NaN.
  */
 #ifndef PURO_FP8_H
@@ -140,6 +148,8 @@ puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t cols,
  *   fprop: A = x   (Xq   [M, K], ACT)    B = w   (Wq   [N, K], WEIGHT)  -> y  [M, N]
  *   dgrad: A = dy  (dYq  [M, N], ACT)    B = w_t (Wq^T [K, N], WEIGHT)  -> dx [M, K]
  *   wgrad: A = dy_t(dYq^T[N, M], ACT)    B = x_t (Xq^T [K, M], ACT)     -> dw [N, K]
+ * (the GEMM itself does not depend on the roles: every BLOCK operand carries
+ * per-row scale vectors).
  * Both operands must use the same `scaling`.  BLOCK: all extents multiples
  * of 128.  TENSOR: extents multiples of 16.  A zero reduction extent writes
  * zeros; a zero output extent is a no-op.
@@ -159,6 +169,12 @@ puro_status_t puro_fp8_linear_dgrad(const puro_fp8_tensor_t *dy, const puro_fp8_
 puro_status_t puro_fp8_linear_wgrad(const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t,
                                     void *dw, void *workspace, size_t workspace_bytes,
                                     int32_t *dev_status, void *stream);
+
+/*
+ * Bytes of a PURO_SCALE_BLOCK scale buffer for an operand [rows, red]
+ * (rows * ceil(red/512) * 4).  Host-only, no CUDA call.
+ */
+size_t puro_fp8_scale_bytes(int64_t rows, int64_t red);
 
 /*
  * Scratch bytes that let a GEMM with output [rows_out, cols_out] and

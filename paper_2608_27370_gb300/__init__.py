@@ -71,6 +71,7 @@ _SIGNATURES = {
     "puro_fp8_linear_dgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_wgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_workspace_size": (ctypes.c_size_t, [_I64, _I64, _I64]),
+    "puro_fp8_scale_bytes": (ctypes.c_size_t, [_I64, _I64]),
     "puro_fp8_get_status": (_I32, [_P, _P, _P]),
     "puro_bf16_linear_fprop": (_I32, [_P, _P, _P, _I64, _I64, _I64, _P, _P]),
     "puro_bf16_linear_dgrad": (_I32, [_P, _P, _P, _I64, _I64, _I64, _P, _P]),
@@ -247,12 +248,20 @@ class Quantized:
     amax: Optional[torch.Tensor] = None
 
 
+def scale_vec_shape(rows: int, red: int):
+    """Shape of a blockwise scale buffer for an operand [rows, red]: 512-byte
+    tensor-core scale-vector chunks per 128 rows and 4 k-blocks."""
+    return (rows // 128, (red // 128 + 3) // 4, 512)
+
+
 def empty_scales(rows: int, red: int, scaling: int, role: int, device) -> torch.Tensor:
     if scaling == SCALE_TENSOR:
         return torch.empty(1, dtype=torch.float32, device=device)
-    if role == ROLE_ACT:
-        return torch.empty((red // 128, rows), dtype=torch.uint8, device=device)
-    return torch.empty((rows // 128, red // 128), dtype=torch.uint8, device=device)
+    return torch.empty(scale_vec_shape(rows, red), dtype=torch.uint8, device=device)
+
+
+def puro_fp8_scale_bytes(rows: int, red: int) -> int:
+    return int(load_library().puro_fp8_scale_bytes(rows, red))
 
 
 def quantize(x: torch.Tensor, fmt: int = E4M3, scaling: int = SCALE_BLOCK, role: int = ROLE_ACT,
@@ -281,5 +290,5 @@ def quantize(x: torch.Tensor, fmt: int = E4M3, scaling: int = SCALE_BLOCK, role:
 
 __all__ = [n for n in dir() if n.startswith("puro_")] + [
     "E4M3", "E5M2", "SCALE_TENSOR", "SCALE_BLOCK", "ROLE_ACT", "ROLE_WEIGHT", "PuroError", "FP8Operand",
-    "Quantized", "quantize", "load_library", "empty_scales", "LIB_PATH", "HEADER_PATH",
+    "Quantized", "quantize", "load_library", "empty_scales", "scale_vec_shape", "LIB_PATH", "HEADER_PATH",
 ]

@@ -65,14 +65,13 @@ puro_status_t cuda_status(cudaError_t e) { return e == cudaSuccess ? PURO_OK : P
 bool valid_fmt(int32_t f) { return f == PURO_E4M3 || f == PURO_E5M2; }
 
 // Shape/pointer checks shared by the FP8 GEMM entry points.
-puro_status_t check_operand(const puro_fp8_tensor_t *t, bool must_be_act) {
+puro_status_t check_operand(const puro_fp8_tensor_t *t) {
     if (!t || !t->data || !t->scale) return PURO_ERR_INVALID_ARG;
     if (!aligned16(t->data) || !aligned16(t->scale)) return PURO_ERR_INVALID_ARG;
     if (t->rows < 0 || t->red < 0 || !valid_fmt(t->fmt) || t->reserved != 0) return PURO_ERR_INVALID_ARG;
     if (t->rows > INT32_MAX || t->red > INT32_MAX) return PURO_ERR_UNSUPPORTED;
     if (t->scaling == PURO_SCALE_BLOCK) {
         if (t->role != PURO_ROLE_ACT && t->role != PURO_ROLE_WEIGHT) return PURO_ERR_INVALID_ARG;
-        if (must_be_act && t->role != PURO_ROLE_ACT) return PURO_ERR_INVALID_ARG;
         if (t->rows % 128 || t->red % 128) return PURO_ERR_INVALID_ARG;
     } else if (t->scaling == PURO_SCALE_TENSOR) {
         if (t->rows % 16 || t->red % 16) return PURO_ERR_INVALID_ARG;
@@ -85,9 +84,9 @@ puro_status_t check_operand(const puro_fp8_tensor_t *t, bool must_be_act) {
 // D[M,N] = A[M,K] * B[N,K]^T over quantised operands.
 puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, void *d, int32_t *dev_status,
                        void *stream) {
-    puro_status_t st = check_operand(a, /*must_be_act=*/true);
+    puro_status_t st = check_operand(a);
     if (st != PURO_OK) return st;
-    st = check_operand(b, /*must_be_act=*/false);
+    st = check_operand(b);
     if (st != PURO_OK) return st;
     if (a->red != b->red || a->scaling != b->scaling) return PURO_ERR_INVALID_ARG;
     if (!d || !aligned16(d)) return PURO_ERR_INVALID_ARG;
@@ -96,7 +95,6 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
     if (M == 0 || N == 0) return PURO_OK;
     if (K == 0) return cuda_status(cudaMemsetAsync(d, 0, static_cast<size_t>(M * N) * 2, s));
     const bool block = a->scaling == PURO_SCALE_BLOCK;
-    if (block && b->role == PURO_ROLE_WEIGHT && K / 128 > 256) return PURO_ERR_UNSUPPORTED;
 
     CUtensorMap tm_a, tm_b, tm_d;
     if (!make_map(&tm_a, CU_TENSOR_MAP_DATA_TYPE_UINT8, a->data, K, M, K, 128, kGemmBM,
@@ -115,7 +113,6 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
     if (block) {
         g.sfa = static_cast<const uint8_t *>(a->scale);
         g.sfb = static_cast<const uint8_t *>(b->scale);
-        g.sfb_blk = b->role == PURO_ROLE_WEIGHT ? 1 : 0;
     } else {
         g.sia = static_cast<const float *>(a->scale);
         g.sib = static_cast<const float *>(b->scale);
@@ -251,6 +248,11 @@ PURO_API size_t puro_fp8_workspace_size(int64_t rows_out, int64_t cols_out, int6
     (void)cols_out;
     (void)red;
     return 0;
+}
+
+PURO_API size_t puro_fp8_scale_bytes(int64_t rows, int64_t red) {
+    if (rows <= 0 || red <= 0) return 0;
+    return static_cast<size_t>(rows) * static_cast<size_t>((red / 128 + 3) / 4) * 4;
 }
 
 PURO_API puro_status_t puro_fp8_get_status(const int32_t *dev_status, int32_t *host_out, void *stream) {

@@ -6,16 +6,16 @@
 //
 // One persistent, warp-specialised CTA per SM:
 //   warp 0      TMA producer: A/B tiles (128-byte swizzle) and, for the
-//               block-scaled kind, the raw E8M0 row scales, into a
-//               STAGES-deep shared-memory ring gated by mbarriers;
-//   warp 1      MMA issuer: allocates tensor memory, copies the staged
-//               block scales into tensor memory (tcgen05.cp), issues
-//               tcgen05.mma (kind::f16 / kind::f8f6f4 /
-//               kind::mxf8f6f4.block_scale) and commits stage releases and
-//               accumulator hand-offs;
-//   warp 2      (block-scaled kind) scale staging: rearranges each stage's
-//               E8M0 exponents into the tcgen05.cp source layout, off the
-//               MMA issuer's critical path;
+//               block-scaled kind, the E8M0 scale vectors (already in the
+//               tensor-core layout, 512 bytes per 128 rows and four
+//               k-blocks), into a STAGES-deep shared-memory ring gated by
+//               mbarriers;
+//   warp 1      MMA issuer: allocates tensor memory, copies the scale
+//               vectors into tensor memory (tcgen05.cp, once per four
+//               k-blocks), issues tcgen05.mma (kind::f16 / kind::f8f6f4 /
+//               kind::mxf8f6f4.block_scale, the scale id picking the
+//               k-block's byte) and commits stage releases and accumulator
+//               hand-offs;
 //   warps 4..7  epilogue: tcgen05.ld the 128x256 FP32 accumulator (one
 //               32-lane quarter per warp), release it, convert to BF16
 //               (times scale_inv_a * scale_inv_b for the per-tensor kind)
@@ -36,7 +36,8 @@ constexpr int kBKBytes = 128;      // bytes of K per pipeline stage (one swizzle
 constexpr int kStages = 4;
 constexpr int kThreads = 256;
 constexpr int kTmemCols = 512;
-constexpr int kSfColsPerStage = 12;  // 4 for A (128 rows) + 8 for B (256 rows)
+constexpr int kSfColsPerSet = 12;  // 4 for A (128 rows) + 8 for B (256 rows)
+constexpr int kSfSets = 2;         // double-buffered across groups of four k-blocks
 constexpr uint64_t kDrainTimeoutNs = 2000000000ull;
 constexpr int32_t kStatusTimeout = 4;  // PURO_ERR_TIMEOUT
 
@@ -44,12 +45,9 @@ struct GemmSmem {
     alignas(1024) uint8_t a[kStages][kBM * kBKBytes];
     alignas(1024) uint8_t b[kStages][kBN * kBKBytes];
     alignas(1024) uint8_t epi[4][32 * 128];          // per epilogue warp: 32 rows x 64 bf16
-    alignas(128) uint8_t sf_utccp_a[kStages][512];   // 32 lines x 16 B
-    alignas(128) uint8_t sf_utccp_b[kStages][1024];  // 2 x (32 lines x 16 B)
-    alignas(16) uint8_t sf_raw_a[kStages][kBM];
-    alignas(16) uint8_t sf_raw_b[kStages][kBN];
+    alignas(128) uint8_t sf_a[kStages][512];   // scale vectors of A: 32 lines x 16 B
+    alignas(128) uint8_t sf_b[kStages][1024];  // scale vectors of B: 2 x (32 lines x 16 B)
     uint64_t full[kStages];
-    uint64_t sf_ready[kStages];  // block-scaled kind: scale vectors staged for tcgen05.cp
     uint64_t empty[kStages];
     uint64_t tfull[2];
     uint64_t tempty[2];
@@ -62,10 +60,9 @@ struct GemmParams {
     int M, N, K;
     int num_n, num_kb, num_tiles;
     uint32_t idesc;
-    const uint8_t *sfa;
-    const uint8_t *sfb;
-    int sfb_blk;
-    int sfb_kb;  // K / 128 (row length of the 128x128 grid)
+    const uint8_t *sfa;  // scale vectors of A, [M/128][kgroups][512]
+    const uint8_t *sfb;  // scale vectors of B, [N/128][kgroups][512]
+    int kgroups;         // ceil(K / 512)
     const float *sia;
     const float *sib;
     int32_t *status;
@@ -77,7 +74,8 @@ struct GemmParams {
 //     [10,13) B type, [17,23) N >> 3, [24,29) M >> 4.
 //   kind::mxf8f6f4: [4,6) B scale id, [7,10) A type, [10,13) B type,
 //     [17,23) N >> 3, [23] scale type (1 = UE8M0), [24,29) M >> 4,
-//     [29,31) A scale id.
+//     [29,31) A scale id.  The scale id selects the byte of the 32-bit
+//     tensor-memory scale word: here the k-block within its group of four.
 __host__ __device__ constexpr uint32_t idesc_dense(uint32_t atype, uint32_t btype) {
     return (1u << 4) | (atype << 7) | (btype << 10) | (static_cast<uint32_t>(kBN >> 3) << 17) |
            (static_cast<uint32_t>(kBM >> 4) << 24);
@@ -98,11 +96,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                    const __grid_constant__ CUtensorMap tm_d, const GemmParams p) {
     constexpr bool kMX = (KIND == kGemmFP8Block);
     constexpr int kAccBufs = kMX ? 1 : 2;              // accumulators of kBN columns
-    constexpr int kSfBase = kAccBufs * kBN;            // first scale-factor column (MX)
+    constexpr int kSfBase = kAccBufs * kBN;            // first scale-vector column (MX)
     constexpr int kElemBytes = (KIND == kGemmBF16) ? 2 : 1;
     constexpr int kBK = kBKBytes / kElemBytes;         // elements of K per stage
     constexpr int kKSteps = kBKBytes / 32;             // MMAs per stage (32 bytes of K each)
-    static_assert(!kMX || kSfBase + kStages * kSfColsPerStage <= kTmemCols, "TMEM budget");
+    static_assert(!kMX || kSfBase + kSfSets * kSfColsPerSet <= kTmemCols, "TMEM budget");
 
     extern __shared__ uint8_t smem_raw[];
     GemmSmem &sm = *reinterpret_cast<GemmSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -113,7 +111,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(&sm.full[s], 1);
-            mbar_init(&sm.sf_ready[s], 1);
             mbar_init(&sm.empty[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -145,24 +142,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int tile = blockIdx.x; tile < p.num_tiles && !aborted; tile += gridDim.x) {
                 const int m0 = (tile / p.num_n) * kBM;
                 const int n0 = (tile % p.num_n) * kBN;
-                const uint32_t sfb_bytes = static_cast<uint32_t>(min(kBN, p.N - n0));
+                const bool b_second = n0 + 128 < p.N;  // second 128-row block of B in range
                 for (int kb = 0; kb < p.num_kb; ++kb) {
                     if (sm.abort_flag || !mbar_wait_bounded(&sm.empty[stage], phase ^ 1u, p.wait_ns)) {
                         record_timeout(sm, p.status);
                         aborted = true;
                         break;
                     }
-                    uint32_t bytes = (kBM + kBN) * kBKBytes;
-                    if (kMX) bytes += kBM + (p.sfb_blk ? 0u : sfb_bytes);
+                    const bool sf_load = kMX && (kb & 3) == 0;
+                    const uint32_t bytes = (kBM + kBN) * kBKBytes + (sf_load ? 512u + 1024u : 0u);
                     mbar_arrive_expect_tx(&sm.full[stage], bytes);
                     tma_load_2d(sm.a[stage], &tm_a, &sm.full[stage], kb * kBK, m0);
                     tma_load_2d(sm.b[stage], &tm_b, &sm.full[stage], kb * kBK, n0);
-                    if (kMX) {
-                        bulk_load(sm.sf_raw_a[stage], p.sfa + static_cast<int64_t>(kb) * p.M + m0, kBM,
+                    if (sf_load) {
+                        const int64_t kg = kb >> 2;
+                        bulk_load(sm.sf_a[stage], p.sfa + ((m0 / 128) * static_cast<int64_t>(p.kgroups) + kg) * 512, 512,
                                   &sm.full[stage]);
-                        if (!p.sfb_blk)
-                            bulk_load(sm.sf_raw_b[stage], p.sfb + static_cast<int64_t>(kb) * p.N + n0, sfb_bytes,
-                                      &sm.full[stage]);
+                        const uint8_t *b0 = p.sfb + ((n0 / 128) * static_cast<int64_t>(p.kgroups) + kg) * 512;
+                        bulk_load(sm.sf_b[stage], b0, 512, &sm.full[stage]);
+                        // beyond N the B rows are zero-filled; any finite scale will do
+                        bulk_load(sm.sf_b[stage] + 512, b_second ? b0 + static_cast<int64_t>(p.kgroups) * 512 : b0, 512,
+                                  &sm.full[stage]);
                     }
                     ++issued;
                     if (++stage == kStages) {
@@ -196,11 +196,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t d_tmem = tmem + static_cast<uint32_t>(buf * kBN);
 
             for (int kb = 0; kb < p.num_kb; ++kb) {
-                // block-scaled: the scale warp has staged this stage's scale
-                // vectors (and has itself seen the operands land)
-                ok = (sm.abort_flag == 0) &&
-                     mbar_wait_bounded(kMX ? &sm.sf_ready[stage] : &sm.full[stage], phase, p.wait_ns) &&
-                     (!kMX || mbar_wait_bounded(&sm.full[stage], phase, p.wait_ns));
+                ok = (sm.abort_flag == 0) && mbar_wait_bounded(&sm.full[stage], phase, p.wait_ns);
                 if (!__all_sync(0xFFFFFFFFu, ok)) {
                     if (lane == 0) record_timeout(sm, p.status);
                     aborted = true;
@@ -208,13 +204,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc_fence_after_sync();
                 if (lane == 0) {
-                    const uint32_t sfa_col = kSfBase + stage * kSfColsPerStage;
+                    const uint32_t sfa_col = kSfBase + ((kb >> 2) & 1) * kSfColsPerSet;
                     const uint32_t sfb_col = sfa_col + 4;
+                    uint32_t idesc = p.idesc;
                     if constexpr (kMX) {
-                        tmem_cp_32x128b_warpx4(tmem + sfa_col, smem_desc_plain_16B_rows(smem_u32(sm.sf_utccp_a[stage])));
-                        tmem_cp_32x128b_warpx4(tmem + sfb_col, smem_desc_plain_16B_rows(smem_u32(sm.sf_utccp_b[stage])));
-                        tmem_cp_32x128b_warpx4(tmem + sfb_col + 4,
-                                               smem_desc_plain_16B_rows(smem_u32(sm.sf_utccp_b[stage] + 512)));
+                        if ((kb & 3) == 0) {  // new group of four k-blocks: its scale vectors
+                            tmem_cp_32x128b_warpx4(tmem + sfa_col, smem_desc_plain_16B_rows(smem_u32(sm.sf_a[stage])));
+                            tmem_cp_32x128b_warpx4(tmem + sfb_col, smem_desc_plain_16B_rows(smem_u32(sm.sf_b[stage])));
+                            tmem_cp_32x128b_warpx4(tmem + sfb_col + 4,
+                                                   smem_desc_plain_16B_rows(smem_u32(sm.sf_b[stage] + 512)));
+                        }
+                        const uint32_t sf_id = static_cast<uint32_t>(kb & 3);
+                        idesc |= (sf_id << 29) | (sf_id << 4);
                     }
                     const uint32_t a_addr = smem_u32(sm.a[stage]);
                     const uint32_t b_addr = smem_u32(sm.b[stage]);
@@ -224,11 +225,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint64_t bd = smem_desc_k_sw128(b_addr + 32 * k);
                         const uint32_t acc = (kb > 0 || k > 0) ? 1u : 0u;
                         if constexpr (KIND == kGemmBF16)
-                            mma_f16(d_tmem, ad, bd, p.idesc, acc);
+                            mma_f16(d_tmem, ad, bd, idesc, acc);
                         else if constexpr (KIND == kGemmFP8Tensor)
-                            mma_f8(d_tmem, ad, bd, p.idesc, acc);
+                            mma_f8(d_tmem, ad, bd, idesc, acc);
                         else
-                            mma_mxf8(d_tmem, ad, bd, p.idesc, tmem + sfa_col, tmem + sfb_col, acc);
+                            mma_mxf8(d_tmem, ad, bd, idesc, tmem + sfa_col, tmem + sfb_col, acc);
                     }
                     tc_commit(&sm.empty[stage]);  // stage reusable once these MMAs finish
                 }
@@ -248,91 +249,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_wait_bounded(&sm.drain, 0, kDrainTimeoutNs);
         }
         __syncwarp();
-    } else if (kMX && warp == 2) {
-        // ------------------------------------------------ scale staging
-        // Turns each stage's raw E8M0 exponents into the tcgen05.cp source
-        // layout: row r of a 128-row operand block goes to line r % 32, word
-        // r / 32, all four bytes of the word carrying the exponent (one 1x128
-        // group spans four K=32 MMAs, each reading one scale per row).
-        uint32_t stage = 0, phase = 0;
-        bool aborted = false;
-        // 128x128 weight-block scales of the current / next tile: lane j
-        // holds k-blocks 8j .. 8j+7 of n-block 0 (words 0,1) and 1 (2,3).
-        uint32_t blk_cur[4] = {0, 0, 0, 0}, blk_nxt[4] = {0, 0, 0, 0};
-        auto load_blk = [&](int tile, uint32_t (&r)[4]) {
-            const int nb0 = (tile % p.num_n) * (kBN / 128);
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int nb = nb0 + h;
-                const bool nb_ok = nb * 128 < p.N;
-#pragma unroll
-                for (int w = 0; w < 2; ++w) {
-                    uint32_t word = 0;
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        const int kb = 8 * lane + 4 * w + i;
-                        uint32_t v = 127u;
-                        if (nb_ok && kb < p.sfb_kb) v = p.sfb[static_cast<int64_t>(nb) * p.sfb_kb + kb];
-                        word |= v << (8 * i);
-                    }
-                    r[2 * h + w] = word;
-                }
-            }
-        };
-        if (p.sfb_blk && static_cast<int>(blockIdx.x) < p.num_tiles) load_blk(blockIdx.x, blk_cur);
-        for (int tile = blockIdx.x; tile < p.num_tiles && !aborted; tile += gridDim.x) {
-            const int n0 = (tile % p.num_n) * kBN;
-            if (p.sfb_blk && tile + static_cast<int>(gridDim.x) < p.num_tiles) load_blk(tile + gridDim.x, blk_nxt);
-            for (int kb = 0; kb < p.num_kb; ++kb) {
-                bool ok = (sm.abort_flag == 0) && mbar_wait_bounded(&sm.full[stage], phase, p.wait_ns);
-                if (!__all_sync(0xFFFFFFFFu, ok)) {
-                    if (lane == 0) record_timeout(sm, p.status);
-                    aborted = true;
-                    break;
-                }
-                const uint8_t *ra = sm.sf_raw_a[stage];
-                uint4 la;
-                la.x = ra[lane] * 0x01010101u;
-                la.y = ra[lane + 32] * 0x01010101u;
-                la.z = ra[lane + 64] * 0x01010101u;
-                la.w = ra[lane + 96] * 0x01010101u;
-                *reinterpret_cast<uint4 *>(sm.sf_utccp_a[stage] + 16 * lane) = la;
-                uint32_t wb[8];
-                if (p.sfb_blk) {
-                    const int src = kb >> 3, wsel = (kb >> 2) & 1, sh = 8 * (kb & 3);
-                    const uint32_t w00 = __shfl_sync(0xFFFFFFFFu, blk_cur[0], src);
-                    const uint32_t w01 = __shfl_sync(0xFFFFFFFFu, blk_cur[1], src);
-                    const uint32_t w10 = __shfl_sync(0xFFFFFFFFu, blk_cur[2], src);
-                    const uint32_t w11 = __shfl_sync(0xFFFFFFFFu, blk_cur[3], src);
-                    const uint32_t s0 = ((wsel ? w01 : w00) >> sh) & 0xFFu;
-                    const uint32_t s1 = ((wsel ? w11 : w10) >> sh) & 0xFFu;
-#pragma unroll
-                    for (int j = 0; j < 8; ++j) wb[j] = (j < 4 ? s0 : s1) * 0x01010101u;
-                } else {
-                    const uint8_t *rb = sm.sf_raw_b[stage];
-                    const int valid = p.N - n0;
-#pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        const int r = lane + 32 * j;
-                        wb[j] = (r < valid ? static_cast<uint32_t>(rb[r]) : 127u) * 0x01010101u;
-                    }
-                }
-                *reinterpret_cast<uint4 *>(sm.sf_utccp_b[stage] + 16 * lane) = make_uint4(wb[0], wb[1], wb[2], wb[3]);
-                *reinterpret_cast<uint4 *>(sm.sf_utccp_b[stage] + 512 + 16 * lane) =
-                    make_uint4(wb[4], wb[5], wb[6], wb[7]);
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&sm.sf_ready[stage]);
-                if (++stage == kStages) {
-                    stage = 0;
-                    phase ^= 1u;
-                }
-            }
-            if (p.sfb_blk) {
-#pragma unroll
-                for (int i = 0; i < 4; ++i) blk_cur[i] = blk_nxt[i];
-            }
-        }
     } else if (warp >= 4) {
         // ------------------------------------------------ epilogue
         const int q = warp & 3;  // TMEM lane quarter of this warp
@@ -431,8 +347,7 @@ static cudaError_t launch_kind(const GemmArgs &g, const CUtensorMap &tm_a, const
         p.idesc = idesc_mx(static_cast<uint32_t>(g.a_fmt), static_cast<uint32_t>(g.b_fmt));
     p.sfa = g.sfa;
     p.sfb = g.sfb;
-    p.sfb_blk = g.sfb_blk;
-    p.sfb_kb = static_cast<int>(g.K / 128);
+    p.kgroups = static_cast<int>((g.K / 128 + 3) / 4);
     p.sia = g.sia;
     p.sib = g.sib;
     p.status = g.status;

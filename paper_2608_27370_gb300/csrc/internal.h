@@ -22,8 +22,8 @@ struct QuantArgs {
     int fmt;                  // 0 = E4M3, 1 = E5M2
     QuantKind kind;
     const uint32_t *amax;     // kQuantTensor only
-    uint8_t *scale_u8;        // block scales of q
-    uint8_t *scale_t_u8;      // block scales of q_t
+    uint8_t *scale_u8;        // block scale vectors of q (tensor-core layout)
+    uint8_t *scale_t_u8;      // block scale vectors of q_t (tensor-core layout)
     float *scale_f;           // tensor scale_inv for q
     float *scale_t_f;         // tensor scale_inv for q_t (may be null)
     bool has_t;
@@ -50,12 +50,10 @@ struct GemmArgs {
     GemmKind kind;
     int a_fmt, b_fmt;            // FP8 formats (0 = E4M3, 1 = E5M2)
     int64_t M, N, K;
-    // kGemmFP8Block: A scales are 1x128 groups, group-major [K/128][M].
+    // kGemmFP8Block: scale vectors of A and B in the tensor-core layout,
+    // [rows/128][ceil(K/512)][512] bytes each.
     const uint8_t *sfa;
-    // B scales: group-major [K/128][N] (sfb_blk = 0) or 128x128 grid
-    // [N/128][K/128] (sfb_blk = 1).
     const uint8_t *sfb;
-    int sfb_blk;
     // kGemmFP8Tensor: dequantisation factors of A and B.
     const float *sia, *sib;
     int32_t *status;             // optional device status word

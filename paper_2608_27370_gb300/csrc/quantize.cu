@@ -135,6 +135,22 @@ PURO_DEV float tensor_scale(uint32_t amax_bits) {
     return isinf(s) ? FLT_MAX : s;
 }
 
+// Tensor-core scale-vector layout of an FP8 operand [R, red] (see the
+// public header): 512-byte chunks per (128-row block, group of four
+// k-blocks); byte 16*l + 4*j + b of chunk (rb, kg) is the exponent of row
+// 128*rb + 32*j + l for k-block 4*kg + b.  The tile that owns the last
+// k-block also fills the group's unused bytes with 127 (scale 1).
+PURO_DEV void store_scale_vec(uint8_t *__restrict__ base, int64_t row, int64_t kb, int64_t kblocks, uint8_t g) {
+    const int64_t groups = (kblocks + 3) / 4;
+    const int64_t rb = row / 128;
+    const int i = static_cast<int>(row & 127);
+    uint8_t *chunk = base + (rb * groups + kb / 4) * 512 + 16 * (i & 31) + 4 * (i >> 5);
+    const int b = static_cast<int>(kb & 3);
+    chunk[b] = g;
+    if (kb == kblocks - 1)
+        for (int pb = b + 1; pb < 4; ++pb) chunk[pb] = 127;
+}
+
 // ------------------------------------------------------ cast kernel
 constexpr int kQT = 128;          // tile edge
 constexpr int kQThreads = 256;
@@ -313,19 +329,22 @@ __global__ void __launch_bounds__(kQThreads, 2)
             if (HAS_T) tma_store_2d(&tm_qt, sm.qt_stage, static_cast<int32_t>(r0), static_cast<int32_t>(c0));
             bulk_commit_group();
         }
-        if constexpr (KIND == kQuantBlockAct) {
-            if (tid < 32) {
-                *reinterpret_cast<uint32_t *>(scale_u8 + (c0 / kQT) * rows + r0 + 4 * tid) =
-                    *reinterpret_cast<const uint32_t *>(sm.row_g + 4 * tid);
-            } else if (HAS_T && tid < 64) {
-                const int t = tid - 32;
-                *reinterpret_cast<uint32_t *>(scale_t_u8 + (r0 / kQT) * cols + c0 + 4 * t) =
-                    *reinterpret_cast<const uint32_t *>(sm.col_g + 4 * t);
-            }
-        } else if constexpr (KIND == kQuantBlockWeight) {
-            if (tid == 0) {
-                scale_u8[(r0 / kQT) * (cols / kQT) + c0 / kQT] = static_cast<uint8_t>(blk_g);
-                if (HAS_T) scale_t_u8[(c0 / kQT) * (rows / kQT) + r0 / kQT] = static_cast<uint8_t>(blk_g);
+        if constexpr (KIND != kQuantTensor) {
+            // Scale vectors in the tensor-core layout: thread i < 128 writes
+            // row i of the rowwise operand (k-block c0/128), thread 128 + i
+            // writes row i of the transposed operand (k-block r0/128).
+            const bool col = tid >= kQT;
+            if (!col || HAS_T) {
+                const int i = tid & (kQT - 1);
+                const int64_t op_rows0 = col ? c0 : r0;       // first operand row of this tile
+                const int64_t kb = (col ? r0 : c0) / kQT;     // k-block of this tile
+                const int64_t kblocks = (col ? rows : cols) / kQT;
+                uint8_t g;
+                if constexpr (KIND == kQuantBlockAct)
+                    g = col ? sm.col_g[i] : sm.row_g[i];
+                else
+                    g = static_cast<uint8_t>(blk_g);
+                store_scale_vec(col ? scale_t_u8 : scale_u8, op_rows0 + i, kb, kblocks, g);
             }
         }
     }

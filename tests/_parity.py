@@ -4,7 +4,7 @@ C ABI, rebuild the oracle's view of the same bytes, compare.
 The oracle never sees a byte produced by the CUDA path: it quantises the
 same BF16 inputs itself and forms its own fp64 products.  Layout
 conversions between the oracle's natural scale grids and the library's
-group-major ones are plain transposes.
+tensor-core scale vectors are plain index permutations.
 """
 from __future__ import annotations
 
@@ -52,6 +52,32 @@ def run_linear(x, w, dy, scaling=P.SCALE_BLOCK, fmt_x=P.E4M3, fmt_w=P.E4M3, fmt_
 
 
 # --------------------------------------------------------------------------
+# Scale layouts: the oracle's natural per-row grid [rows, KB] <-> the
+# library's tensor-core scale vectors [rows/128, ceil(KB/4), 512]
+# (byte 16*l + 4*j + b of chunk (rb, kg) = row 128*rb + 32*j + l,
+# k-block 4*kg + b; padding k-blocks hold 127).  Pure index permutations.
+# --------------------------------------------------------------------------
+def to_scale_vec(g_rows: np.ndarray) -> np.ndarray:
+    rows, kb = g_rows.shape
+    kg = (kb + 3) // 4
+    pad = np.full((rows, kg * 4), 127, np.uint8)
+    pad[:, :kb] = g_rows
+    a = pad.reshape(rows // 128, 4, 32, kg, 4)           # [rb, j, l, kg, b]
+    return np.ascontiguousarray(a.transpose(0, 3, 2, 1, 4).reshape(rows // 128, kg, 512))
+
+
+def from_scale_vec(v: np.ndarray, kb: int) -> np.ndarray:
+    rb, kg, _ = v.shape
+    a = v.reshape(rb, kg, 32, 4, 4).transpose(0, 3, 2, 1, 4)  # [rb, j, l, kg, b]
+    return np.ascontiguousarray(a.reshape(rb * 128, kg * 4)[:, :kb])
+
+
+def scales_of(op: "P.FP8Operand") -> np.ndarray:
+    """The exponents of an operand's scale vectors as a [rows, KB] grid."""
+    return from_scale_vec(host(op.scale), op.red // 128)
+
+
+# --------------------------------------------------------------------------
 # Comparisons
 # --------------------------------------------------------------------------
 def assert_close(gpu: torch.Tensor, ref: np.ndarray, what: str):
@@ -82,26 +108,31 @@ def check_block_act_quant(x: torch.Tensor, q: P.Quantized, fmt: int, rows=None, 
     xb = bits(x if rows is None else x[rows])
     q_ref, s_ref = O.quantize_rows_1x128(xb, fmt)
     qr = q.rowwise.data if rows is None else q.rowwise.data[rows]
-    sr = q.rowwise.scale if rows is None else q.rowwise.scale[:, rows]
     assert_bytes(qr, q_ref, "rowwise codes")
-    assert_bytes(sr, np.ascontiguousarray(s_ref.T), "rowwise scales")
+    if rows is None:  # the whole buffer, padding bytes included
+        assert_bytes(q.rowwise.scale, to_scale_vec(s_ref), "rowwise scale vectors")
+    else:
+        assert np.array_equal(scales_of(q.rowwise)[host(rows)], s_ref), "rowwise scales (sampled rows)"
     if q.colwise is None:
         return
     xc = bits(x if cols is None else x[:, cols])
     qt_ref, st_ref = O.quantize_cols_128x1(xc, fmt)
     qc = q.colwise.data if cols is None else q.colwise.data[cols]
-    sc = q.colwise.scale if cols is None else q.colwise.scale[:, cols]
     assert_bytes(qc, qt_ref, "transposed codes")
-    assert_bytes(sc, np.ascontiguousarray(st_ref.T), "transposed scales")
+    if cols is None:
+        assert_bytes(q.colwise.scale, to_scale_vec(st_ref), "transposed scale vectors")
+    else:
+        assert np.array_equal(scales_of(q.colwise)[host(cols)], st_ref), "transposed scales (sampled columns)"
 
 
 def check_block_weight_quant(w: torch.Tensor, q: P.Quantized, fmt: int):
     q_ref, s_ref = O.quantize_blocks_128x128(bits(w), fmt)
     assert_bytes(q.rowwise.data, q_ref, "weight codes")
-    assert_bytes(q.rowwise.scale, s_ref, "weight block scales")
+    assert_bytes(q.rowwise.scale, to_scale_vec(np.repeat(s_ref, 128, axis=0)), "weight scale vectors")
     if q.colwise is not None:
         assert_bytes(q.colwise.data, np.ascontiguousarray(q_ref.T), "transposed weight codes")
-        assert_bytes(q.colwise.scale, np.ascontiguousarray(s_ref.T), "transposed weight scales")
+        assert_bytes(q.colwise.scale, to_scale_vec(np.repeat(np.ascontiguousarray(s_ref.T), 128, axis=0)),
+                     "transposed weight scale vectors")
 
 
 def check_tensor_quant(x: torch.Tensor, q: P.Quantized, fmt: int):

@@ -11,7 +11,7 @@ import torch
 import oracle as O
 import paper_2608_27370_gb300 as P
 from paper_2608_27370_gb300 import workloads as W
-from _parity import bits, check_block_act_quant, check_block_weight_quant, check_tensor_quant, host
+from _parity import bits, check_block_act_quant, check_block_weight_quant, check_tensor_quant, host, scales_of
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda"
@@ -59,7 +59,7 @@ def test_amax_nonfinite_and_sign():
 
 # ------------------------------------------------- 1x128 groups (activations)
 @pytest.mark.parametrize("fmt", FMTS)
-@pytest.mark.parametrize("shape", [(128, 128), (384, 640), (256, 1536), (1024, 256)])
+@pytest.mark.parametrize("shape", [(128, 128), (384, 640), (256, 1536), (1024, 256), (640, 384)])
 def test_block_act_quantize(shape, fmt):
     x = _t3(shape, 7 + shape[0] + shape[1])
     x[:, 5] *= 50.0  # an outlier channel
@@ -94,8 +94,8 @@ def test_block_act_special_values(fmt):
     q = P.quantize(x, fmt, P.SCALE_BLOCK, P.ROLE_ACT)
     torch.cuda.synchronize()
     check_block_act_quant(x, q, fmt)
-    s = host(q.rowwise.scale)
-    assert s[1, 3] == 0xFF and s[0, 0] == 127 and s[3, 130] == 0  # non-finite / zero / clamped
+    s = scales_of(q.rowwise)  # [row, k-block]
+    assert s[3, 1] == 0xFF and s[0, 0] == 127 and s[130, 3] == 0  # non-finite / zero / clamped
 
 
 def test_block_act_canaries():
@@ -107,17 +107,18 @@ def test_block_act_canaries():
         buf = torch.full((n + 2 * pad,), 0xA5, dtype=torch.uint8, device=DEV)
         return buf, buf[pad:pad + n]
 
+    ss, sst = P.scale_vec_shape(R, C), P.scale_vec_shape(C, R)
     bq, q = guarded(R * C)
-    bs, s = guarded(R * C // 128)
+    bs, s = guarded(int(np.prod(ss)))
     bqt, qt = guarded(R * C)
-    bst, st = guarded(R * C // 128)
-    P.puro_fp8_quantize(x, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT, None, q.view(R, C), s.view(C // 128, R),
-                        qt.view(C, R), st.view(R // 128, C))
+    bst, st = guarded(int(np.prod(sst)))
+    P.puro_fp8_quantize(x, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT, None, q.view(R, C), s.view(*ss),
+                        qt.view(C, R), st.view(*sst))
     torch.cuda.synchronize()
     for b in (bq, bs, bqt, bst):
         h = host(b)
         assert np.all(h[:pad] == 0xA5) and np.all(h[-pad:] == 0xA5)
-    out = P.Quantized(P.FP8Operand(q.view(R, C), s.view(C // 128, R)), P.FP8Operand(qt.view(C, R), st.view(R // 128, C)))
+    out = P.Quantized(P.FP8Operand(q.view(R, C), s.view(*ss)), P.FP8Operand(qt.view(C, R), st.view(*sst)))
     check_block_act_quant(x, out, P.E4M3)
 
 
@@ -138,7 +139,7 @@ def test_block_weight_nonfinite_block():
     q = P.quantize(w, P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT)
     torch.cuda.synchronize()
     check_block_weight_quant(w, q, P.E4M3)
-    assert host(q.rowwise.scale)[1, 0] == 0xFF
+    assert np.all(scales_of(q.rowwise)[128:256, 0] == 0xFF)
 
 
 # ------------------------------------------------------- per-tensor scaling

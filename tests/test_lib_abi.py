@@ -7,6 +7,7 @@ import os
 import re
 import subprocess
 
+import numpy as np
 import pytest
 import torch
 
@@ -105,7 +106,7 @@ def test_gemm_validation(lib):
     assert f(r(x), r(w), None, None, 0, None, None) == BAD                       # no output
     assert f(r(x), r(w), A + 4, None, 0, None, None) == BAD                      # misaligned output
     assert f(r(x), r(_op(512, 256, role=P.ROLE_WEIGHT)), A, None, 0, None, None) == BAD  # K mismatch
-    assert f(r(_op(256, 384, role=P.ROLE_WEIGHT)), r(w), A, None, 0, None, None) == BAD  # A must be ACT
+    assert f(r(_op(256, 384, role=7)), r(w), A, None, 0, None, None) == BAD      # bad role
     assert f(r(x), r(_op(512, 384, scaling=P.SCALE_TENSOR)), A, None, 0, None, None) == BAD  # mixed scaling
     assert f(r(_op(200, 384)), r(w), A, None, 0, None, None) == BAD              # ragged BLOCK
     assert f(r(_op(256, 384, fmt=3)), r(w), A, None, 0, None, None) == BAD       # bad format
@@ -117,9 +118,6 @@ def test_gemm_validation(lib):
     assert f(None, r(w), A, None, 0, None, None) == BAD
     # empty output extent: valid no-op
     assert f(r(_op(0, 384)), r(w), A, None, 0, None, None) == P.PURO_OK
-    # 128x128 weight grids longer than 256 blocks along K are not implemented
-    big = 128 * 257
-    assert f(r(_op(128, big)), r(_op(128, big, role=P.ROLE_WEIGHT)), A, None, 0, None, None) == P.PURO_ERR_UNSUPPORTED
 
 
 def test_bf16_gemm_validation(lib):
@@ -128,6 +126,13 @@ def test_bf16_gemm_validation(lib):
     assert lib.puro_bf16_linear_dgrad(None, A, A, 16, 16, 16, None, None) == BAD
     assert lib.puro_bf16_linear_wgrad(A, A, A, 16, -8, 16, None, None) == BAD
     assert lib.puro_bf16_linear_fprop(A, A, A, 0, 16, 16, None, None) == P.PURO_OK
+
+
+def test_scale_buffer_size(lib):
+    assert lib.puro_fp8_scale_bytes(256, 1536) == 256 * 3 * 4      # 12 k-blocks -> 3 groups
+    assert lib.puro_fp8_scale_bytes(128, 8960) == 128 * 18 * 4     # 70 k-blocks -> 18 groups
+    assert lib.puro_fp8_scale_bytes(0, 128) == 0
+    assert int(np.prod(P.scale_vec_shape(256, 8960))) == lib.puro_fp8_scale_bytes(256, 8960)
 
 
 def test_get_status_validation(lib):
