@@ -9,7 +9,9 @@
 // column-group scales from the same shared-memory copy, and writes the
 // rowwise codes and the transposed codes through shared memory with TMA
 // stores (the transposed staging tile uses the 128-byte swizzle so the
-// column pass stores without bank conflicts).
+// column pass stores without bank conflicts).  The arithmetic per value is
+// kept to a widening shift, half a packed fp32 multiply and half a paired
+// cvt, since at HBM rates the kernel is otherwise instruction bound.
 #include <cfloat>
 #include <cuda_bf16.h>
 
@@ -103,25 +105,43 @@ PURO_DEV uint32_t cvt_pair(float lo, float hi) {  // -> 16 bits, lo in the low b
 PURO_DEV float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 PURO_DEV float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
-// Codes of four bf16 values (two packed words) as 4 bytes (first value in
-// the low byte).  `mul` is the exact power-of-two multiplier (BLOCK) or the
-// fp32 tensor scale (TENSOR); `nan_group` selects the NaN-code rule.
-template <int FMT>
-PURO_DEV uint32_t quant4(uint32_t w0, uint32_t w1, float mul, bool nan_group) {
-    if (nan_group) {
-        // sign of each element, payload S.1111.111 / S.11111.11
-        uint32_t s = ((w0 >> 8) & 0x80u) | (((w0 >> 24) & 0x80u) << 8) | (((w1 >> 8) & 0x80u) << 16) |
-                     (((w1 >> 24) & 0x80u) << 24);
-        return s | 0x7F7F7F7Fu;
-    }
-    uint32_t lo = cvt_pair<FMT>(__fmul_rn(bf16_lo(w0), mul), __fmul_rn(bf16_hi(w0), mul));
-    uint32_t hi = cvt_pair<FMT>(__fmul_rn(bf16_lo(w1), mul), __fmul_rn(bf16_hi(w1), mul));
-    return lo | (hi << 16);
+PURO_DEV uint64_t f32x2(float lo, float hi) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
 }
 
-PURO_DEV uint32_t max_abs_pair(uint32_t w) {  // max of the two bf16 magnitudes
-    uint32_t m = w & 0x7FFF7FFFu;
-    return max(m & 0xFFFFu, m >> 16);
+// Two IEEE round-to-nearest fp32 products in one packed instruction.
+PURO_DEV uint64_t mul_f32x2(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+
+template <int FMT>
+PURO_DEV uint32_t cvt_f32x2(uint64_t v) {
+    float lo, hi;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+    return cvt_pair<FMT>(lo, hi);
+}
+
+// Codes of four values a, b, c, d (exact fp32 widenings of bf16) as four
+// bytes, a in the low byte.  `mul2` holds the multiplier twice: the exact
+// power of two 2^(127-g) (BLOCK) or the fp32 tensor scale (TENSOR).  A
+// non-finite group gives NaN codes that keep each value's sign.
+template <int FMT>
+PURO_DEV uint32_t quant4(float a, float b, float c, float d, uint64_t mul2, bool nan_group) {
+    if (__builtin_expect(nan_group, 0)) {
+        const uint32_t s = ((__float_as_uint(a) >> 24) & 0x80u) | (((__float_as_uint(b) >> 24) & 0x80u) << 8) |
+                           (((__float_as_uint(c) >> 24) & 0x80u) << 16) | (((__float_as_uint(d) >> 24) & 0x80u) << 24);
+        return s | 0x7F7F7F7Fu;
+    }
+    return cvt_f32x2<FMT>(mul_f32x2(f32x2(a, b), mul2)) | (cvt_f32x2<FMT>(mul_f32x2(f32x2(c, d), mul2)) << 16);
+}
+
+// max of the bf16 magnitudes in each 16-bit half, over four words
+PURO_DEV uint32_t max_abs4(uint4 v) {
+    return __vmaxu2(__vmaxu2(v.x & 0x7FFF7FFFu, v.y & 0x7FFF7FFFu), __vmaxu2(v.z & 0x7FFF7FFFu, v.w & 0x7FFF7FFFu));
 }
 
 // Exact 2^(127 - g) as fp32 for g in [0, 247] (always a normal number).
@@ -159,7 +179,7 @@ struct QuantSmem {
     alignas(1024) uint8_t qt_stage[kQT * kQT];    // transposed codes, 128B-swizzled rows
     alignas(1024) uint8_t q_stage[kQT * kQT];     // rowwise codes, plain rows
     alignas(128) uint16_t in[2][kQT * kQT];       // bf16 tile, double buffered
-    uint32_t col_amax[2][kQT];
+    uint32_t col_amax2[4][kQT / 2];  // per row quarter, two columns per word
     uint32_t red[8];
     alignas(16) uint8_t row_g[kQT];
     alignas(16) uint8_t col_g[kQT];
@@ -235,8 +255,9 @@ __global__ void __launch_bounds__(kQThreads, 2)
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
                 const uint4 v = *reinterpret_cast<const uint4 *>(in + (tid + kQThreads * i) * 8);
-                m = max(m, max(max(max_abs_pair(v.x), max_abs_pair(v.y)), max(max_abs_pair(v.z), max_abs_pair(v.w))));
+                m = __vmaxu2(m, max_abs4(v));
             }
+            m = max(m & 0xFFFFu, m >> 16);
             m = __reduce_max_sync(0xFFFFFFFFu, m);
             if (lane == 0) sm.red[warp] = m;
             __syncthreads();
@@ -245,7 +266,8 @@ __global__ void __launch_bounds__(kQThreads, 2)
             blk_g = e8m0_exponent<FMT>(m);
         }
 
-        // ---- row pass: 1x128 groups along cols -> q
+        // ---- row pass: 1x128 groups along cols -> q.  A half-warp per row,
+        // eight values per thread.
         {
             const int h = lane >> 4, j = lane & 15;
 #pragma unroll 2
@@ -256,12 +278,11 @@ __global__ void __launch_bounds__(kQThreads, 2)
                 bool nan_group;
                 uint32_t g = 0;
                 if constexpr (KIND == kQuantBlockAct) {
-                    uint32_t m = max(max(max_abs_pair(v.x), max_abs_pair(v.y)), max(max_abs_pair(v.z), max_abs_pair(v.w)));
-                    m = max(m, __shfl_xor_sync(0xFFFFFFFFu, m, 8));
-                    m = max(m, __shfl_xor_sync(0xFFFFFFFFu, m, 4));
-                    m = max(m, __shfl_xor_sync(0xFFFFFFFFu, m, 2));
-                    m = max(m, __shfl_xor_sync(0xFFFFFFFFu, m, 1));
-                    g = e8m0_exponent<FMT>(m);
+                    const uint32_t m2 = max_abs4(v);
+                    const uint32_t m = max(m2 & 0xFFFFu, m2 >> 16);
+                    const uint32_t m_lo = __reduce_max_sync(0xFFFFFFFFu, h == 0 ? m : 0u);
+                    const uint32_t m_hi = __reduce_max_sync(0xFFFFFFFFu, h == 1 ? m : 0u);
+                    g = e8m0_exponent<FMT>(h ? m_hi : m_lo);
                     nan_group = (g == 0xFFu);
                     mul = pow2_inv_scale(nan_group ? 0u : g);
                 } else if constexpr (KIND == kQuantBlockWeight) {
@@ -271,54 +292,72 @@ __global__ void __launch_bounds__(kQThreads, 2)
                     nan_group = t_nan;
                     mul = t_scale;
                 }
+                const uint64_t mul2 = f32x2(mul, mul);
                 uint2 out;
-                out.x = quant4<FMT>(v.x, v.y, mul, nan_group);
-                out.y = quant4<FMT>(v.z, v.w, mul, nan_group);
+                out.x = quant4<FMT>(bf16_lo(v.x), bf16_hi(v.x), bf16_lo(v.y), bf16_hi(v.y), mul2, nan_group);
+                out.y = quant4<FMT>(bf16_lo(v.z), bf16_hi(v.z), bf16_lo(v.w), bf16_hi(v.w), mul2, nan_group);
                 *reinterpret_cast<uint2 *>(sm.q_stage + r * kQT + 8 * j) = out;
                 if (KIND == kQuantBlockAct && j == 0) sm.row_g[r] = static_cast<uint8_t>(g);
             }
         }
 
-        // ---- column pass: 128x1 groups along rows -> q_t (transposed)
+        // ---- column pass: 128x1 groups along rows -> q_t (transposed).
+        // Thread t owns columns 2cp, 2cp+1 (cp = t % 64) over the 32 rows of
+        // quarter rq = t / 64: one 4-byte load per row feeds both columns.
         if constexpr (HAS_T) {
-            const int c = tid & 127, hh = tid >> 7;
-            uint32_t vals[32];
+            const int cp = tid & 63, rq = tid >> 6;
+            uint32_t w[32];
 #pragma unroll
-            for (int p = 0; p < 32; ++p) {
-                const int r = 64 * hh + 2 * p;
-                vals[p] = static_cast<uint32_t>(in[r * kQT + c]) | (static_cast<uint32_t>(in[(r + 1) * kQT + c]) << 16);
-            }
-            uint32_t g = 0;
-            float mul;
-            bool nan_group;
+            for (int k = 0; k < 32; ++k) w[k] = *reinterpret_cast<const uint32_t *>(in + (32 * rq + k) * kQT + 2 * cp);
+            float mul_lo, mul_hi;
+            bool nan_lo, nan_hi;
             if constexpr (KIND == kQuantBlockAct) {
-                uint32_t m = 0;
+                uint32_t m2 = 0;
 #pragma unroll
-                for (int p = 0; p < 32; ++p) m = max(m, max_abs_pair(vals[p]));
-                sm.col_amax[hh][c] = m;
+                for (int k = 0; k < 32; ++k) m2 = __vmaxu2(m2, w[k] & 0x7FFF7FFFu);
+                sm.col_amax2[rq][cp] = m2;
                 __syncthreads();  // (S2)
-                m = max(sm.col_amax[0][c], sm.col_amax[1][c]);
-                g = e8m0_exponent<FMT>(m);
-                nan_group = (g == 0xFFu);
-                mul = pow2_inv_scale(nan_group ? 0u : g);
-                if (hh == 0) sm.col_g[c] = static_cast<uint8_t>(g);
+                m2 = __vmaxu2(__vmaxu2(sm.col_amax2[0][cp], sm.col_amax2[1][cp]),
+                              __vmaxu2(sm.col_amax2[2][cp], sm.col_amax2[3][cp]));
+                const uint32_t g_lo = e8m0_exponent<FMT>(m2 & 0xFFFFu), g_hi = e8m0_exponent<FMT>(m2 >> 16);
+                nan_lo = (g_lo == 0xFFu);
+                nan_hi = (g_hi == 0xFFu);
+                mul_lo = pow2_inv_scale(nan_lo ? 0u : g_lo);
+                mul_hi = pow2_inv_scale(nan_hi ? 0u : g_hi);
+                if (rq == 0) {
+                    sm.col_g[2 * cp] = static_cast<uint8_t>(g_lo);
+                    sm.col_g[2 * cp + 1] = static_cast<uint8_t>(g_hi);
+                }
             } else if constexpr (KIND == kQuantBlockWeight) {
-                nan_group = (blk_g == 0xFFu);
-                mul = pow2_inv_scale(nan_group ? 0u : blk_g);
+                nan_lo = nan_hi = (blk_g == 0xFFu);
+                mul_lo = mul_hi = pow2_inv_scale(nan_lo ? 0u : blk_g);
             } else {
-                nan_group = t_nan;
-                mul = t_scale;
+                nan_lo = nan_hi = t_nan;
+                mul_lo = mul_hi = t_scale;
             }
-            uint8_t *row = sm.qt_stage + c * kQT;
+            const uint64_t m2lo = f32x2(mul_lo, mul_lo), m2hi = f32x2(mul_hi, mul_hi);
+            uint32_t c_lo[8], c_hi[8];  // 32 codes of each column, rows 32rq .. 32rq+31
 #pragma unroll
-            for (int ch = 0; ch < 4; ++ch) {
-                uint4 o;
-                o.x = quant4<FMT>(vals[8 * ch + 0], vals[8 * ch + 1], mul, nan_group);
-                o.y = quant4<FMT>(vals[8 * ch + 2], vals[8 * ch + 3], mul, nan_group);
-                o.z = quant4<FMT>(vals[8 * ch + 4], vals[8 * ch + 5], mul, nan_group);
-                o.w = quant4<FMT>(vals[8 * ch + 6], vals[8 * ch + 7], mul, nan_group);
-                const int logical = 4 * hh + ch;
-                *reinterpret_cast<uint4 *>(row + 16 * (logical ^ (c & 7))) = o;
+            for (int q4 = 0; q4 < 8; ++q4) {
+                const uint32_t a = w[4 * q4], b = w[4 * q4 + 1], c = w[4 * q4 + 2], d = w[4 * q4 + 3];
+                c_lo[q4] = quant4<FMT>(bf16_lo(a), bf16_lo(b), bf16_lo(c), bf16_lo(d), m2lo, nan_lo);
+                c_hi[q4] = quant4<FMT>(bf16_hi(a), bf16_hi(b), bf16_hi(c), bf16_hi(d), m2hi, nan_hi);
+            }
+            // Store the two transposed rows; lanes with cp bit 2 set store the
+            // odd row first, so each 8-lane phase touches 8 distinct rows mod 8
+            // (distinct swizzled chunks: no bank conflicts).
+            const int sel = (cp >> 2) & 1;
+#pragma unroll
+            for (int pass = 0; pass < 2; ++pass) {
+                const int which = sel ^ pass;  // 0: column 2cp, 1: column 2cp+1
+                const int row = 2 * cp + which;
+                uint8_t *dst = sm.qt_stage + row * kQT;
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                    const uint4 o = which ? make_uint4(c_hi[4 * i], c_hi[4 * i + 1], c_hi[4 * i + 2], c_hi[4 * i + 3])
+                                          : make_uint4(c_lo[4 * i], c_lo[4 * i + 1], c_lo[4 * i + 2], c_lo[4 * i + 3]);
+                    *reinterpret_cast<uint4 *>(dst + 16 * ((2 * rq + i) ^ (row & 7))) = o;
+                }
             }
         }
 
