@@ -195,6 +195,11 @@ class LinearStack:
             self.dx.append(torch.empty((M, K), dtype=bf, device=device))
             self.dw.append(torch.empty((N, K), dtype=bf, device=device))
         self.xamax = [torch.zeros(1, dtype=torch.int32, device=device) for _ in wl.linears]
+        # scratch for split reductions of small-output GEMMs (Wgrad of qkv / o_proj)
+        ws = max([P.puro_fp8_workspace_size(N, K, M) for _, N, K in wl.linears] +
+                 [P.puro_fp8_workspace_size(M, N, K) for _, N, K in wl.linears] +
+                 [P.puro_fp8_workspace_size(M, K, N) for _, N, K in wl.linears] + [16])
+        self.workspace = torch.empty(ws, dtype=torch.uint8, device=device)
 
     # bytes each quantise launch moves by definition (read bf16, write both
     # FP8 copies and their scales)
@@ -217,6 +222,11 @@ class LinearStack:
               q.colwise.data, q.colwise.scale)
         self.launches_per_step += 1
 
+    def _gemm_launches(self, rows_out, cols_out, red):
+        # one GEMM kernel, plus the reduction kernel when the split schedule is taken
+        ws = self.P.puro_fp8_workspace_size(rows_out, cols_out, red)
+        return 2 if 0 < ws <= self.workspace.numel() else 1
+
     def step(self):
         P, T = self.P, self.timer
         self.launches_per_step = 0
@@ -227,18 +237,18 @@ class LinearStack:
                 xq = P.Quantized(self.xq[j], self.xqt[l][j], self.xamax[j])
                 self._quant(li.x, P.ROLE_ACT, xq)
                 T.run("gemm", 2.0 * self.M * N * K, P.puro_fp8_linear_fprop, self.xq[j], self.wq[l][j].rowwise,
-                      self.y[j])
-                self.launches_per_step += 1
+                      self.y[j], self.workspace)
+                self.launches_per_step += self._gemm_launches(self.M, N, K)
         for l in reversed(range(self.L)):
             for j in reversed(range(len(self.wl.linears))):
                 _, N, K = self.wl.linears[j]
                 li = self.inputs[l][j]
                 self._quant(li.dy, P.ROLE_ACT, self.dyq[j])
                 T.run("gemm", 2.0 * self.M * N * K, P.puro_fp8_linear_dgrad, self.dyq[j].rowwise,
-                      self.wq[l][j].colwise, self.dx[j])
+                      self.wq[l][j].colwise, self.dx[j], self.workspace)
                 T.run("gemm", 2.0 * self.M * N * K, P.puro_fp8_linear_wgrad, self.dyq[j].colwise, self.xqt[l][j],
-                      self.dw[j])
-                self.launches_per_step += 2
+                      self.dw[j], self.workspace)
+                self.launches_per_step += self._gemm_launches(self.M, K, N) + self._gemm_launches(N, K, self.M)
 
     def flops_per_step(self):
         return self.L * sum(6.0 * self.M * N * K for _, N, K in self.wl.linears)
@@ -267,8 +277,8 @@ def bf16_layer_speedup(P, torch, stack):
         for j, (_, N, K) in enumerate(stack.wl.linears):
             P.puro_fp8_linear_fprop(stack.xq[j], stack.wq[0][j].rowwise, stack.y[j])
         for j, (_, N, K) in enumerate(stack.wl.linears):
-            P.puro_fp8_linear_dgrad(stack.dyq[j].rowwise, stack.wq[0][j].colwise, stack.dx[j])
-            P.puro_fp8_linear_wgrad(stack.dyq[j].colwise, stack.xqt[0][j], stack.dw[j])
+            P.puro_fp8_linear_dgrad(stack.dyq[j].rowwise, stack.wq[0][j].colwise, stack.dx[j], stack.workspace)
+            P.puro_fp8_linear_wgrad(stack.dyq[j].colwise, stack.xqt[0][j], stack.dw[j], stack.workspace)
 
     def timeit(fn, reps=5):
         for _ in range(2):
@@ -323,15 +333,15 @@ def e2e_measure(P, torch, stack, steps):
                 stack._quant(li.w, P_.ROLE_WEIGHT, stack.wq[l][j])
                 xq = P_.Quantized(stack.xq[j], stack.xqt[l][j], stack.xamax[j])
                 stack._quant(li.x, P_.ROLE_ACT, xq)
-                P_.puro_fp8_linear_fprop(stack.xq[j], stack.wq[l][j].rowwise, stack.y[j])
+                P_.puro_fp8_linear_fprop(stack.xq[j], stack.wq[l][j].rowwise, stack.y[j], stack.workspace)
         for l in reversed(range(stack.L)):
             for j in reversed(range(len(stack.wl.linears))):
                 li = stack.inputs[l][j]
                 li.dy.copy_(hdy[j], non_blocking=True)
                 h2d += hdy[j].numel() * 2
                 stack._quant(li.dy, P_.ROLE_ACT, stack.dyq[j])
-                P_.puro_fp8_linear_dgrad(stack.dyq[j].rowwise, stack.wq[l][j].colwise, stack.dx[j])
-                P_.puro_fp8_linear_wgrad(stack.dyq[j].colwise, stack.xqt[l][j], stack.dw[j])
+                P_.puro_fp8_linear_dgrad(stack.dyq[j].rowwise, stack.wq[l][j].colwise, stack.dx[j], stack.workspace)
+                P_.puro_fp8_linear_wgrad(stack.dyq[j].colwise, stack.xqt[l][j], stack.dw[j], stack.workspace)
                 hdw[j].copy_(stack.dw[j], non_blocking=True)
                 d2h += stack.dw[j].numel() * 2
 

@@ -153,10 +153,14 @@ puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t cols,
  * Both operands must use the same `scaling`.  BLOCK: all extents multiples
  * of 128.  TENSOR: extents multiples of 16.  A zero reduction extent writes
  * zeros; a zero output extent is a no-op.
- *   workspace, workspace_bytes: optional scratch (may be NULL/0).  When at
- *     least puro_fp8_workspace_size(...) bytes are given, small-output
- *     GEMMs may split the reduction across CTAs; results are the same
- *     within the output tolerance either way.
+ *   workspace, workspace_bytes: optional scratch (may be NULL/0), 16-byte
+ *     aligned.  When the output has fewer 128x256 tiles than the GPU has
+ *     SMs and at least puro_fp8_workspace_size(...) bytes are given, the
+ *     reduction is split into chunks whose FP32 partial tiles go to the
+ *     workspace and are summed (in fixed chunk order, then rounded once to
+ *     BF16) by a second kernel on the same stream.  Results are within the
+ *     output tolerance either way, and deterministic for a given split.
+ *     The workspace is only written, never read before being written.
  *   dev_status: optional device int32, written only on a device-side
  *     timeout (PURO_ERR_TIMEOUT).  The caller zeroes it.
  */
@@ -179,7 +183,8 @@ size_t puro_fp8_scale_bytes(int64_t rows, int64_t red);
 /*
  * Scratch bytes that let a GEMM with output [rows_out, cols_out] and
  * reduction extent `red` use its split-reduction schedule (0 if it never
- * would).  Host-only, no CUDA call.
+ * would): splits * ceil(rows_out/128)*128 * cols_out * 4.  Host-only, no
+ * CUDA call.
  */
 size_t puro_fp8_workspace_size(int64_t rows_out, int64_t cols_out, int64_t red);
 

@@ -82,8 +82,8 @@ puro_status_t check_operand(const puro_fp8_tensor_t *t) {
 }
 
 // D[M,N] = A[M,K] * B[N,K]^T over quantised operands.
-puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, void *d, int32_t *dev_status,
-                       void *stream) {
+puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, void *d, void *workspace,
+                       size_t workspace_bytes, int32_t *dev_status, void *stream) {
     puro_status_t st = check_operand(a);
     if (st != PURO_OK) return st;
     st = check_operand(b);
@@ -121,7 +121,21 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
     g.wait_timeout_ns = g_wait_timeout_ns.load();
     g.num_sms = sm_count();
     if (g.num_sms <= 0) return PURO_ERR_CUDA;
-    return cuda_status(launch_gemm(g, tm_a, tm_b, tm_d, s));
+    g.out = d;
+    g.splits = 1;
+    CUtensorMap tm_ws = tm_d;
+    // Split the reduction across CTAs when the output has too few tiles to
+    // fill the GPU and the caller supplied enough aligned scratch.
+    const int sp = choose_splits(M, N, K, false);
+    if (sp > 1 && workspace && aligned16(workspace) && workspace_bytes >= splitk_workspace_bytes(M, N, K, false)) {
+        const uint64_t m_pad = static_cast<uint64_t>((M + kGemmBM - 1) / kGemmBM * kGemmBM);
+        if (!make_map(&tm_ws, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, workspace, N, static_cast<uint64_t>(sp) * m_pad, N * 4,
+                      32, 32, CU_TENSOR_MAP_SWIZZLE_128B))
+            return PURO_ERR_CUDA;
+        g.splits = sp;
+        g.workspace = workspace;
+    }
+    return cuda_status(launch_gemm(g, tm_a, tm_b, tm_d, tm_ws, s));
 }
 
 puro_status_t bf16_gemm(const void *a, const void *b, void *d, int64_t M, int64_t N, int64_t K,
@@ -146,7 +160,9 @@ puro_status_t bf16_gemm(const void *a, const void *b, void *d, int64_t M, int64_
     g.wait_timeout_ns = g_wait_timeout_ns.load();
     g.num_sms = sm_count();
     if (g.num_sms <= 0) return PURO_ERR_CUDA;
-    return cuda_status(launch_gemm(g, tm_a, tm_b, tm_d, s));
+    g.splits = 1;
+    g.out = d;
+    return cuda_status(launch_gemm(g, tm_a, tm_b, tm_d, tm_d, s));
 }
 
 }  // namespace
@@ -222,32 +238,24 @@ PURO_API puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t co
 PURO_API puro_status_t puro_fp8_linear_fprop(const puro_fp8_tensor_t *x, const puro_fp8_tensor_t *w, void *y,
                                              void *workspace, size_t workspace_bytes, int32_t *dev_status,
                                              void *stream) {
-    (void)workspace;
-    (void)workspace_bytes;
-    return fp8_gemm(x, w, y, dev_status, stream);
+    return fp8_gemm(x, w, y, workspace, workspace_bytes, dev_status, stream);
 }
 
 PURO_API puro_status_t puro_fp8_linear_dgrad(const puro_fp8_tensor_t *dy, const puro_fp8_tensor_t *w_t, void *dx,
                                              void *workspace, size_t workspace_bytes, int32_t *dev_status,
                                              void *stream) {
-    (void)workspace;
-    (void)workspace_bytes;
-    return fp8_gemm(dy, w_t, dx, dev_status, stream);
+    return fp8_gemm(dy, w_t, dx, workspace, workspace_bytes, dev_status, stream);
 }
 
 PURO_API puro_status_t puro_fp8_linear_wgrad(const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t, void *dw,
                                              void *workspace, size_t workspace_bytes, int32_t *dev_status,
                                              void *stream) {
-    (void)workspace;
-    (void)workspace_bytes;
-    return fp8_gemm(dy_t, x_t, dw, dev_status, stream);
+    return fp8_gemm(dy_t, x_t, dw, workspace, workspace_bytes, dev_status, stream);
 }
 
 PURO_API size_t puro_fp8_workspace_size(int64_t rows_out, int64_t cols_out, int64_t red) {
-    (void)rows_out;
-    (void)cols_out;
-    (void)red;
-    return 0;
+    if (rows_out <= 0 || cols_out <= 0 || red <= 0) return 0;
+    return splitk_workspace_bytes(rows_out, cols_out, red, false);
 }
 
 PURO_API size_t puro_fp8_scale_bytes(int64_t rows, int64_t red) {

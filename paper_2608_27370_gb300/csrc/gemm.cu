@@ -40,6 +40,7 @@ constexpr int kSfColsPerSet = 12;  // 4 for A (128 rows) + 8 for B (256 rows)
 constexpr int kSfSets = 2;         // double-buffered across groups of four k-blocks
 constexpr uint64_t kDrainTimeoutNs = 2000000000ull;
 constexpr int32_t kStatusTimeout = 4;  // PURO_ERR_TIMEOUT
+constexpr int64_t kSplitRefSms = 152;  // SM count the split heuristic plans for (GB300)
 
 struct GemmSmem {
     alignas(1024) uint8_t a[kStages][kBM * kBKBytes];
@@ -58,7 +59,11 @@ struct GemmSmem {
 
 struct GemmParams {
     int M, N, K;
-    int num_n, num_kb, num_tiles;
+    int num_m, num_n, num_kb, num_tiles;
+    int splits;        // reduction split into this many chunks (1: no split)
+    int kb_per_split;  // k-blocks per chunk (a multiple of 4)
+    int num_units;     // num_tiles * splits
+    int m_fastest;     // tile order: 1 = row blocks of A vary fastest
     uint32_t idesc;
     const uint8_t *sfa;  // scale vectors of A, [M/128][kgroups][512]
     const uint8_t *sfb;  // scale vectors of B, [N/128][kgroups][512]
@@ -90,7 +95,31 @@ PURO_DEV void record_timeout(GemmSmem &sm, int32_t *status) {
     if (status) atomicExch(status, kStatusTimeout);
 }
 
-template <int KIND>
+// One unit of work: an output tile and a chunk of the reduction.  Units of
+// the same chunk are consecutive; within a chunk the tile order iterates the
+// blocks of the smaller operand fastest, so the CTAs of a wave share (and
+// read once) the blocks of the larger one.
+struct WorkUnit {
+    int m0, n0, kb0, kb1, split;
+};
+
+PURO_DEV WorkUnit work_unit(const GemmParams &p, int u) {
+    WorkUnit w;
+    w.split = u / p.num_tiles;
+    const int tile = u - w.split * p.num_tiles;
+    const int mb = p.m_fastest ? tile % p.num_m : tile / p.num_n;
+    const int nb = p.m_fastest ? tile / p.num_m : tile % p.num_n;
+    w.m0 = mb * kBM;
+    w.n0 = nb * kBN;
+    w.kb0 = w.split * p.kb_per_split;
+    w.kb1 = min(p.num_kb, w.kb0 + p.kb_per_split);
+    return w;
+}
+
+// OUT_F32: write FP32 partial tiles of a split reduction to the workspace
+// [splits * Mp, N], Mp = M rounded up to 128 (rows split * Mp + m), instead
+// of the BF16 output; a ragged last row tile then stays inside its chunk.
+template <int KIND, bool OUT_F32>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tn_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
                    const __grid_constant__ CUtensorMap tm_d, const GemmParams p) {
@@ -139,11 +168,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t stage = 0, phase = 0;
             uint32_t issued = 0;  // stage fills started by this thread
             bool aborted = false;
-            for (int tile = blockIdx.x; tile < p.num_tiles && !aborted; tile += gridDim.x) {
-                const int m0 = (tile / p.num_n) * kBM;
-                const int n0 = (tile % p.num_n) * kBN;
+            for (int u = blockIdx.x; u < p.num_units && !aborted; u += gridDim.x) {
+                const WorkUnit wu = work_unit(p, u);
+                const int m0 = wu.m0, n0 = wu.n0;
                 const bool b_second = n0 + 128 < p.N;  // second 128-row block of B in range
-                for (int kb = 0; kb < p.num_kb; ++kb) {
+                for (int kb = wu.kb0; kb < wu.kb1; ++kb) {
                     if (sm.abort_flag || !mbar_wait_bounded(&sm.empty[stage], phase ^ 1u, p.wait_ns)) {
                         record_timeout(sm, p.status);
                         aborted = true;
@@ -183,7 +212,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t stage = 0, phase = 0;
         bool aborted = false;
         int local = 0;
-        for (int tile = blockIdx.x; tile < p.num_tiles && !aborted; tile += gridDim.x, ++local) {
+        for (int u = blockIdx.x; u < p.num_units && !aborted; u += gridDim.x, ++local) {
+            const WorkUnit wu = work_unit(p, u);
             const int buf = local % kAccBufs;
             const uint32_t acc_phase = static_cast<uint32_t>(local / kAccBufs) & 1u;
             bool ok = (sm.abort_flag == 0) && mbar_wait_bounded(&sm.tempty[buf], acc_phase ^ 1u, p.wait_ns);
@@ -195,7 +225,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after_sync();
             const uint32_t d_tmem = tmem + static_cast<uint32_t>(buf * kBN);
 
-            for (int kb = 0; kb < p.num_kb; ++kb) {
+            for (int kb = wu.kb0; kb < wu.kb1; ++kb) {
                 ok = (sm.abort_flag == 0) && mbar_wait_bounded(&sm.full[stage], phase, p.wait_ns);
                 if (!__all_sync(0xFFFFFFFFu, ok)) {
                     if (lane == 0) record_timeout(sm, p.status);
@@ -223,7 +253,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int k = 0; k < kKSteps; ++k) {
                         const uint64_t ad = smem_desc_k_sw128(a_addr + 32 * k);
                         const uint64_t bd = smem_desc_k_sw128(b_addr + 32 * k);
-                        const uint32_t acc = (kb > 0 || k > 0) ? 1u : 0u;
+                        const uint32_t acc = (kb > wu.kb0 || k > 0) ? 1u : 0u;
                         if constexpr (KIND == kGemmBF16)
                             mma_f16(d_tmem, ad, bd, idesc, acc);
                         else if constexpr (KIND == kGemmFP8Tensor)
@@ -256,9 +286,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if constexpr (KIND == kGemmFP8Tensor) sab = __fmul_rn(*p.sia, *p.sib);
         uint8_t *stage_buf = sm.epi[q];
         int local = 0;
-        for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x, ++local) {
-            const int m0 = (tile / p.num_n) * kBM;
-            const int n0 = (tile % p.num_n) * kBN;
+        for (int u = blockIdx.x; u < p.num_units; u += gridDim.x, ++local) {
+            const WorkUnit wu = work_unit(p, u);
+            const int m0 = wu.m0, n0 = wu.n0;
             const int buf = local % kAccBufs;
             const uint32_t acc_phase = static_cast<uint32_t>(local / kAccBufs) & 1u;
             bool ok = (sm.abort_flag == 0) && mbar_wait_bounded(&sm.tfull[buf], acc_phase, p.wait_ns);
@@ -268,49 +298,89 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_after_sync();
             const uint32_t t_row = tmem + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(buf * kBN);
-            uint32_t packed[kBN / 2];  // the whole 256-column row as bf16 pairs
+            if constexpr (OUT_F32) {
+                // FP32 partial tile: 8 chunks of 32 columns (128 bytes per row)
+                const int row0 = wu.split * p.num_m * kBM + m0 + 32 * q;  // chunks 128-row aligned
 #pragma unroll
-            for (int h = 0; h < kBN / 128; ++h) {
-                uint32_t r[4][32];
+                for (int h = 0; h < kBN / 128; ++h) {
+                    uint32_t r[4][32];
 #pragma unroll
-                for (int c = 0; c < 4; ++c) tmem_ld_32x32b_x32(t_row + 128 * h + 32 * c, r[c]);
-                tmem_ld_wait();
+                    for (int c = 0; c < 4; ++c) tmem_ld_32x32b_x32(t_row + 128 * h + 32 * c, r[c]);
+                    tmem_ld_wait();
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
+                    for (int c = 0; c < 4; ++c) {
+                        const int col = n0 + 128 * h + 32 * c;
+                        if (col >= p.N) break;
+                        if (lane == 0) bulk_wait_group_read0();
+                        __syncwarp();
+                        uint8_t *row = stage_buf + 128 * lane;
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        float lo = __uint_as_float(r[c][2 * i]), hi = __uint_as_float(r[c][2 * i + 1]);
-                        if constexpr (KIND == kGemmFP8Tensor) {
-                            lo = __fmul_rn(lo, sab);
-                            hi = __fmul_rn(hi, sab);
+                        for (int i = 0; i < 8; ++i) {
+                            uint4 v = make_uint4(r[c][4 * i], r[c][4 * i + 1], r[c][4 * i + 2], r[c][4 * i + 3]);
+                            if constexpr (KIND == kGemmFP8Tensor) {
+                                v.x = __float_as_uint(__fmul_rn(__uint_as_float(v.x), sab));
+                                v.y = __float_as_uint(__fmul_rn(__uint_as_float(v.y), sab));
+                                v.z = __float_as_uint(__fmul_rn(__uint_as_float(v.z), sab));
+                                v.w = __float_as_uint(__fmul_rn(__uint_as_float(v.w), sab));
+                            }
+                            *reinterpret_cast<uint4 *>(row + 16 * (i ^ (lane & 7))) = v;
                         }
-                        __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-                        packed[64 * h + 16 * c + i] = *reinterpret_cast<uint32_t *>(&v);
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) {
+                            tma_store_2d(&tm_d, stage_buf, col, row0);
+                            bulk_commit_group();
+                        }
                     }
                 }
-            }
-            tc_fence_before_sync();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&sm.tempty[buf]);  // accumulator free for the next tile
-            // Store 4 chunks of 64 columns (128 bytes per row) through the
-            // per-warp staging tile, 16-byte chunk i of row l at i ^ (l % 8).
-#pragma unroll
-            for (int ch = 0; ch < kBN / 64; ++ch) {
-                if (n0 + 64 * ch >= p.N) break;
-                if (lane == 0) bulk_wait_group_read0();
+                tc_fence_before_sync();
                 __syncwarp();
-                uint8_t *row = stage_buf + 128 * lane;
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const uint4 v = make_uint4(packed[32 * ch + 4 * i], packed[32 * ch + 4 * i + 1],
-                                               packed[32 * ch + 4 * i + 2], packed[32 * ch + 4 * i + 3]);
-                    *reinterpret_cast<uint4 *>(row + 16 * (i ^ (lane & 7))) = v;
+                if (lane == 0) mbar_arrive(&sm.tempty[buf]);
+            } else {
+                uint32_t packed[kBN / 2];  // the whole 256-column row as bf16 pairs
+    #pragma unroll
+                for (int h = 0; h < kBN / 128; ++h) {
+                    uint32_t r[4][32];
+    #pragma unroll
+                    for (int c = 0; c < 4; ++c) tmem_ld_32x32b_x32(t_row + 128 * h + 32 * c, r[c]);
+                    tmem_ld_wait();
+    #pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+    #pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            float lo = __uint_as_float(r[c][2 * i]), hi = __uint_as_float(r[c][2 * i + 1]);
+                            if constexpr (KIND == kGemmFP8Tensor) {
+                                lo = __fmul_rn(lo, sab);
+                                hi = __fmul_rn(hi, sab);
+                            }
+                            __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+                            packed[64 * h + 16 * c + i] = *reinterpret_cast<uint32_t *>(&v);
+                        }
+                    }
                 }
-                fence_proxy_async_smem();
+                tc_fence_before_sync();
                 __syncwarp();
-                if (lane == 0) {
-                    tma_store_2d(&tm_d, stage_buf, n0 + 64 * ch, m0 + 32 * q);
-                    bulk_commit_group();
+                if (lane == 0) mbar_arrive(&sm.tempty[buf]);  // accumulator free for the next tile
+                // Store 4 chunks of 64 columns (128 bytes per row) through the
+                // per-warp staging tile, 16-byte chunk i of row l at i ^ (l % 8).
+    #pragma unroll
+                for (int ch = 0; ch < kBN / 64; ++ch) {
+                    if (n0 + 64 * ch >= p.N) break;
+                    if (lane == 0) bulk_wait_group_read0();
+                    __syncwarp();
+                    uint8_t *row = stage_buf + 128 * lane;
+    #pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const uint4 v = make_uint4(packed[32 * ch + 4 * i], packed[32 * ch + 4 * i + 1],
+                                                   packed[32 * ch + 4 * i + 2], packed[32 * ch + 4 * i + 3]);
+                        *reinterpret_cast<uint4 *>(row + 16 * (i ^ (lane & 7))) = v;
+                    }
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_2d(&tm_d, stage_buf, n0 + 64 * ch, m0 + 32 * q);
+                        bulk_commit_group();
+                    }
                 }
             }
         }
@@ -326,19 +396,75 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-template <int KIND>
+// Split-K reduction: out[i] = bf16(sum_s ws[s][i]) in fixed order s = 0, 1, ...
+// (chunk s starts split_stride4 float4s after chunk s-1).
+__global__ void __launch_bounds__(256) splitk_reduce_kernel(const float4 *__restrict__ ws, int splits, int64_t n4,
+                                                            int64_t split_stride4, uint2 *__restrict__ out) {
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
+        float4 a = ws[i];
+        for (int sp = 1; sp < splits; ++sp) {
+            const float4 b = ws[sp * split_stride4 + i];
+            a.x += b.x;
+            a.y += b.y;
+            a.z += b.z;
+            a.w += b.w;
+        }
+        __nv_bfloat162 lo = __floats2bfloat162_rn(a.x, a.y), hi = __floats2bfloat162_rn(a.z, a.w);
+        out[i] = make_uint2(*reinterpret_cast<uint32_t *>(&lo), *reinterpret_cast<uint32_t *>(&hi));
+    }
+}
+
+int choose_splits(int64_t M, int64_t N, int64_t K, bool bf16) {
+    if (bf16) return 1;
+    const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + kBN - 1) / kBN);
+    const int64_t kblocks = (K + kBKBytes - 1) / kBKBytes;
+    if (tiles >= kSplitRefSms) return 1;
+    // Modelled time = waves x k-blocks per chunk; chunks keep >= 16 k-blocks
+    // (whole groups of four).  Split only for a >= 15% modelled gain.
+    auto cost = [&](int64_t sp) {
+        const int64_t chunk = ((kblocks + sp - 1) / sp + 3) / 4 * 4;
+        const int64_t chunks = (kblocks + chunk - 1) / chunk;
+        return ((tiles * chunks + kSplitRefSms - 1) / kSplitRefSms) * chunk;
+    };
+    const int64_t base = cost(1);
+    int best = 1;
+    int64_t best_cost = base;
+    for (int sp = 2; sp <= 8; ++sp) {
+        if (kblocks / sp < 16) break;
+        const int64_t c = cost(sp);
+        if (c < best_cost) {
+            best = sp;
+            best_cost = c;
+        }
+    }
+    return (best_cost * 100 <= base * 85) ? best : 1;
+}
+
+size_t splitk_workspace_bytes(int64_t M, int64_t N, int64_t K, bool bf16) {
+    const int sp = choose_splits(M, N, K, bf16);
+    const int64_t m_pad = (M + kBM - 1) / kBM * kBM;
+    return sp > 1 ? static_cast<size_t>(sp) * static_cast<size_t>(m_pad) * static_cast<size_t>(N) * sizeof(float) : 0;
+}
+
+template <int KIND, bool OUT_F32>
 static cudaError_t launch_kind(const GemmArgs &g, const CUtensorMap &tm_a, const CUtensorMap &tm_b,
-                               const CUtensorMap &tm_d, cudaStream_t s) {
+                               const CUtensorMap &tm_d, int splits, cudaStream_t s) {
     constexpr int kElemBytes = (KIND == kGemmBF16) ? 2 : 1;
     constexpr int kBK = kBKBytes / kElemBytes;
     GemmParams p{};
     p.M = static_cast<int>(g.M);
     p.N = static_cast<int>(g.N);
     p.K = static_cast<int>(g.K);
+    p.num_m = static_cast<int>((g.M + kBM - 1) / kBM);
     p.num_n = static_cast<int>((g.N + kBN - 1) / kBN);
-    const int num_m = static_cast<int>((g.M + kBM - 1) / kBM);
     p.num_kb = static_cast<int>((g.K + kBK - 1) / kBK);
-    p.num_tiles = num_m * p.num_n;
+    p.num_tiles = p.num_m * p.num_n;
+    p.splits = splits;
+    p.kb_per_split = ((p.num_kb + splits - 1) / splits + 3) / 4 * 4;
+    p.splits = (p.num_kb + p.kb_per_split - 1) / p.kb_per_split;  // no empty chunk
+    p.num_units = p.num_tiles * p.splits;
+    p.m_fastest = g.M < g.N ? 1 : 0;  // re-read the smaller operand, stream the larger once
     if (KIND == kGemmBF16)
         p.idesc = idesc_dense(1u, 1u);
     else if (KIND == kGemmFP8Tensor)
@@ -353,21 +479,37 @@ static cudaError_t launch_kind(const GemmArgs &g, const CUtensorMap &tm_a, const
     p.status = g.status;
     p.wait_ns = g.wait_timeout_ns;
 
-    auto kern = gemm_tn_kernel<KIND>;
+    auto kern = gemm_tn_kernel<KIND, OUT_F32>;
     const size_t smem = sizeof(GemmSmem) + 1024;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    const int grid = p.num_tiles < g.num_sms ? p.num_tiles : g.num_sms;
+    const int grid = p.num_units < g.num_sms ? p.num_units : g.num_sms;
     kern<<<grid, kThreads, smem, s>>>(tm_a, tm_b, tm_d, p);
     return cudaGetLastError();
 }
 
+template <int KIND>
+static cudaError_t launch_split_or_not(const GemmArgs &g, const CUtensorMap &tm_a, const CUtensorMap &tm_b,
+                                       const CUtensorMap &tm_d, const CUtensorMap &tm_ws, cudaStream_t s) {
+    if (g.splits <= 1) return launch_kind<KIND, false>(g, tm_a, tm_b, tm_d, 1, s);
+    cudaError_t e = launch_kind<KIND, true>(g, tm_a, tm_b, tm_ws, g.splits, s);
+    if (e != cudaSuccess) return e;
+    const int64_t n4 = g.M * g.N / 4;
+    const int64_t stride4 = (g.M + kBM - 1) / kBM * kBM * g.N / 4;
+    int64_t want = (n4 + 255) / 256;
+    const int64_t cap = static_cast<int64_t>(g.num_sms) * 8;
+    const int grid = static_cast<int>(want < cap ? want : cap);
+    splitk_reduce_kernel<<<grid, 256, 0, s>>>(reinterpret_cast<const float4 *>(g.workspace), g.splits, n4, stride4,
+                                              reinterpret_cast<uint2 *>(g.out));
+    return cudaGetLastError();
+}
+
 cudaError_t launch_gemm(const GemmArgs &g, const CUtensorMap &tm_a, const CUtensorMap &tm_b,
-                        const CUtensorMap &tm_d, cudaStream_t s) {
+                        const CUtensorMap &tm_d, const CUtensorMap &tm_ws, cudaStream_t s) {
     switch (g.kind) {
-        case kGemmBF16: return launch_kind<kGemmBF16>(g, tm_a, tm_b, tm_d, s);
-        case kGemmFP8Tensor: return launch_kind<kGemmFP8Tensor>(g, tm_a, tm_b, tm_d, s);
-        default: return launch_kind<kGemmFP8Block>(g, tm_a, tm_b, tm_d, s);
+        case kGemmBF16: return launch_kind<kGemmBF16, false>(g, tm_a, tm_b, tm_d, 1, s);
+        case kGemmFP8Tensor: return launch_split_or_not<kGemmFP8Tensor>(g, tm_a, tm_b, tm_d, tm_ws, s);
+        default: return launch_split_or_not<kGemmFP8Block>(g, tm_a, tm_b, tm_d, tm_ws, s);
     }
 }
 

@@ -59,12 +59,24 @@ struct GemmArgs {
     int32_t *status;             // optional device status word
     uint64_t wait_timeout_ns;
     int num_sms;
+    // split reduction (FP8 kinds only): splits > 1 needs `workspace` of
+    // splitk_workspace_bytes(M, N, K) bytes; `out` is D (bf16)
+    int splits;
+    void *workspace;
+    void *out;
 };
 
 // tm_a: A [M, K], tm_b: B [N, K] (128-byte swizzle, box {128 bytes, rows}),
-// tm_d: D [M, N] bf16 (128-byte swizzle, box {64, 32}).
+// tm_d: D [M, N] bf16 (128-byte swizzle, box {64, 32}),
+// tm_ws: workspace [splits * M, N] fp32 (128-byte swizzle, box {32, 32});
+// only read when g.splits > 1.
 cudaError_t launch_gemm(const GemmArgs &g, const CUtensorMap &tm_a, const CUtensorMap &tm_b,
-                        const CUtensorMap &tm_d, cudaStream_t s);
+                        const CUtensorMap &tm_d, const CUtensorMap &tm_ws, cudaStream_t s);
+
+// Split count the GEMM uses for a shape (1: no split), and the workspace it
+// then needs.  Host-only, shape-only (plans for 152 SMs).
+int choose_splits(int64_t M, int64_t N, int64_t K, bool bf16);
+size_t splitk_workspace_bytes(int64_t M, int64_t N, int64_t K, bool bf16);
 
 // Tile shape of the GEMM kernel (rows of A per CTA tile, rows of B).
 constexpr int kGemmBM = 128;

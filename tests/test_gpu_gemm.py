@@ -115,3 +115,30 @@ def test_gemm_status_word_stays_clear_on_success():
     x, w, dy = _inputs(M, N, K, 91)
     out = run_linear(x, w, dy, P.SCALE_BLOCK)  # asserts the status word is 0
     assert torch.isfinite(out["y"].float()).all()
+
+
+@pytest.mark.parametrize("scaling,M,N,K", [(P.SCALE_BLOCK, 8192, 256, 256), (P.SCALE_BLOCK, 4096, 384, 1536),
+                                           (P.SCALE_TENSOR, 4112, 400, 208)])
+def test_wgrad_split_reduction(scaling, M, N, K):
+    """Small-output Wgrad with a long reduction (tokens): with a workspace
+    the reduction is split across CTAs (FP32 partials + a fixed-order sum);
+    both schedules must meet the tolerance against the oracle."""
+    x, w, dy = _inputs(M, N, K, 4000 + M + N, t3=True)
+    xq = P.quantize(x, P.E4M3, scaling, P.ROLE_ACT)
+    dyq = P.quantize(dy, P.E4M3, scaling, P.ROLE_ACT)
+    ws_bytes = P.puro_fp8_workspace_size(N, K, M)
+    assert ws_bytes > 0, "this shape should take the split schedule"
+    ws = torch.full((ws_bytes,), 0xFF, dtype=torch.uint8, device=DEV)  # NaN garbage: must be overwritten
+    dw_split = torch.empty((N, K), dtype=torch.bfloat16, device=DEV)
+    dw_plain = torch.empty((N, K), dtype=torch.bfloat16, device=DEV)
+    P.puro_fp8_linear_wgrad(dyq.colwise, xq.colwise, dw_split, workspace=ws)
+    P.puro_fp8_linear_wgrad(dyq.colwise, xq.colwise, dw_plain)
+    torch.cuda.synchronize()
+    ref = oracle_linear(x, w, dy, scaling)["dw"]
+    assert_close(dw_split, ref, "wgrad (split reduction)")
+    assert_close(dw_plain, ref, "wgrad (single pass)")
+    # too small a workspace silently falls back to the single-pass schedule
+    dw_small = torch.empty((N, K), dtype=torch.bfloat16, device=DEV)
+    P.puro_fp8_linear_wgrad(dyq.colwise, xq.colwise, dw_small, workspace=ws[: ws_bytes // 2])
+    torch.cuda.synchronize()
+    assert torch.equal(dw_small.view(torch.int16), dw_plain.view(torch.int16))

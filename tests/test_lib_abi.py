@@ -135,6 +135,16 @@ def test_scale_buffer_size(lib):
     assert int(np.prod(P.scale_vec_shape(256, 8960))) == lib.puro_fp8_scale_bytes(256, 8960)
 
 
+def test_workspace_size_plans_split_reductions(lib):
+    # Wgrad of qkv / o_proj at 32768 tokens: 96 / 72 output tiles < 152 SMs
+    assert lib.puro_fp8_workspace_size(2048, 1536, 32768) == 3 * 2048 * 1536 * 4
+    assert lib.puro_fp8_workspace_size(1536, 1536, 32768) == 2 * 1536 * 1536 * 4
+    # enough tiles, or too short a reduction: no split
+    assert lib.puro_fp8_workspace_size(17920, 1536, 32768) == 0
+    assert lib.puro_fp8_workspace_size(1536, 1536, 256) == 0
+    assert lib.puro_fp8_workspace_size(0, 1536, 32768) == 0
+
+
 def test_get_status_validation(lib):
     out = ctypes.c_int32(0)
     assert lib.puro_fp8_get_status(None, ctypes.byref(out), None) == BAD
