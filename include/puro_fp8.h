@@ -175,6 +175,37 @@ puro_status_t puro_fp8_linear_wgrad(const puro_fp8_tensor_t *dy_t, const puro_fp
                                     int32_t *dev_status, void *stream);
 
 /*
+ * Wgrad without allocation and without caller-supplied scratch.
+ *
+ * The paper has no counterpart to this entry point; it serves callers that
+ * cannot allocate device memory while they run the backward pass -- plugin
+ * hosts that own every device buffer and forbid allocations in their
+ * execution callbacks, latency-critical code that cannot afford
+ * cudaMalloc's device-wide synchronisation, or callers with a fixed memory
+ * budget -- and so cannot provide the scratch puro_fp8_linear_wgrad's
+ * split-reduction schedule wants.
+ *
+ * Same operands, output and results as puro_fp8_linear_wgrad with a large
+ * enough workspace.  The scratch is a fixed PURO_NOALLOC_SCRATCH_BYTES
+ * (40 MiB) array inside the library's device image, held by every GPU that
+ * loads the library until the process exits; no cudaMalloc, cudaFree or
+ * allocating library call is made.
+ *   - A shape whose split schedule needs more than PURO_NOALLOC_SCRATCH_BYTES
+ *     (see puro_fp8_workspace_size) returns PURO_ERR_UNSUPPORTED before any
+ *     work is enqueued.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current and caches it; make
+ *     that first call before any stream capture begins.
+ *   - All calls share the one array, which keeps the last call's contents.
+ *     Nothing in it needs to start at zero: each call writes every scratch
+ *     byte before reading it.  Calls whose executions overlap on the GPU
+ *     (different streams without ordering) race on the array: order them.
+ */
+#define PURO_NOALLOC_SCRATCH_BYTES (40u * 1024u * 1024u)
+puro_status_t puro_fp8_linear_wgrad_noalloc(const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t, void *dw,
+                                            int32_t *dev_status, void *stream);
+
+/*
  * Bytes of a PURO_SCALE_BLOCK scale buffer for an operand [rows, red]
  * (rows * ceil(red/512) * 4).  Host-only, no CUDA call.
  */

@@ -70,6 +70,7 @@ _SIGNATURES = {
     "puro_fp8_linear_fprop": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_dgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_wgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
+    "puro_fp8_linear_wgrad_noalloc": (_I32, [_P, _P, _P, _P, _P]),
     "puro_fp8_workspace_size": (ctypes.c_size_t, [_I64, _I64, _I64]),
     "puro_fp8_scale_bytes": (ctypes.c_size_t, [_I64, _I64]),
     "puro_fp8_get_status": (_I32, [_P, _P, _P]),
@@ -200,6 +201,19 @@ def puro_fp8_linear_wgrad(dy_t: FP8Operand, x_t: FP8Operand, dw: torch.Tensor, w
                           stream=None) -> None:
     """dW [N,K] = dY^T [N,M] . X [M,K] (operands dY^T [N,M], X^T [K,M])."""
     _gemm("puro_fp8_linear_wgrad", dy_t, x_t, dw, workspace, dev_status, stream)
+
+
+def puro_fp8_linear_wgrad_noalloc(dy_t: FP8Operand, x_t: FP8Operand, dw: torch.Tensor, dev_status=None,
+                                  stream=None) -> None:
+    """dW [N,K] = dY^T X without allocating and without caller scratch: for
+    callers that cannot obtain device memory while running the backward
+    pass.  The split-reduction scratch is a fixed 40 MiB array inside the
+    library (see the header for the limits and ordering rules)."""
+    ca, cb = dy_t.as_c(), x_t.as_c()
+    st = load_library().puro_fp8_linear_wgrad_noalloc(ctypes.byref(ca), ctypes.byref(cb),
+                                                      _ptr(dw, torch.bfloat16, "dw"),
+                                                      _ptr(dev_status, torch.int32, "dev_status"), _stream(stream))
+    _check("puro_fp8_linear_wgrad_noalloc", st)
 
 
 def puro_fp8_workspace_size(rows_out: int, cols_out: int, red: int) -> int:

@@ -166,6 +166,12 @@ puro_status_t bf16_gemm(const void *a, const void *b, void *d, int64_t M, int64_
 }
 
 }  // namespace
+
+puro_status_t fp8_gemm_entry(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, void *d, void *workspace,
+                             size_t workspace_bytes, int32_t *dev_status, void *stream) {
+    return fp8_gemm(a, b, d, workspace, workspace_bytes, dev_status, stream);
+}
+
 }  // namespace puro
 
 using namespace puro;

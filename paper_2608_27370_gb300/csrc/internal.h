@@ -7,6 +7,8 @@
 #include <cstddef>
 #include <cstdint>
 
+#include "puro_fp8.h"
+
 namespace puro {
 
 // How a quantiser groups values (section "FP8 Mixed-Precision Training").
@@ -72,6 +74,11 @@ struct GemmArgs {
 // only read when g.splits > 1.
 cudaError_t launch_gemm(const GemmArgs &g, const CUtensorMap &tm_a, const CUtensorMap &tm_b,
                         const CUtensorMap &tm_d, const CUtensorMap &tm_ws, cudaStream_t s);
+
+// The FP8 GEMM entry behind puro_fp8_linear_{fprop,dgrad,wgrad}: validates,
+// encodes the tensor maps and launches (D = A * B^T).
+puro_status_t fp8_gemm_entry(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, void *d, void *workspace,
+                             size_t workspace_bytes, int32_t *dev_status, void *stream);
 
 // Split count the GEMM uses for a shape (1: no split), and the workspace it
 // then needs.  Host-only, shape-only (plans for 152 SMs).
