@@ -228,8 +228,10 @@ PURO_API puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t co
         return PURO_OK;
     }
     a.x = static_cast<const uint16_t *>(x);
-    CUtensorMap tm_q, tm_qt;
-    if (!make_map(&tm_q, CU_TENSOR_MAP_DATA_TYPE_UINT8, q, cols, rows, cols, 128, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
+    CUtensorMap tm_x, tm_q, tm_qt;
+    if (!make_map(&tm_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, x, cols, rows, cols * 2, 128, 128,
+                  CU_TENSOR_MAP_SWIZZLE_NONE) ||
+        !make_map(&tm_q, CU_TENSOR_MAP_DATA_TYPE_UINT8, q, cols, rows, cols, 128, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
         return PURO_ERR_CUDA;
     if (has_t) {
         if (!make_map(&tm_qt, CU_TENSOR_MAP_DATA_TYPE_UINT8, q_t, rows, cols, rows, 128, 128,
@@ -238,7 +240,7 @@ PURO_API puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t co
     } else {
         tm_qt = tm_q;
     }
-    return cuda_status(launch_quantize(a, tm_q, tm_qt, static_cast<cudaStream_t>(stream)));
+    return cuda_status(launch_quantize(a, tm_x, tm_q, tm_qt, static_cast<cudaStream_t>(stream)));
 }
 
 PURO_API puro_status_t puro_fp8_linear_fprop(const puro_fp8_tensor_t *x, const puro_fp8_tensor_t *w, void *y,

@@ -33,10 +33,11 @@ struct QuantArgs {
 
 cudaError_t launch_amax(const uint16_t *x, int64_t n, uint32_t *amax, cudaStream_t s);
 
+// tm_x: bf16 [rows, cols], box {128, 128}, no swizzle.
 // tm_q: u8 [rows, cols], box {128, 128}, no swizzle.
 // tm_qt: u8 [cols, rows], box {128, 128}, 128-byte swizzle (only if has_t).
-cudaError_t launch_quantize(const QuantArgs &a, const CUtensorMap &tm_q, const CUtensorMap &tm_qt,
-                            cudaStream_t s);
+cudaError_t launch_quantize(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
+                            const CUtensorMap &tm_qt, cudaStream_t s);
 
 // Writes only the per-tensor scale_inv (used for empty tensors).
 cudaError_t launch_tensor_scale_only(const QuantArgs &a, cudaStream_t s);

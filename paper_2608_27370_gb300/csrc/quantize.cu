@@ -5,7 +5,7 @@
 // 128x128 blocks for weights -- each a power of two).
 //
 // Both kernels are HBM-bandwidth bound.  The cast kernel reads each 128x128
-// BF16 tile once (cp.async, double buffered), computes the row-group and the
+// BF16 tile once (one TMA load per tile, double buffered), computes the row-group and the
 // column-group scales from the same shared-memory copy, and writes the
 // rowwise codes and the transposed codes through shared memory with TMA
 // stores (the transposed staging tile uses the 128-byte swizzle so the
@@ -175,48 +175,55 @@ PURO_DEV void store_scale_vec(uint8_t *__restrict__ base, int64_t row, int64_t k
 constexpr int kQT = 128;          // tile edge
 constexpr int kQThreads = 256;
 
+// Shared memory of one CTA.  Both staging tiles are TMA store sources and
+// so 1024-byte aligned; the transposed tile uses the 128-byte swizzle
+// (16-byte chunk k of row r at k ^ (r % 8)).
 struct QuantSmem {
-    alignas(1024) uint8_t qt_stage[kQT * kQT];    // transposed codes, 128B-swizzled rows
-    alignas(1024) uint8_t q_stage[kQT * kQT];     // rowwise codes, plain rows
-    alignas(128) uint16_t in[2][kQT * kQT];       // bf16 tile, double buffered
-    uint32_t col_amax2[4][kQT / 2];  // per row quarter, two columns per word
+    alignas(1024) uint8_t q_stage[kQT * kQT];    // rowwise codes, plain rows
+    alignas(1024) uint8_t qt_stage[kQT * kQT];   // transposed codes, 128B-swizzled rows
+    alignas(128) uint16_t in[2][kQT * kQT];                // bf16 tile, double buffered
+    uint32_t row_part[kQT / 2][16];   // [row pair][column block]: 16-bit row maxima, two rows per word
+    uint32_t col_part[16][kQT / 2];   // [row block][column pair]: 16-bit column maxima, two columns per word
+    alignas(16) float row_mul[kQT];   // 2^(127-g) per row (NaN marks a non-finite group)
+    alignas(16) float col_mul[kQT];   // 2^(127-g) per column
     uint32_t red[8];
     alignas(16) uint8_t row_g[kQT];
     alignas(16) uint8_t col_g[kQT];
+    uint64_t full[2];                 // TMA tile loads into in[0], in[1]
 };
 
-PURO_DEV void load_tile_async(uint16_t *dst, const uint16_t *__restrict__ x, int64_t rows, int64_t cols,
-                              int64_t r0, int64_t c0) {
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        const int k = threadIdx.x + kQThreads * i;  // 16-byte chunk id in the tile
-        const int r = k >> 4, cc = (k & 15) * 8;
-        const int64_t gr = r0 + r, gc = c0 + cc;
-        const bool ok = (gr < rows) && (gc < cols);
-        const uint16_t *src = ok ? x + gr * cols + gc : x;
-        cp_async_16(dst + r * kQT + cc, src, ok ? 16u : 0u);
-    }
-    cp_async_commit();
-}
+constexpr uint64_t kQuantWaitNs = 2000000000ull;  // a TMA load always lands long before this
 
+// 2^(127-g) for a scale exponent, NaN for the non-finite marker 0xFF.
+PURO_DEV float mul_of(uint32_t g) { return g == 0xFFu ? __uint_as_float(0x7FC00000u) : pow2_inv_scale(g); }
+
+// Tile kernel: each thread owns one 8x8 block of the 128x128 tile (rows
+// 8*br .. 8*br+7, columns 8*bc .. 8*bc+7; a warp holds two block rows of 16
+// blocks).  It loads the block once and produces both its rowwise codes
+// (q) and its transposed codes (q_t) from the same registers:
+//   A  partial maxima of its 8 rows and 8 columns -> shared memory
+//   B  128 threads finish the 128 row scales and 128 column scales
+//   C  every thread quantises its block twice (row scales, column scales)
 template <int FMT, int KIND, bool HAS_T>
 __global__ void __launch_bounds__(kQThreads, 2)
-    quant_tile_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_qt,
-                      const uint16_t *__restrict__ x, int64_t rows, int64_t cols,
+    quant_tile_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_q,
+                      const __grid_constant__ CUtensorMap tm_qt, int64_t rows, int64_t cols,
                       uint8_t *__restrict__ scale_u8, uint8_t *__restrict__ scale_t_u8, float *scale_f,
                       float *scale_t_f, const uint32_t *__restrict__ amax_bits, int tiles_n, int ntiles) {
     extern __shared__ uint8_t smem_raw[];
     QuantSmem &sm = *reinterpret_cast<QuantSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                    ~static_cast<uintptr_t>(1023));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int br = 2 * warp + (lane >> 4);  // block row: tile rows 8br .. 8br+7
+    const int bc = lane & 15;               // block column: tile columns 8bc .. 8bc+7
 
     // Per-tensor mode: the one scale, from the device amax.
-    float t_scale = 1.0f;
-    bool t_nan = false;
+    float t_mul = 1.0f;
     if constexpr (KIND == kQuantTensor) {
         const uint32_t a = *amax_bits & 0xFFFFu;
-        t_nan = a >= 0x7F80u;
-        t_scale = tensor_scale<FMT>(a);
+        const bool t_nan = a >= 0x7F80u;
+        const float t_scale = tensor_scale<FMT>(a);
+        t_mul = t_nan ? __uint_as_float(0x7FC00000u) : t_scale;
         if (blockIdx.x == 0 && tid == 0) {
             const float si = t_nan ? __uint_as_float(0x7FC00000u) : __fdiv_rn(1.0f, t_scale);
             *scale_f = si;
@@ -224,145 +231,173 @@ __global__ void __launch_bounds__(kQThreads, 2)
         }
     }
     if (tid == 0) {
+        mbar_init(&sm.full[0], 1);
+        mbar_init(&sm.full[1], 1);
+        fence_mbarrier_init();
+        tma_prefetch_desc(&tm_x);
         tma_prefetch_desc(&tm_q);
         if (HAS_T) tma_prefetch_desc(&tm_qt);
     }
+    __syncthreads();
 
+    // One TMA load per 128x128 bf16 tile (out-of-range parts read as zero),
+    // double buffered: tile it+1 streams in while tile it is processed.
+    auto issue_load = [&](int t, int b) {
+        mbar_arrive_expect_tx(&sm.full[b], kQT * kQT * 2);
+        tma_load_2d(sm.in[b], &tm_x, &sm.full[b], (t % tiles_n) * kQT, (t / tiles_n) * kQT);
+    };
     int tile = blockIdx.x;
-    if (tile < ntiles)
-        load_tile_async(sm.in[0], x, rows, cols, static_cast<int64_t>(tile / tiles_n) * kQT,
-                        static_cast<int64_t>(tile % tiles_n) * kQT);
+    if (tid == 0 && tile < ntiles) issue_load(tile, 0);
     for (int it = 0; tile < ntiles; ++it, tile += gridDim.x) {
         const int buf = it & 1;
         const int64_t r0 = static_cast<int64_t>(tile / tiles_n) * kQT;
         const int64_t c0 = static_cast<int64_t>(tile % tiles_n) * kQT;
-        const int next = tile + gridDim.x;
-        if (next < ntiles)
-            load_tile_async(sm.in[buf ^ 1], x, rows, cols, static_cast<int64_t>(next / tiles_n) * kQT,
-                            static_cast<int64_t>(next % tiles_n) * kQT);
-        else
-            cp_async_commit();
-        cp_async_wait<1>();
-        if (tid == 0) bulk_wait_group_read0();  // previous tile's stores have read the staging
-        __syncthreads();                         // (S1) tile visible, staging free
+        if (tid == 0) {
+            const int next = tile + gridDim.x;
+            if (next < ntiles) issue_load(next, buf ^ 1);  // its buffer was last read before (S2) of it-1
+            bulk_wait_group_read0();                        // previous tile's stores have read the staging
+        }
+        mbar_wait_bounded(&sm.full[buf], static_cast<uint32_t>(it >> 1) & 1u, kQuantWaitNs);
+        __syncthreads();                                    // (S1) staging free
 
+        // ---- the thread's 8x8 block: v[i] = row 8br+i, columns 8bc .. 8bc+7
         const uint16_t *in = sm.in[buf];
+        uint4 v[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[i] = *reinterpret_cast<const uint4 *>(in + (8 * br + i) * kQT + 8 * bc);
 
-        // ---- 128x128 block scale (weights): amax over the whole tile
-        uint32_t blk_g = 0;
-        if constexpr (KIND == kQuantBlockWeight) {
+        // ---- A: partial maxima
+        if constexpr (KIND == kQuantBlockAct) {
+#pragma unroll
+            for (int p = 0; p < 4; ++p) {  // row pair (2p, 2p+1) -> one word
+                const uint32_t m0 = max_abs4(v[2 * p]), m1 = max_abs4(v[2 * p + 1]);
+                const uint32_t a0 = max(m0 & 0xFFFFu, m0 >> 16), a1 = max(m1 & 0xFFFFu, m1 >> 16);
+                sm.row_part[4 * br + p][bc] = a0 | (a1 << 16);
+            }
+            uint4 cm;  // column pair k: max over the 8 rows, 16 bits per column
+            cm.x = cm.y = cm.z = cm.w = 0u;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                cm.x = __vmaxu2(cm.x, v[i].x & 0x7FFF7FFFu);
+                cm.y = __vmaxu2(cm.y, v[i].y & 0x7FFF7FFFu);
+                cm.z = __vmaxu2(cm.z, v[i].z & 0x7FFF7FFFu);
+                cm.w = __vmaxu2(cm.w, v[i].w & 0x7FFF7FFFu);
+            }
+            *reinterpret_cast<uint4 *>(&sm.col_part[br][4 * bc]) = cm;
+        } else if constexpr (KIND == kQuantBlockWeight) {
             uint32_t m = 0;
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const uint4 v = *reinterpret_cast<const uint4 *>(in + (tid + kQThreads * i) * 8);
-                m = __vmaxu2(m, max_abs4(v));
-            }
-            m = max(m & 0xFFFFu, m >> 16);
-            m = __reduce_max_sync(0xFFFFFFFFu, m);
+            for (int i = 0; i < 8; ++i) m = __vmaxu2(m, max_abs4(v[i]));
+            m = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
             if (lane == 0) sm.red[warp] = m;
-            __syncthreads();
-            m = sm.red[lane & 7];
-            m = __reduce_max_sync(0xFFFFFFFFu, m);
-            blk_g = e8m0_exponent<FMT>(m);
         }
+        if constexpr (KIND != kQuantTensor) __syncthreads();  // (S2) partials written
 
-        // ---- row pass: 1x128 groups along cols -> q.  A half-warp per row,
-        // eight values per thread.
-        {
-            const int h = lane >> 4, j = lane & 15;
-#pragma unroll 2
-            for (int i = 0; i < 8; ++i) {
-                const int r = 16 * warp + 2 * i + h;
-                const uint4 v = *reinterpret_cast<const uint4 *>(in + r * kQT + 8 * j);
-                float mul;
-                bool nan_group;
-                uint32_t g = 0;
-                if constexpr (KIND == kQuantBlockAct) {
-                    const uint32_t m2 = max_abs4(v);
-                    const uint32_t m = max(m2 & 0xFFFFu, m2 >> 16);
-                    const uint32_t m_lo = __reduce_max_sync(0xFFFFFFFFu, h == 0 ? m : 0u);
-                    const uint32_t m_hi = __reduce_max_sync(0xFFFFFFFFu, h == 1 ? m : 0u);
-                    g = e8m0_exponent<FMT>(h ? m_hi : m_lo);
-                    nan_group = (g == 0xFFu);
-                    mul = pow2_inv_scale(nan_group ? 0u : g);
-                } else if constexpr (KIND == kQuantBlockWeight) {
-                    nan_group = (blk_g == 0xFFu);
-                    mul = pow2_inv_scale(nan_group ? 0u : blk_g);
-                } else {
-                    nan_group = t_nan;
-                    mul = t_scale;
-                }
-                const uint64_t mul2 = f32x2(mul, mul);
-                uint2 out;
-                out.x = quant4<FMT>(bf16_lo(v.x), bf16_hi(v.x), bf16_lo(v.y), bf16_hi(v.y), mul2, nan_group);
-                out.y = quant4<FMT>(bf16_lo(v.z), bf16_hi(v.z), bf16_lo(v.w), bf16_hi(v.w), mul2, nan_group);
-                *reinterpret_cast<uint2 *>(sm.q_stage + r * kQT + 8 * j) = out;
-                if (KIND == kQuantBlockAct && j == 0) sm.row_g[r] = static_cast<uint8_t>(g);
+        // ---- B: finish the scales (thread t < 128: row t; t >= 128: column t - 128)
+        if constexpr (KIND == kQuantBlockAct) {
+            if (tid < kQT) {
+                const uint4 *rp = reinterpret_cast<const uint4 *>(sm.row_part[tid >> 1]);
+                const uint4 a = rp[0], b = rp[1], c = rp[2], d = rp[3];
+                uint32_t m = __vmaxu2(__vmaxu2(__vmaxu2(a.x, a.y), __vmaxu2(a.z, a.w)),
+                                      __vmaxu2(__vmaxu2(b.x, b.y), __vmaxu2(b.z, b.w)));
+                m = __vmaxu2(m, __vmaxu2(__vmaxu2(__vmaxu2(c.x, c.y), __vmaxu2(c.z, c.w)),
+                                         __vmaxu2(__vmaxu2(d.x, d.y), __vmaxu2(d.z, d.w))));
+                const uint32_t g = e8m0_exponent<FMT>((tid & 1) ? (m >> 16) : (m & 0xFFFFu));
+                sm.row_mul[tid] = mul_of(g);
+                sm.row_g[tid] = static_cast<uint8_t>(g);
+            } else if (HAS_T) {
+                const int c = tid - kQT;
+                uint32_t m = 0;
+#pragma unroll
+                for (int b = 0; b < 16; ++b) m = __vmaxu2(m, sm.col_part[b][c >> 1]);
+                const uint32_t g = e8m0_exponent<FMT>((c & 1) ? (m >> 16) : (m & 0xFFFFu));
+                sm.col_mul[c] = mul_of(g);
+                sm.col_g[c] = static_cast<uint8_t>(g);
             }
+            __syncthreads();  // (S3) scales ready
         }
 
-        // ---- column pass: 128x1 groups along rows -> q_t (transposed).
-        // Thread t owns columns 2cp, 2cp+1 (cp = t % 64) over the 32 rows of
-        // quarter rq = t / 64: one 4-byte load per row feeds both columns.
+        float rmul[8], cmul[8];
+        uint32_t blk_g = 0;
+        if constexpr (KIND == kQuantBlockAct) {
+            const float4 r_lo = *reinterpret_cast<const float4 *>(&sm.row_mul[8 * br]);
+            const float4 r_hi = *reinterpret_cast<const float4 *>(&sm.row_mul[8 * br + 4]);
+            rmul[0] = r_lo.x; rmul[1] = r_lo.y; rmul[2] = r_lo.z; rmul[3] = r_lo.w;
+            rmul[4] = r_hi.x; rmul[5] = r_hi.y; rmul[6] = r_hi.z; rmul[7] = r_hi.w;
+        } else {
+            float mul = t_mul;
+            if constexpr (KIND == kQuantBlockWeight) {
+                uint32_t m = sm.red[lane & 7];
+                m = __reduce_max_sync(0xFFFFFFFFu, m);
+                blk_g = e8m0_exponent<FMT>(m);
+                mul = mul_of(blk_g);
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i) rmul[i] = cmul[i] = mul;
+        }
+
+        // ---- C: rowwise codes (row i, 8 columns) and transposed codes
+        // (column j, 8 rows) from the same block.  The block is re-read from
+        // shared memory here rather than kept live across (S2)/(S3).
+        if constexpr (KIND != kQuantTensor) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) v[i] = *reinterpret_cast<const uint4 *>(in + (8 * br + i) * kQT + 8 * bc);
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const uint64_t m2 = f32x2(rmul[i], rmul[i]);
+            const bool nan_row = isnan(rmul[i]);
+            uint2 o;
+            o.x = quant4<FMT>(bf16_lo(v[i].x), bf16_hi(v[i].x), bf16_lo(v[i].y), bf16_hi(v[i].y), m2, nan_row);
+            o.y = quant4<FMT>(bf16_lo(v[i].z), bf16_hi(v[i].z), bf16_lo(v[i].w), bf16_hi(v[i].w), m2, nan_row);
+            *reinterpret_cast<uint2 *>(sm.q_stage + (8 * br + i) * kQT + 8 * bc) = o;
+        }
         if constexpr (HAS_T) {
-            const int cp = tid & 63, rq = tid >> 6;
-            uint32_t w[32];
-#pragma unroll
-            for (int k = 0; k < 32; ++k) w[k] = *reinterpret_cast<const uint32_t *>(in + (32 * rq + k) * kQT + 2 * cp);
-            float mul_lo, mul_hi;
-            bool nan_lo, nan_hi;
-            if constexpr (KIND == kQuantBlockAct) {
-                uint32_t m2 = 0;
-#pragma unroll
-                for (int k = 0; k < 32; ++k) m2 = __vmaxu2(m2, w[k] & 0x7FFF7FFFu);
-                sm.col_amax2[rq][cp] = m2;
-                __syncthreads();  // (S2)
-                m2 = __vmaxu2(__vmaxu2(sm.col_amax2[0][cp], sm.col_amax2[1][cp]),
-                              __vmaxu2(sm.col_amax2[2][cp], sm.col_amax2[3][cp]));
-                const uint32_t g_lo = e8m0_exponent<FMT>(m2 & 0xFFFFu), g_hi = e8m0_exponent<FMT>(m2 >> 16);
-                nan_lo = (g_lo == 0xFFu);
-                nan_hi = (g_hi == 0xFFu);
-                mul_lo = pow2_inv_scale(nan_lo ? 0u : g_lo);
-                mul_hi = pow2_inv_scale(nan_hi ? 0u : g_hi);
-                if (rq == 0) {
-                    sm.col_g[2 * cp] = static_cast<uint8_t>(g_lo);
-                    sm.col_g[2 * cp + 1] = static_cast<uint8_t>(g_hi);
-                }
-            } else if constexpr (KIND == kQuantBlockWeight) {
-                nan_lo = nan_hi = (blk_g == 0xFFu);
-                mul_lo = mul_hi = pow2_inv_scale(nan_lo ? 0u : blk_g);
-            } else {
-                nan_lo = nan_hi = t_nan;
-                mul_lo = mul_hi = t_scale;
+            if constexpr (KIND == kQuantBlockAct) {  // column scales, loaded once the row codes are out
+                const float4 c_lo = *reinterpret_cast<const float4 *>(&sm.col_mul[8 * bc]);
+                const float4 c_hi = *reinterpret_cast<const float4 *>(&sm.col_mul[8 * bc + 4]);
+                cmul[0] = c_lo.x; cmul[1] = c_lo.y; cmul[2] = c_lo.z; cmul[3] = c_lo.w;
+                cmul[4] = c_hi.x; cmul[5] = c_hi.y; cmul[6] = c_hi.z; cmul[7] = c_hi.w;
             }
-            const uint64_t m2lo = f32x2(mul_lo, mul_lo), m2hi = f32x2(mul_hi, mul_hi);
-            uint32_t c_lo[8], c_hi[8];  // 32 codes of each column, rows 32rq .. 32rq+31
+            // Column j's 8 codes (rows 8br .. 8br+7) go to transposed row
+            // 8bc + j, bytes 8br .. 8br+7.  Lanes of one half-warp share br,
+            // so they would all hit the same swizzled chunk if they stored
+            // the same j together; instead lane bc stores column (s + bc) % 8
+            // at step s, which spreads the 16 lanes over all 32 banks.  The
+            // per-lane order is a barrel rotation of the code array.
+            uint2 cc[8];
 #pragma unroll
-            for (int q4 = 0; q4 < 8; ++q4) {
-                const uint32_t a = w[4 * q4], b = w[4 * q4 + 1], c = w[4 * q4 + 2], d = w[4 * q4 + 3];
-                c_lo[q4] = quant4<FMT>(bf16_lo(a), bf16_lo(b), bf16_lo(c), bf16_lo(d), m2lo, nan_lo);
-                c_hi[q4] = quant4<FMT>(bf16_hi(a), bf16_hi(b), bf16_hi(c), bf16_hi(d), m2hi, nan_hi);
-            }
-            // Store the two transposed rows; lanes with cp bit 2 set store the
-            // odd row first, so each 8-lane phase touches 8 distinct rows mod 8
-            // (distinct swizzled chunks: no bank conflicts).
-            const int sel = (cp >> 2) & 1;
+            for (int j = 0; j < 8; ++j) {
+                const uint64_t m2 = f32x2(cmul[j], cmul[j]);
+                const bool nan_col = isnan(cmul[j]);
+                float c[8];
 #pragma unroll
-            for (int pass = 0; pass < 2; ++pass) {
-                const int which = sel ^ pass;  // 0: column 2cp, 1: column 2cp+1
-                const int row = 2 * cp + which;
-                uint8_t *dst = sm.qt_stage + row * kQT;
-#pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    const uint4 o = which ? make_uint4(c_hi[4 * i], c_hi[4 * i + 1], c_hi[4 * i + 2], c_hi[4 * i + 3])
-                                          : make_uint4(c_lo[4 * i], c_lo[4 * i + 1], c_lo[4 * i + 2], c_lo[4 * i + 3]);
-                    *reinterpret_cast<uint4 *>(dst + 16 * ((2 * rq + i) ^ (row & 7))) = o;
+                for (int i = 0; i < 8; ++i) {
+                    const uint32_t w = (j >> 1) == 0 ? v[i].x : (j >> 1) == 1 ? v[i].y : (j >> 1) == 2 ? v[i].z : v[i].w;
+                    c[i] = (j & 1) ? bf16_hi(w) : bf16_lo(w);
                 }
+                cc[j].x = quant4<FMT>(c[0], c[1], c[2], c[3], m2, nan_col);
+                cc[j].y = quant4<FMT>(c[4], c[5], c[6], c[7], m2, nan_col);
+            }
+            const int rot = bc & 7;
+#pragma unroll
+            for (int b = 1; b < 8; b <<= 1) {  // cc[s] <- cc[(s + rot) % 8], one rotate-by-b stage per bit
+                const bool on = (rot & b) != 0;
+                uint2 t[8];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) t[k] = on ? cc[(k + b) & 7] : cc[k];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) cc[k] = t[k];
+            }
+#pragma unroll
+            for (int st = 0; st < 8; ++st) {
+                const int r = 8 * bc + ((st + rot) & 7);  // transposed row (tile column)
+                *reinterpret_cast<uint2 *>(sm.qt_stage + r * kQT + 16 * ((br >> 1) ^ (r & 7)) + 8 * (br & 1)) = cc[st];
             }
         }
 
         fence_proxy_async_smem();
-        __syncthreads();  // (S3) staging complete
+        __syncthreads();  // (S4) staging complete
         if (tid == 0) {
             tma_store_2d(&tm_q, sm.q_stage, static_cast<int32_t>(c0), static_cast<int32_t>(r0));
             if (HAS_T) tma_store_2d(&tm_qt, sm.qt_stage, static_cast<int32_t>(r0), static_cast<int32_t>(c0));
@@ -387,7 +422,6 @@ __global__ void __launch_bounds__(kQThreads, 2)
             }
         }
     }
-    cp_async_wait<0>();
     if (tid == 0) bulk_wait_group0();
 }
 
@@ -409,8 +443,8 @@ cudaError_t launch_tensor_scale_only(const QuantArgs &a, cudaStream_t s) {
 }
 
 template <int FMT, int KIND, bool HAS_T>
-static cudaError_t launch_quant_t(const QuantArgs &a, const CUtensorMap &tm_q, const CUtensorMap &tm_qt,
-                                  cudaStream_t s) {
+static cudaError_t launch_quant_t(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
+                                  const CUtensorMap &tm_qt, cudaStream_t s) {
     auto kern = quant_tile_kernel<FMT, KIND, HAS_T>;
     const size_t smem = sizeof(QuantSmem) + 1024;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
@@ -422,31 +456,31 @@ static cudaError_t launch_quant_t(const QuantArgs &a, const CUtensorMap &tm_q, c
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int grid = ntiles < 2 * sms ? ntiles : 2 * sms;  // persistent: two CTAs per SM
-    kern<<<grid, kQThreads, smem, s>>>(tm_q, tm_qt, a.x, a.rows, a.cols, a.scale_u8, a.scale_t_u8, a.scale_f,
+    kern<<<grid, kQThreads, smem, s>>>(tm_x, tm_q, tm_qt, a.rows, a.cols, a.scale_u8, a.scale_t_u8, a.scale_f,
                                        a.scale_t_f, a.amax, tiles_n, ntiles);
     return cudaGetLastError();
 }
 
 template <int FMT, int KIND>
-static cudaError_t launch_quant_k(const QuantArgs &a, const CUtensorMap &tm_q, const CUtensorMap &tm_qt,
-                                  cudaStream_t s) {
-    return a.has_t ? launch_quant_t<FMT, KIND, true>(a, tm_q, tm_qt, s)
-                   : launch_quant_t<FMT, KIND, false>(a, tm_q, tm_qt, s);
+static cudaError_t launch_quant_k(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
+                                  const CUtensorMap &tm_qt, cudaStream_t s) {
+    return a.has_t ? launch_quant_t<FMT, KIND, true>(a, tm_x, tm_q, tm_qt, s)
+                   : launch_quant_t<FMT, KIND, false>(a, tm_x, tm_q, tm_qt, s);
 }
 
 template <int FMT>
-static cudaError_t launch_quant_f(const QuantArgs &a, const CUtensorMap &tm_q, const CUtensorMap &tm_qt,
-                                  cudaStream_t s) {
+static cudaError_t launch_quant_f(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
+                                  const CUtensorMap &tm_qt, cudaStream_t s) {
     switch (a.kind) {
-        case kQuantBlockAct: return launch_quant_k<FMT, kQuantBlockAct>(a, tm_q, tm_qt, s);
-        case kQuantBlockWeight: return launch_quant_k<FMT, kQuantBlockWeight>(a, tm_q, tm_qt, s);
-        default: return launch_quant_k<FMT, kQuantTensor>(a, tm_q, tm_qt, s);
+        case kQuantBlockAct: return launch_quant_k<FMT, kQuantBlockAct>(a, tm_x, tm_q, tm_qt, s);
+        case kQuantBlockWeight: return launch_quant_k<FMT, kQuantBlockWeight>(a, tm_x, tm_q, tm_qt, s);
+        default: return launch_quant_k<FMT, kQuantTensor>(a, tm_x, tm_q, tm_qt, s);
     }
 }
 
-cudaError_t launch_quantize(const QuantArgs &a, const CUtensorMap &tm_q, const CUtensorMap &tm_qt,
-                            cudaStream_t s) {
-    return a.fmt == 0 ? launch_quant_f<0>(a, tm_q, tm_qt, s) : launch_quant_f<1>(a, tm_q, tm_qt, s);
+cudaError_t launch_quantize(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
+                            const CUtensorMap &tm_qt, cudaStream_t s) {
+    return a.fmt == 0 ? launch_quant_f<0>(a, tm_x, tm_q, tm_qt, s) : launch_quant_f<1>(a, tm_x, tm_q, tm_qt, s);
 }
 
 }  // namespace puro
