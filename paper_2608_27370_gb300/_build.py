@@ -1,6 +1,6 @@
 """Build the CUDA library libpuro_fp8.so in-tree with nvcc for sm_103a.
 
-Three translation units are compiled in parallel and linked into one shared
+Four translation units are compiled in parallel and linked into one shared
 object with the CUDA runtime linked statically, so the library loads on a
 machine without a GPU driver (only the first CUDA call needs one).
 """

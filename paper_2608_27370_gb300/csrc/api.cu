@@ -49,6 +49,10 @@ bool make_map(CUtensorMap *m, CUtensorMapDataType dt, const void *base, uint64_t
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// GEMM operand tiles: one swizzle row of kGemmBKBytes bytes per K stage.
+constexpr CUtensorMapSwizzle kOperandSwizzle =
+    kGemmBKBytes == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+
 int sm_count() {
     static int cache[64] = {0};
     int dev = 0;
@@ -97,10 +101,8 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
     const bool block = a->scaling == PURO_SCALE_BLOCK;
 
     CUtensorMap tm_a, tm_b, tm_d;
-    if (!make_map(&tm_a, CU_TENSOR_MAP_DATA_TYPE_UINT8, a->data, K, M, K, 128, kGemmBM,
-                  CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&tm_b, CU_TENSOR_MAP_DATA_TYPE_UINT8, b->data, K, N, K, 128, kGemmBN,
-                  CU_TENSOR_MAP_SWIZZLE_128B) ||
+    if (!make_map(&tm_a, CU_TENSOR_MAP_DATA_TYPE_UINT8, a->data, K, M, K, kGemmBKBytes, kGemmBM, kOperandSwizzle) ||
+        !make_map(&tm_b, CU_TENSOR_MAP_DATA_TYPE_UINT8, b->data, K, N, K, kGemmBKBytes, kGemmBN, kOperandSwizzle) ||
         !make_map(&tm_d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B))
         return PURO_ERR_CUDA;
     GemmArgs g{};
@@ -147,8 +149,10 @@ puro_status_t bf16_gemm(const void *a, const void *b, void *d, int64_t M, int64_
     if (M == 0 || N == 0) return PURO_OK;
     if (K == 0) return cuda_status(cudaMemsetAsync(d, 0, static_cast<size_t>(M * N) * 2, s));
     CUtensorMap tm_a, tm_b, tm_d;
-    if (!make_map(&tm_a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a, K, M, K * 2, 64, kGemmBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, b, K, N, K * 2, 64, kGemmBN, CU_TENSOR_MAP_SWIZZLE_128B) ||
+    if (!make_map(&tm_a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a, K, M, K * 2, kGemmBKBytes / 2, kGemmBM,
+                  kOperandSwizzle) ||
+        !make_map(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, b, K, N, K * 2, kGemmBKBytes / 2, kGemmBN,
+                  kOperandSwizzle) ||
         !make_map(&tm_d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B))
         return PURO_ERR_CUDA;
     GemmArgs g{};

@@ -32,8 +32,10 @@ namespace puro {
 
 constexpr int kBM = kGemmBM;       // rows of A per tile (= TMEM lanes)
 constexpr int kBN = kGemmBN;       // rows of B per tile (= accumulator columns)
-constexpr int kBKBytes = 128;      // bytes of K per pipeline stage (one swizzle row)
-constexpr int kStages = 4;
+constexpr int kBKBytes = kGemmBKBytes;             // bytes of K per pipeline stage (one swizzle row)
+constexpr int kStages = kBKBytes == 128 ? 4 : 8;   // ~192 KB of operand ring either way
+constexpr int kStagesPerKBlock = 128 / kBKBytes;   // stages per 128-byte k-block (one FP8 scale group)
+constexpr int kStagesPerGroup = 512 / kBKBytes;    // stages per group of four k-blocks (one scale chunk)
 constexpr int kThreads = 256;
 constexpr int kTmemCols = 512;
 constexpr int kSfColsPerSet = 12;  // 4 for A (128 rows) + 8 for B (256 rows)
@@ -61,7 +63,7 @@ struct GemmParams {
     int M, N, K;
     int num_m, num_n, num_kb, num_tiles;
     int splits;        // reduction split into this many chunks (1: no split)
-    int kb_per_split;  // k-blocks per chunk (a multiple of 4)
+    int kb_per_split;  // stages per chunk (a whole number of scale groups)
     int num_units;     // num_tiles * splits
     int m_fastest;     // tile order: 1 = row blocks of A vary fastest
     uint32_t idesc;
@@ -178,13 +180,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                         aborted = true;
                         break;
                     }
-                    const bool sf_load = kMX && (kb & 3) == 0;
+                    const bool sf_load = kMX && (kb % kStagesPerGroup) == 0;
                     const uint32_t bytes = (kBM + kBN) * kBKBytes + (sf_load ? 512u + 1024u : 0u);
                     mbar_arrive_expect_tx(&sm.full[stage], bytes);
                     tma_load_2d(sm.a[stage], &tm_a, &sm.full[stage], kb * kBK, m0);
                     tma_load_2d(sm.b[stage], &tm_b, &sm.full[stage], kb * kBK, n0);
                     if (sf_load) {
-                        const int64_t kg = kb >> 2;
+                        const int64_t kg = kb / kStagesPerGroup;
                         bulk_load(sm.sf_a[stage], p.sfa + ((m0 / 128) * static_cast<int64_t>(p.kgroups) + kg) * 512, 512,
                                   &sm.full[stage]);
                         const uint8_t *b0 = p.sfb + ((n0 / 128) * static_cast<int64_t>(p.kgroups) + kg) * 512;
@@ -234,25 +236,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc_fence_after_sync();
                 if (lane == 0) {
-                    const uint32_t sfa_col = kSfBase + ((kb >> 2) & 1) * kSfColsPerSet;
+                    const uint32_t sfa_col = kSfBase + ((kb / kStagesPerGroup) & 1) * kSfColsPerSet;
                     const uint32_t sfb_col = sfa_col + 4;
                     uint32_t idesc = p.idesc;
                     if constexpr (kMX) {
-                        if ((kb & 3) == 0) {  // new group of four k-blocks: its scale vectors
+                        if (kb % kStagesPerGroup == 0) {  // new group of four k-blocks: its scale vectors
                             tmem_cp_32x128b_warpx4(tmem + sfa_col, smem_desc_plain_16B_rows(smem_u32(sm.sf_a[stage])));
                             tmem_cp_32x128b_warpx4(tmem + sfb_col, smem_desc_plain_16B_rows(smem_u32(sm.sf_b[stage])));
                             tmem_cp_32x128b_warpx4(tmem + sfb_col + 4,
                                                    smem_desc_plain_16B_rows(smem_u32(sm.sf_b[stage] + 512)));
                         }
-                        const uint32_t sf_id = static_cast<uint32_t>(kb & 3);
+                        const uint32_t sf_id = static_cast<uint32_t>((kb / kStagesPerKBlock) & 3);
                         idesc |= (sf_id << 29) | (sf_id << 4);
                     }
                     const uint32_t a_addr = smem_u32(sm.a[stage]);
                     const uint32_t b_addr = smem_u32(sm.b[stage]);
 #pragma unroll
                     for (int k = 0; k < kKSteps; ++k) {
-                        const uint64_t ad = smem_desc_k_sw128(a_addr + 32 * k);
-                        const uint64_t bd = smem_desc_k_sw128(b_addr + 32 * k);
+                        const uint64_t ad = smem_desc_k_swizzled<kBKBytes>(a_addr + 32 * k);
+                        const uint64_t bd = smem_desc_k_swizzled<kBKBytes>(b_addr + 32 * k);
                         const uint32_t acc = (kb > wu.kb0 || k > 0) ? 1u : 0u;
                         if constexpr (KIND == kGemmBF16)
                             mma_f16(d_tmem, ad, bd, idesc, acc);
@@ -418,7 +420,7 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const float4 *__rest
 int choose_splits(int64_t M, int64_t N, int64_t K, bool bf16) {
     if (bf16) return 1;
     const int64_t tiles = ((M + kBM - 1) / kBM) * ((N + kBN - 1) / kBN);
-    const int64_t kblocks = (K + kBKBytes - 1) / kBKBytes;
+    const int64_t kblocks = (K + 127) / 128;  // 128-byte k-blocks (independent of the stage size)
     if (tiles >= kSplitRefSms) return 1;
     // Modelled time = waves x k-blocks per chunk; chunks keep >= 16 k-blocks
     // (whole groups of four).  Split only for a >= 15% modelled gain.
@@ -461,7 +463,7 @@ static cudaError_t launch_kind(const GemmArgs &g, const CUtensorMap &tm_a, const
     p.num_kb = static_cast<int>((g.K + kBK - 1) / kBK);
     p.num_tiles = p.num_m * p.num_n;
     p.splits = splits;
-    p.kb_per_split = ((p.num_kb + splits - 1) / splits + 3) / 4 * 4;
+    p.kb_per_split = ((p.num_kb + splits - 1) / splits + kStagesPerGroup - 1) / kStagesPerGroup * kStagesPerGroup;
     p.splits = (p.num_kb + p.kb_per_split - 1) / p.kb_per_split;  // no empty chunk
     p.num_units = p.num_tiles * p.splits;
     p.m_fastest = g.M < g.N ? 1 : 0;  // re-read the smaller operand, stream the larger once

@@ -86,8 +86,11 @@ puro_status_t fp8_gemm_entry(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t
 int choose_splits(int64_t M, int64_t N, int64_t K, bool bf16);
 size_t splitk_workspace_bytes(int64_t M, int64_t N, int64_t K, bool bf16);
 
-// Tile shape of the GEMM kernel (rows of A per CTA tile, rows of B).
+// Tile shape of the GEMM kernel (rows of A per CTA tile, rows of B) and the
+// bytes of K per pipeline stage (128: 4 stages, 128-byte swizzle; 64: 8
+// stages, 64-byte swizzle).
 constexpr int kGemmBM = 128;
 constexpr int kGemmBN = 256;
+constexpr int kGemmBKBytes = 128;
 
 }  // namespace puro

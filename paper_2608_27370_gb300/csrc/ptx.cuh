@@ -222,6 +222,20 @@ PURO_DEV uint64_t smem_desc_k_sw128(uint32_t saddr) {
     return d;
 }
 
+// The same for a tile whose K rows are kRowBytes (128 or 64) bytes, written by
+// TMA with the matching swizzle: 8-row atoms of 8 * kRowBytes bytes.
+template <int kRowBytes>
+PURO_DEV uint64_t smem_desc_k_swizzled(uint32_t saddr) {
+    static_assert(kRowBytes == 128 || kRowBytes == 64, "128- or 64-byte swizzle");
+    uint64_t d = 0;
+    d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+    d |= static_cast<uint64_t>(1) << 16;
+    d |= static_cast<uint64_t>((8 * kRowBytes) >> 4) << 32;
+    d |= static_cast<uint64_t>(1) << 46;
+    d |= static_cast<uint64_t>(kRowBytes == 128 ? 2 : 4) << 61;  // 2: 128-byte swizzle, 4: 64-byte swizzle
+    return d;
+}
+
 // Un-swizzled K-major layout of 8-row x 16-byte core matrices stored
 // contiguously (128 bytes each): SBO = 128 between 8-row groups; a single
 // core matrix along K, so LBO is unused (0).  Source form of tcgen05.cp.
