@@ -38,6 +38,36 @@ METRIC = "FP8 linear fwd+bwd TFLOP/s and % of FP8 peak; quantise HBM GB/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 FP8_PER_BF16 = 2.0  # nominal dense ratio (4.5 / 2.25 PFLOP/s)
 
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per call, averaged
+# over the 12 GEMM calls (split reductions included) and the 12 quantise calls
+# of one layer, from a one-pass ncu capture of one full-size layer of the C5
+# workload (block scaling, M = 32768).  All 28 layers have the same shapes, so
+# one layer's calls stand for the step.  Each figure holds only for the kernel
+# sources it was captured on (sha1 prefix over the listed files) and is
+# reported as null once they change or for another workload.
+CAPTURED_TRAFFIC = {
+    "gemm": {"files": ["gemm.cu", "ptx.cuh", "internal.h", "api.cu"], "sha1": "907b42adcb895d7e",
+             "bytes_per_call": 441649365, "algorithmic_bytes_per_call": 417016966},
+    "quantize": {"files": ["quantize.cu", "ptx.cuh", "internal.h", "api.cu"], "sha1": "8c2ff2161340d6b2",
+                 "bytes_per_call": 379174165, "algorithmic_bytes_per_call": 417016966},
+}
+CAPTURED_TRAFFIC_WORKLOAD = ("C5", 32768, "block")
+CAPTURED_TRAFFIC_PROFILE = "profiles/dram_traffic_C5_layer_M32768.md"
+
+
+def captured_traffic(kind: str, workload) -> "int | None":
+    """Per-call DRAM bytes of `kind` if the capture applies, else None."""
+    import hashlib
+
+    if tuple(workload) != CAPTURED_TRAFFIC_WORKLOAD:
+        return None
+    rec = CAPTURED_TRAFFIC[kind]
+    h = hashlib.sha1()
+    for f in rec["files"]:
+        with open(os.path.join(ROOT, "paper_2608_27370_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return rec["bytes_per_call"] if h.hexdigest().startswith(rec["sha1"]) else None
+
 
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -531,6 +561,7 @@ def main():
     gemm_tflops = g["units"] / g["time_s"] / 1e12
     quant_gbs = q["units"] / q["time_s"] / 1e9
     total_kernel_time = sum(c["time_s"] for c in per_kernel.values())
+    traffic_wl = (args.config, M, args.scaling)
     shares = {k: c["time_s"] / total_kernel_time for k, c in per_kernel.items()}
 
     result = {
@@ -553,10 +584,14 @@ def main():
         "roofline": {"bound": "tensor", "kernel": "gemm_tn_kernel<FP8 block-scaled>", "achieved": gemm_tflops,
                      "peak": fp8_peak_sust, "unit": "TFLOP/s", "frac": gemm_tflops / fp8_peak_sust,
                      "peak_source": f"2 x bf16_tflops_sustained ({peak_src}); kernel timed inside a long step",
-                     "traffic": None},
+                     "traffic": captured_traffic("gemm", traffic_wl),
+                     "traffic_note": "DRAM bytes per GEMM call (avg of one layer's 12), " + CAPTURED_TRAFFIC_PROFILE},
         "roofline_quantize": {"bound": "hbm", "kernel": "quant_tile_kernel", "achieved": quant_gbs,
                               "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": quant_gbs / peaks["hbm_gbs"],
-                              "peak_source": f"hbm_gbs ({peak_src})", "traffic": None},
+                              "peak_source": f"hbm_gbs ({peak_src})",
+                              "traffic": captured_traffic("quantize", traffic_wl),
+                              "traffic_note": "DRAM bytes per quantise call (avg of one layer's 12), " +
+                                              CAPTURED_TRAFFIC_PROFILE},
     }
     if args.scaling == "tensor":
         result["roofline"]["kernel"] = "gemm_tn_kernel<FP8 per-tensor>"
