@@ -96,6 +96,29 @@ def parse_args():
 
 
 # ----------------------------------------------------------------------------
+# multi-rank timing: one process per GPU, each a full replica of the step
+# (the linears of different replicas share nothing, so no collective runs on
+# the data path); the job's time is the slowest rank's
+# ----------------------------------------------------------------------------
+def max_over_ranks(seconds: float, world: int, device) -> float:
+    """The maximum of a per-rank duration over all ranks, then a barrier."""
+    if world <= 1:
+        return seconds
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([seconds], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.barrier()
+    return float(t.item())
+
+
+def job_value(world: int, units_per_rank: float, step_seconds: float) -> float:
+    """Whole-job throughput: the units every rank processed over the job's step time."""
+    return world * units_per_rank / step_seconds
+
+
+# ----------------------------------------------------------------------------
 # clocks during the timed region
 # ----------------------------------------------------------------------------
 class ClockSampler:
@@ -491,7 +514,8 @@ def reference_arm(args):
     line = {"metric": METRIC, "value": v, "unit": "TFLOP/s", "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": t * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": wl.description, "tokens_per_step": M_s},
+            "config": {"workload": f"{wl.key}: " + wl.description, "tokens_per_step": M_s,
+                       "scaling": "block", "sample": "bounded CPU sample of the workload, see cpu_baseline"},
             "cpu_baseline": {"value": v, "unit": "TFLOP/s", "cores": threads, "kind": "oracle", "sample": sample},
             "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -543,16 +567,11 @@ def main():
     torch.cuda.synchronize()
     clk = clocks.stop()
     stack.timer.enabled = False
-    elapsed = t_start.elapsed_time(t_end) * 1e-3
-    if world > 1:
-        t = torch.tensor([elapsed], device=device, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed = float(t.item())
-        dist.barrier()
+    elapsed = max_over_ranks(t_start.elapsed_time(t_end) * 1e-3, world, device)
     per_kernel = stack.timer.totals()
     step_s = elapsed / args.steps
     flops = stack.flops_per_step()
-    value = world * flops / step_s / 1e12
+    value = job_value(world, flops, step_s) / 1e12
 
     fp8_peak_burst = peaks["bf16_tflops"] * FP8_PER_BF16
     fp8_peak_sust = peaks["bf16_tflops_sustained"] * FP8_PER_BF16
@@ -605,10 +624,9 @@ def main():
     if not args.no_e2e:
         result["e2e"] = e2e_measure(P, torch, stack, max(1, min(args.steps, 3)))
         if world > 1:
-            t = torch.tensor([result["e2e"]["ms_per_step"]], device=device, dtype=torch.float64)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            result["e2e"]["ms_per_step"] = float(t.item())
-            result["e2e"]["value"] = world * flops / (float(t.item()) * 1e-3) / 1e12
+            ms = max_over_ranks(result["e2e"]["ms_per_step"], world, device)
+            result["e2e"]["ms_per_step"] = ms
+            result["e2e"]["value"] = job_value(world, flops, ms * 1e-3) / 1e12
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(torch, stack)
     if rank == 0:
