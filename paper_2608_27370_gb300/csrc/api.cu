@@ -49,9 +49,13 @@ bool make_map(CUtensorMap *m, CUtensorMapDataType dt, const void *base, uint64_t
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// GEMM operand tiles: one swizzle row of kGemmBKBytes bytes per K stage.
-constexpr CUtensorMapSwizzle kOperandSwizzle =
-    kGemmBKBytes == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+// Scale vectors of a BLOCK operand [rows, red] as uint32 [rows/128 *
+// ceil(red/512), 128]: one 512-byte chunk (128 rows x four k-blocks) per row
+// of the map, loaded whole (box {128, 1}); rows past the end read as zero.
+bool make_scale_map(CUtensorMap *m, const void *scale, int64_t rows, int64_t red) {
+    const uint64_t chunks = static_cast<uint64_t>((rows + 127) / 128) * static_cast<uint64_t>((red / 128 + 3) / 4);
+    return make_map(m, CU_TENSOR_MAP_DATA_TYPE_UINT32, scale, 128, chunks, 512, 128, 1, CU_TENSOR_MAP_SWIZZLE_NONE);
+}
 
 int sm_count() {
     static int cache[64] = {0};
@@ -100,11 +104,16 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
     if (K == 0) return cuda_status(cudaMemsetAsync(d, 0, static_cast<size_t>(M * N) * 2, s));
     const bool block = a->scaling == PURO_SCALE_BLOCK;
 
-    CUtensorMap tm_a, tm_b, tm_d;
-    if (!make_map(&tm_a, CU_TENSOR_MAP_DATA_TYPE_UINT8, a->data, K, M, K, kGemmBKBytes, kGemmBM, kOperandSwizzle) ||
-        !make_map(&tm_b, CU_TENSOR_MAP_DATA_TYPE_UINT8, b->data, K, N, K, kGemmBKBytes, kGemmBN, kOperandSwizzle) ||
-        !make_map(&tm_d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B))
+    GemmMaps m{};
+    if (!make_map(&m.a, CU_TENSOR_MAP_DATA_TYPE_UINT8, a->data, K, M, K, kGemmBKBytes, kGemmBM,
+                  CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, b->data, K, N, K, kGemmBKBytes, kGemmBN / 2,
+                  CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m.d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B))
         return PURO_ERR_CUDA;
+    m.ws = m.d;
+    m.sfa = m.d;
+    m.sfb = m.d;
     GemmArgs g{};
     g.kind = block ? kGemmFP8Block : kGemmFP8Tensor;
     g.a_fmt = a->fmt;
@@ -113,8 +122,7 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
     g.N = N;
     g.K = K;
     if (block) {
-        g.sfa = static_cast<const uint8_t *>(a->scale);
-        g.sfb = static_cast<const uint8_t *>(b->scale);
+        if (!make_scale_map(&m.sfa, a->scale, M, K) || !make_scale_map(&m.sfb, b->scale, N, K)) return PURO_ERR_CUDA;
     } else {
         g.sia = static_cast<const float *>(a->scale);
         g.sib = static_cast<const float *>(b->scale);
@@ -125,19 +133,18 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
     if (g.num_sms <= 0) return PURO_ERR_CUDA;
     g.out = d;
     g.splits = 1;
-    CUtensorMap tm_ws = tm_d;
-    // Split the reduction across CTAs when the output has too few tiles to
-    // fill the GPU and the caller supplied enough aligned scratch.
+    // Split the reduction across CTA pairs when the output has too few tiles
+    // to fill the GPU and the caller supplied enough aligned scratch.
     const int sp = choose_splits(M, N, K, false);
     if (sp > 1 && workspace && aligned16(workspace) && workspace_bytes >= splitk_workspace_bytes(M, N, K, false)) {
-        const uint64_t m_pad = static_cast<uint64_t>((M + kGemmBM - 1) / kGemmBM * kGemmBM);
-        if (!make_map(&tm_ws, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, workspace, N, static_cast<uint64_t>(sp) * m_pad, N * 4,
-                      32, 32, CU_TENSOR_MAP_SWIZZLE_128B))
+        const uint64_t rows = static_cast<uint64_t>(sp) * static_cast<uint64_t>(splitk_rows_per_chunk(M));
+        if (!make_map(&m.ws, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, workspace, N, rows, N * 4, 32, 32,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
             return PURO_ERR_CUDA;
         g.splits = sp;
         g.workspace = workspace;
     }
-    return cuda_status(launch_gemm(g, tm_a, tm_b, tm_d, tm_ws, s));
+    return cuda_status(launch_gemm(g, m, s));
 }
 
 puro_status_t bf16_gemm(const void *a, const void *b, void *d, int64_t M, int64_t N, int64_t K,
@@ -148,13 +155,16 @@ puro_status_t bf16_gemm(const void *a, const void *b, void *d, int64_t M, int64_
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (M == 0 || N == 0) return PURO_OK;
     if (K == 0) return cuda_status(cudaMemsetAsync(d, 0, static_cast<size_t>(M * N) * 2, s));
-    CUtensorMap tm_a, tm_b, tm_d;
-    if (!make_map(&tm_a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a, K, M, K * 2, kGemmBKBytes / 2, kGemmBM,
-                  kOperandSwizzle) ||
-        !make_map(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, b, K, N, K * 2, kGemmBKBytes / 2, kGemmBN,
-                  kOperandSwizzle) ||
-        !make_map(&tm_d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B))
+    GemmMaps m{};
+    if (!make_map(&m.a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a, K, M, K * 2, kGemmBKBytes / 2, kGemmBM,
+                  CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m.b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, b, K, N, K * 2, kGemmBKBytes / 2, kGemmBN / 2,
+                  CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m.d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B))
         return PURO_ERR_CUDA;
+    m.ws = m.d;
+    m.sfa = m.d;
+    m.sfb = m.d;
     GemmArgs g{};
     g.kind = kGemmBF16;
     g.M = M;
@@ -166,7 +176,7 @@ puro_status_t bf16_gemm(const void *a, const void *b, void *d, int64_t M, int64_
     if (g.num_sms <= 0) return PURO_ERR_CUDA;
     g.splits = 1;
     g.out = d;
-    return cuda_status(launch_gemm(g, tm_a, tm_b, tm_d, tm_d, s));
+    return cuda_status(launch_gemm(g, m, s));
 }
 
 }  // namespace

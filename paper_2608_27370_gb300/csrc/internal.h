@@ -53,10 +53,6 @@ struct GemmArgs {
     GemmKind kind;
     int a_fmt, b_fmt;            // FP8 formats (0 = E4M3, 1 = E5M2)
     int64_t M, N, K;
-    // kGemmFP8Block: scale vectors of A and B in the tensor-core layout,
-    // [rows/128][ceil(K/512)][512] bytes each.
-    const uint8_t *sfa;
-    const uint8_t *sfb;
     // kGemmFP8Tensor: dequantisation factors of A and B.
     const float *sia, *sib;
     int32_t *status;             // optional device status word
@@ -69,12 +65,20 @@ struct GemmArgs {
     void *out;
 };
 
-// tm_a: A [M, K], tm_b: B [N, K] (128-byte swizzle, box {128 bytes, rows}),
-// tm_d: D [M, N] bf16 (128-byte swizzle, box {64, 32}),
-// tm_ws: workspace [splits * M, N] fp32 (128-byte swizzle, box {32, 32});
-// only read when g.splits > 1.
-cudaError_t launch_gemm(const GemmArgs &g, const CUtensorMap &tm_a, const CUtensorMap &tm_b,
-                        const CUtensorMap &tm_d, const CUtensorMap &tm_ws, cudaStream_t s);
+// Tensor maps of one GEMM launch.
+//   a:   A [M, K] (128-byte swizzle, box {128 bytes, 128 rows})
+//   b:   B [N, K] (the same box: half of a 256-row tile per CTA)
+//   d:   D [M, N] bf16 (128-byte swizzle, box {64, 32})
+//   ws:  workspace [splits * splitk_rows_per_chunk(M), N] fp32 (128-byte
+//        swizzle, box {32, 32}); only read when g.splits > 1
+//   sfa, sfb (kGemmFP8Block only): the scale vectors of A / B,
+//        [rows/128][ceil(K/512)][512] bytes viewed as uint32
+//        [rows/128 * ceil(K/512), 128], box {128, 1}
+struct GemmMaps {
+    CUtensorMap a, b, d, ws, sfa, sfb;
+};
+
+cudaError_t launch_gemm(const GemmArgs &g, const GemmMaps &m, cudaStream_t s);
 
 // The FP8 GEMM entry behind puro_fp8_linear_{fprop,dgrad,wgrad}: validates,
 // encodes the tensor maps and launches (D = A * B^T).
@@ -85,10 +89,11 @@ puro_status_t fp8_gemm_entry(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t
 // then needs.  Host-only, shape-only (plans for 152 SMs).
 int choose_splits(int64_t M, int64_t N, int64_t K, bool bf16);
 size_t splitk_workspace_bytes(int64_t M, int64_t N, int64_t K, bool bf16);
+int64_t splitk_rows_per_chunk(int64_t M);  // M rounded up to a whole 256-row pair tile
 
-// Tile shape of the GEMM kernel (rows of A per CTA tile, rows of B) and the
-// bytes of K per pipeline stage (128: 4 stages, 128-byte swizzle; 64: 8
-// stages, 64-byte swizzle).
+// Tile shape of the GEMM kernel: rows of A per CTA (a CTA pair computes
+// 2 * kGemmBM rows), columns of a tile (rows of B per pair), and the bytes
+// of K per pipeline stage (one 128-byte swizzle row).
 constexpr int kGemmBM = 128;
 constexpr int kGemmBN = 256;
 constexpr int kGemmBKBytes = 128;

@@ -127,53 +127,106 @@ PURO_DEV void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) 
 // Tensor memory: 128 lanes x 512 columns of 32-bit cells per SM.  An
 // address is (lane << 16) | column.
 
-PURO_DEV void tmem_alloc(uint32_t *dst_smem, uint32_t ncols) {  // whole warp
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst_smem)),
+// The GEMM runs every tcgen05 operation as a CTA pair (cta_group::2): the
+// two CTAs of a 2-CTA cluster allocate the same tensor-memory columns
+// collectively (one warp in each), a pair MMA issued by one thread of the
+// even CTA reads A and B from both CTAs' shared memory (each holds its own
+// 128 rows of A and half of the N rows of B) and writes each CTA's 128 rows
+// of D into that CTA's tensor memory, and a pair tcgen05.cp copies each
+// CTA's shared memory into its own tensor memory.  All tcgen05 instructions
+// of a kernel use the same cta_group.
+
+PURO_DEV uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// All threads of both CTAs of the cluster (release / acquire).
+PURO_DEV void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Address of the same shared-memory variable in cluster CTA `rank`.
+PURO_DEV uint32_t mapa_shared(uint32_t saddr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+    return r;
+}
+
+// Arrive on an mbarrier given by its shared::cluster address (this CTA's or
+// a peer's), releasing this thread's prior writes at cluster scope.
+PURO_DEV void mbar_arrive_cluster(uint32_t bar_cluster) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+}
+
+// 2-D tiled load into this CTA's shared memory whose completion is counted
+// on an mbarrier that may live in the peer CTA of the pair.
+PURO_DEV void tma_load_2d_pair(void *dst, const CUtensorMap *map, uint32_t bar_cluster, int32_t x, int32_t y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cta.global.tile.mbarrier::complete_tx::bytes.cta_group::2"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar_cluster)
+        : "memory");
+}
+
+PURO_DEV void tmem_alloc_pair(uint32_t *dst_smem, uint32_t ncols) {  // one warp in each CTA of the pair
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst_smem)),
                  "r"(ncols)
                  : "memory");
 }
-PURO_DEV void tmem_relinquish_alloc_permit() {  // whole warp
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+PURO_DEV void tmem_relinquish_alloc_permit_pair() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
 }
-PURO_DEV void tmem_dealloc(uint32_t taddr, uint32_t ncols) {  // whole warp
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+PURO_DEV void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {  // one warp in each CTA of the pair
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
 }
 PURO_DEV void tc_fence_before_sync() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 PURO_DEV void tc_fence_after_sync() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
-// Arrive (once) on `bar` when every tcgen05.mma / tcgen05.cp previously
+// Arrive (once) on `bar` of this CTA when every pair MMA / copy previously
 // issued by this thread has completed.
-PURO_DEV void tc_commit(uint64_t *bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+PURO_DEV void tc_commit_pair(uint64_t *bar) {
+    asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                      smem_u32(bar))
                  : "memory");
 }
+// The same, arriving on `bar` in every cluster CTA of `cta_mask`.
+PURO_DEV void tc_commit_pair_multicast(uint64_t *bar, uint16_t cta_mask) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+            smem_u32(bar)),
+        "h"(cta_mask)
+        : "memory");
+}
 
-// D(tmem) (+)= A(smem) * B(smem)^T, kind::f16 (bf16/fp16 inputs, f32 accumulate).
-PURO_DEV void mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t accumulate) {
+// Pair MMA D(tmem) (+)= A(smem) * B(smem)^T, kind::f16 (bf16/fp16 inputs,
+// f32 accumulate).
+PURO_DEV void mma_pair_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t accumulate) {
     asm volatile(
         "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
         "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
 
 // kind::f8f6f4 (e4m3/e5m2 inputs, f32 accumulate), no block scaling.
-PURO_DEV void mma_f8(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t accumulate) {
+PURO_DEV void mma_pair_f8(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t accumulate) {
     asm volatile(
         "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+        "tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
         "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
 
 // kind::mxf8f6f4 with one UE8M0 scale per 32 elements of K for each row of
-// A and of B (scale_vec::1X); the scales are read from tensor memory.
-PURO_DEV void mma_mxf8(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t sfa_tmem,
-                       uint32_t sfb_tmem, uint32_t accumulate) {
+// A and of B (scale_vec::1X); the scales are read from tensor memory (each
+// CTA's own: its 128 rows of A, all N rows of B).
+PURO_DEV void mma_pair_mxf8(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t sfa_tmem,
+                            uint32_t sfb_tmem, uint32_t accumulate) {
     asm volatile(
         "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], %1, %2, %3, [%5], [%6], p;\n\t}\n" ::"r"(
+        "tcgen05.mma.cta_group::2.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], %1, %2, %3, [%5], [%6], p;\n\t}\n" ::"r"(
             d_tmem),
         "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate), "r"(sfa_tmem), "r"(sfb_tmem)
         : "memory");
@@ -181,9 +234,10 @@ PURO_DEV void mma_mxf8(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t
 
 // Copy 32 rows x 128 bits from shared memory into tensor memory, replicated
 // into each of the four 32-lane quarters (warpx4): row r lands in lane r of
-// every quarter, its four 32-bit words in columns taddr .. taddr+3.
-PURO_DEV void tmem_cp_32x128b_warpx4(uint32_t taddr, uint64_t sdesc) {
-    asm volatile("tcgen05.cp.cta_group::1.32x128b.warpx4 [%0], %1;" ::"r"(taddr), "l"(sdesc) : "memory");
+// every quarter, its four 32-bit words in columns taddr .. taddr+3.  The
+// pair form copies each CTA's shared memory into its own tensor memory.
+PURO_DEV void tmem_cp_pair_32x128b_warpx4(uint32_t taddr, uint64_t sdesc) {
+    asm volatile("tcgen05.cp.cta_group::2.32x128b.warpx4 [%0], %1;" ::"r"(taddr), "l"(sdesc) : "memory");
 }
 
 // Each thread of the warp reads 32 consecutive 32-bit columns of its own
