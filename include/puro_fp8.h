@@ -252,6 +252,17 @@ puro_status_t puro_bf16_linear_wgrad(const void *dy_t, const void *x_t, void *dw
  */
 void puro_set_wait_timeout_ns(uint64_t ns);
 
+/*
+ * Tile width of unsplit block-scaled GEMMs (process-wide): 0 (default) lets
+ * a per-shape cost model choose; 256 or 224 forces that form.  The 256-wide
+ * form shares half of its tensor-memory accumulator between consecutive
+ * tiles; the 224-wide form double-buffers it.  Both compute the same
+ * products (summation order differs only by tile boundaries, which do not
+ * cross the reduction).  Any other value returns PURO_ERR_INVALID_ARG.
+ * For tests and tuning; the paper has no counterpart.
+ */
+puro_status_t puro_set_gemm_tile_n(int32_t tile_n);
+
 /* Human-readable name of a status code (static string). */
 const char *puro_status_string(puro_status_t s);
 

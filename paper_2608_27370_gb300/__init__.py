@@ -78,6 +78,7 @@ _SIGNATURES = {
     "puro_bf16_linear_dgrad": (_I32, [_P, _P, _P, _I64, _I64, _I64, _P, _P]),
     "puro_bf16_linear_wgrad": (_I32, [_P, _P, _P, _I64, _I64, _I64, _P, _P]),
     "puro_set_wait_timeout_ns": (None, [ctypes.c_uint64]),
+    "puro_set_gemm_tile_n": (ctypes.c_int, [ctypes.c_int32]),
     "puro_status_string": (ctypes.c_char_p, [_I32]),
 }
 
@@ -249,6 +250,11 @@ def puro_bf16_linear_wgrad(dy_t, x_t, dw, M, N, K, dev_status=None, stream=None)
 
 def puro_set_wait_timeout_ns(ns: int) -> None:
     load_library().puro_set_wait_timeout_ns(int(ns))
+
+
+def puro_set_gemm_tile_n(tile_n: int) -> None:
+    """0: per-shape choice; 224 or 256: force that block-scaled GEMM form."""
+    _check("puro_set_gemm_tile_n", load_library().puro_set_gemm_tile_n(int(tile_n)))
 
 
 # --------------------------------------------------------------------------

@@ -14,6 +14,7 @@ namespace puro {
 namespace {
 
 std::atomic<uint64_t> g_wait_timeout_ns{2000000000ull};  // 2 s
+std::atomic<int> g_tile_n{0};                             // 0: cost model; 224 / 256: forced
 
 using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
                                    const cuuint64_t *, const cuuint32_t *, const cuuint32_t *,
@@ -104,12 +105,23 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
     if (K == 0) return cuda_status(cudaMemsetAsync(d, 0, static_cast<size_t>(M * N) * 2, s));
     const bool block = a->scaling == PURO_SCALE_BLOCK;
 
+    // Split the reduction across CTA pairs when the output has too few tiles
+    // to fill the GPU and the caller supplied enough aligned scratch;
+    // otherwise the block-scaled kind picks its tile width.
+    const int sp = choose_splits(M, N, K, false);
+    const bool split = sp > 1 && workspace && aligned16(workspace) &&
+                       workspace_bytes >= splitk_workspace_bytes(M, N, K, false);
+    const int forced = g_tile_n.load();
+    const int tile_n = (block && !split) ? (forced ? forced : choose_tile_n(M, N, K)) : 256;
+
     GemmMaps m{};
     if (!make_map(&m.a, CU_TENSOR_MAP_DATA_TYPE_UINT8, a->data, K, M, K, kGemmBKBytes, kGemmBM,
                   CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&m.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, b->data, K, N, K, kGemmBKBytes, kGemmBN / 2,
-                  CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&m.d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B))
+        !make_map(&m.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, b->data, K, N, K, kGemmBKBytes,
+                  static_cast<uint32_t>(tile_n / 2), CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !(tile_n == 256
+              ? make_map(&m.d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B)
+              : make_map(&m.d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B)))
         return PURO_ERR_CUDA;
     m.ws = m.d;
     m.sfa = m.d;
@@ -121,8 +133,10 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
     g.M = M;
     g.N = N;
     g.K = K;
+    g.tile_n = tile_n;
     if (block) {
         if (!make_scale_map(&m.sfa, a->scale, M, K) || !make_scale_map(&m.sfb, b->scale, N, K)) return PURO_ERR_CUDA;
+        g.sfb = static_cast<const uint8_t *>(b->scale);
     } else {
         g.sia = static_cast<const float *>(a->scale);
         g.sib = static_cast<const float *>(b->scale);
@@ -133,10 +147,7 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
     if (g.num_sms <= 0) return PURO_ERR_CUDA;
     g.out = d;
     g.splits = 1;
-    // Split the reduction across CTA pairs when the output has too few tiles
-    // to fill the GPU and the caller supplied enough aligned scratch.
-    const int sp = choose_splits(M, N, K, false);
-    if (sp > 1 && workspace && aligned16(workspace) && workspace_bytes >= splitk_workspace_bytes(M, N, K, false)) {
+    if (split) {
         const uint64_t rows = static_cast<uint64_t>(sp) * static_cast<uint64_t>(splitk_rows_per_chunk(M));
         if (!make_map(&m.ws, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, workspace, N, rows, N * 4, 32, 32,
                       CU_TENSOR_MAP_SWIZZLE_128B))
@@ -170,6 +181,7 @@ puro_status_t bf16_gemm(const void *a, const void *b, void *d, int64_t M, int64_
     g.M = M;
     g.N = N;
     g.K = K;
+    g.tile_n = 256;
     g.status = dev_status;
     g.wait_timeout_ns = g_wait_timeout_ns.load();
     g.num_sms = sm_count();
@@ -311,6 +323,12 @@ PURO_API puro_status_t puro_bf16_linear_wgrad(const void *dy_t, const void *x_t,
 }
 
 PURO_API void puro_set_wait_timeout_ns(uint64_t ns) { g_wait_timeout_ns.store(ns); }
+
+PURO_API puro_status_t puro_set_gemm_tile_n(int32_t tile_n) {
+    if (tile_n != 0 && tile_n != 224 && tile_n != 256) return PURO_ERR_INVALID_ARG;
+    g_tile_n.store(tile_n);
+    return PURO_OK;
+}
 
 PURO_API const char *puro_status_string(puro_status_t s) {
     switch (s) {

@@ -5,18 +5,17 @@
 // Fprop, Dgrad and Wgrad all from E4M3 operands, BF16 output).
 //
 // Persistent, warp-specialised CTA pairs: each 2-CTA cluster (one pair of
-// SMs) computes 256x256 output tiles with pair MMAs (tcgen05 cta_group::2,
-// M = 256): CTA r of the pair holds rows 128r..128r+127 of the A tile and
-// rows 128r..128r+127 of the B tile in its shared memory, and receives its
-// 128 rows x 256 columns of D in its own tensor memory.  Per SM this halves
-// the B bytes moved and read per MMA against a one-SM 128x256 tile, which is
-// what bounds the one-SM form's tensor-pipe utilisation.
-//   warp 0      TMA producer (both CTAs): A/B tiles (128-byte swizzle) and,
-//               for the block-scaled kind, the E8M0 scale vectors (already
-//               in the tensor-core layout: 512 bytes per 128 rows and four
-//               k-blocks; the CTA's own 128 rows of A, all 256 rows of B)
-//               into a 3-deep ring of 256-byte K stages (two k-blocks, two
-//               swizzle atoms each).  Both CTAs' copies of a stage count on
+// SMs) computes 256 x BN output tiles with pair MMAs (tcgen05 cta_group::2,
+// M = 256, N = BN): CTA r of the pair holds rows 128r..128r+127 of the A
+// tile and rows (BN/2)r..(BN/2)r+BN/2-1 of the B tile in its shared memory,
+// and receives its 128 rows x BN columns of D in its own tensor memory.  Per
+// SM this halves the B bytes moved and read per MMA against a one-SM tile.
+//   warp 0      TMA producer (both CTAs): A/B tiles (128-byte swizzle) into
+//               a 3-deep ring of 256-byte K stages (two k-blocks, two swizzle
+//               atoms each), and the E8M0 scale vectors of the CTA's 128 rows
+//               of A (already in the tensor-core layout: 512 bytes per 128
+//               rows and four k-blocks); with BN = 256 also those of the
+//               tile's 256 rows of B.  Both CTAs' copies of a stage count on
 //               the even CTA's `full` barrier.  Stages of two k-blocks (eight
 //               MMAs per stage hand-off) rather than one keep the tensor pipe
 //               busy across the per-stage barrier round trip.
@@ -27,19 +26,26 @@
 //               stage to both CTAs' producers and each accumulator to both
 //               CTAs' epilogues with multicast commits.  Both CTAs: tensor
 //               memory allocation (collective over the pair).
-//   warps 4..7  epilogue (both CTAs): tcgen05.ld the CTA's 128x256 FP32
-//               accumulator (one 32-lane quarter per warp) in two 128-column
-//               halves, release it to the even CTA's MMA warp, convert to
-//               BF16 (times scale_inv_a * scale_inv_b for the per-tensor
-//               kind) and TMA-store it through a swizzled staging tile.
+//   warp 2      BN = 224 only (both CTAs): builds the tensor-core image of
+//               the B scale vectors for tiles that start at any 32-row
+//               offset, which no TMA box can gather (see below).
+//   warps 4..7  epilogue (both CTAs): tcgen05.ld the CTA's 128 x BN FP32
+//               accumulator (one 32-lane quarter per warp), release it to
+//               the even CTA's MMA warp, convert to BF16 (times scale_inv_a *
+//               scale_inv_b for the per-tensor kind) and TMA-store it through
+//               a swizzled staging tile.
 // Accumulators in tensor memory (512 columns):
-//   dense kinds  two 256-column buffers, tiles alternate between them;
-//   block kind   the scale vectors need 24 columns, so two whole buffers do
-//               not fit: tiles alternate between columns [0, 256) and
-//               [128, 384), sharing [128, 256).  The epilogue reads the
-//               shared half first and releases the accumulator as soon as
-//               that half is in registers, so the next tile's MMAs wait for
-//               one half of the drain instead of all of it.
+//   dense kinds       two 256-column buffers, tiles alternate between them;
+//   block, BN = 256   the scale vectors need 24 columns, so two whole
+//                     buffers do not fit: tiles alternate between columns
+//                     [0, 256) and [128, 384), sharing [128, 256).  The
+//                     epilogue reads the shared half first and releases the
+//                     accumulator as soon as that half is in registers, so
+//                     the next tile's MMAs wait for half a drain.
+//   block, BN = 224   two independent buffers at columns 0 and 256 (scale
+//                     vectors at 480): the next tile never waits for a drain.
+//                     The host picks this form where the per-tile hand-off
+//                     of the 256 form would cost more than its narrower MMAs.
 // Every mbarrier wait is bounded in wall time; on expiry the CTA records
 // PURO_ERR_TIMEOUT in the caller's status word, drains its own in-flight
 // copies and MMAs (with a fixed bound), and both CTAs meet at a cluster
@@ -53,33 +59,40 @@ namespace puro {
 
 constexpr int kBM = kGemmBM;       // rows of A per CTA (= TMEM lanes); a pair tile has 2 * kBM rows
 constexpr int kPairM = 2 * kBM;    // rows of A per pair tile
-constexpr int kBN = kGemmBN;       // columns of a tile (= accumulator columns)
-constexpr int kBNHalf = kBN / 2;   // rows of B per CTA
 constexpr int kAtomBytes = kGemmBKBytes;       // one 128-byte swizzle row of K: one k-block of FP8
 constexpr int kAtoms = 2;                      // k-blocks per pipeline stage
 constexpr int kBKBytes = kAtoms * kAtomBytes;  // bytes of K per pipeline stage
-constexpr int kStages = 3;                     // 3 x 64 KB operand ring
+constexpr int kStages = 3;                     // 3-deep operand ring (64 KB / 60 KB per stage)
 constexpr int kStagesPerGroup = 512 / kBKBytes;  // stages per group of four k-blocks (one scale chunk)
 constexpr int kThreads = 256;
 constexpr int kTmemCols = 512;
-constexpr int kSfColsPerSet = 12;  // 4 for A (128 rows) + 8 for B (256 rows)
+constexpr int kSfColsPerSet = 12;  // 4 for A (128 rows) + 8 for B (up to 256 rows)
 constexpr int kSfSets = 2;         // double-buffered across groups of four k-blocks
+constexpr int kSfbSlots = 4;       // BN = 224: ring of helper-built B scale images
 constexpr uint64_t kDrainTimeoutNs = 2000000000ull;
 constexpr uint64_t kSettleNs = 200000ull;  // after an abort: let the peer-counted copies land
 constexpr int32_t kStatusTimeout = 4;  // PURO_ERR_TIMEOUT
 constexpr int64_t kSplitRefPairs = 76;  // SM pairs the split heuristic plans for (GB300: 152 SMs)
 static_assert(kAtomBytes == 128 && kStagesPerGroup * kBKBytes == 512, "whole k-blocks per stage, whole stages per group");
+static_assert(kAtoms == 2 && kStagesPerGroup == 2, "a stage holds k-blocks 2j, 2j+1 of a group of four");
 
+template <int BN>
 struct GemmSmem {
+    static constexpr int kBNHalf = BN / 2;                 // rows of B per CTA
+    static constexpr bool kSfbByHelper = (BN != 256);      // B scale images built by warp 2
     alignas(1024) uint8_t a[kStages][kAtoms][kBM * kAtomBytes];
     alignas(1024) uint8_t b[kStages][kAtoms][kBNHalf * kAtomBytes];
-    alignas(1024) uint8_t epi[4][32 * 128];    // per epilogue warp: 32 rows x 64 bf16
+    alignas(1024) uint8_t epi[4][32 * 128];    // per epilogue warp: 32 rows x 128 bytes
     alignas(128) uint8_t sf_a[kStages][512];   // scale vectors of this CTA's 128 rows of A
-    alignas(128) uint8_t sf_b[kStages][1024];  // scale vectors of the tile's 256 rows of B
+    // scale vectors of the tile's rows of B: per stage (TMA, BN = 256) or per
+    // slot of the helper's ring (BN = 224); 2 x 512 bytes = two tcgen05.cp images
+    alignas(128) uint8_t sf_b[kSfbByHelper ? kSfbSlots : kStages][1024];
     uint64_t full[kStages];   // even CTA: both CTAs' copies of a stage landed
     uint64_t empty[kStages];  // both CTAs: the pair MMAs reading a stage are done
     uint64_t tfull[2];        // both CTAs: accumulator complete
     uint64_t tempty[2];       // even CTA: both CTAs' epilogues released the accumulator
+    uint64_t sfb_full[kSfbSlots];   // even CTA (BN = 224): both CTAs' B scale images built
+    uint64_t sfb_empty[kSfbSlots];  // both CTAs (BN = 224): the copies reading an image are done
     uint64_t drain;
     uint32_t tmem_base;
     volatile int abort_flag;
@@ -94,6 +107,7 @@ struct GemmParams {
     int m_fastest;     // tile order: 1 = row blocks of A vary fastest
     int kgroups;       // ceil(K / 512): scale-vector chunks per 128 rows
     uint32_t idesc;
+    const uint8_t *sfb;  // scale vectors of B (BN = 224: read by the helper warp)
     const float *sia;
     const float *sib;
     int32_t *status;
@@ -101,35 +115,37 @@ struct GemmParams {
 };
 
 // Instruction descriptors (tcgen05.mma), both operands K-major, M = 256
-// (a pair MMA), N = kBN.
+// (a pair MMA), N = bn.
 //   kind::f16 / kind::f8f6f4: [4,6) D format (1 = F32), [7,10) A type,
 //     [10,13) B type, [17,23) N >> 3, [24,29) M >> 4.
 //   kind::mxf8f6f4: [4,6) B scale id, [7,10) A type, [10,13) B type,
 //     [17,23) N >> 3, [23] scale type (1 = UE8M0), [24,29) M >> 4,
 //     [29,31) A scale id.  The scale id selects the byte of the 32-bit
 //     tensor-memory scale word: here the k-block within its group of four.
-__host__ __device__ constexpr uint32_t idesc_dense(uint32_t atype, uint32_t btype) {
-    return (1u << 4) | (atype << 7) | (btype << 10) | (static_cast<uint32_t>(kBN >> 3) << 17) |
+__host__ __device__ constexpr uint32_t idesc_dense(uint32_t atype, uint32_t btype, int bn) {
+    return (1u << 4) | (atype << 7) | (btype << 10) | (static_cast<uint32_t>(bn >> 3) << 17) |
            (static_cast<uint32_t>(kPairM >> 4) << 24);
 }
-__host__ __device__ constexpr uint32_t idesc_mx(uint32_t atype, uint32_t btype) {
-    return (atype << 7) | (btype << 10) | (static_cast<uint32_t>(kBN >> 3) << 17) | (1u << 23) |
+__host__ __device__ constexpr uint32_t idesc_mx(uint32_t atype, uint32_t btype, int bn) {
+    return (atype << 7) | (btype << 10) | (static_cast<uint32_t>(bn >> 3) << 17) | (1u << 23) |
            (static_cast<uint32_t>(kPairM >> 4) << 24);
 }
 
-PURO_DEV void record_timeout(GemmSmem &sm, int32_t *status) {
+template <int BN>
+PURO_DEV void record_timeout(GemmSmem<BN> &sm, int32_t *status) {
     sm.abort_flag = 1;
     if (status) atomicExch(status, kStatusTimeout);
 }
 
-// One unit of work: a 256x256 pair tile and a chunk of the reduction.  Units
-// of the same chunk are consecutive; within a chunk the tile order iterates
-// the blocks of the smaller operand fastest, so the pairs of a wave share
-// (and read once) the blocks of the larger one.
+// One unit of work: a 256 x BN pair tile and a chunk of the reduction.
+// Units of the same chunk are consecutive; within a chunk the tile order
+// iterates the blocks of the smaller operand fastest, so the pairs of a wave
+// share (and read once) the blocks of the larger one.
 struct WorkUnit {
     int m0, n0, kb0, kb1, split;  // m0: first row of the pair tile
 };
 
+template <int BN>
 PURO_DEV WorkUnit work_unit(const GemmParams &p, int u) {
     WorkUnit w;
     w.split = u / p.num_tiles;
@@ -137,37 +153,61 @@ PURO_DEV WorkUnit work_unit(const GemmParams &p, int u) {
     const int mb = p.m_fastest ? tile % p.num_m : tile / p.num_n;
     const int nb = p.m_fastest ? tile / p.num_m : tile % p.num_n;
     w.m0 = mb * kPairM;
-    w.n0 = nb * kBN;
+    w.n0 = nb * BN;
     w.kb0 = w.split * p.kb_per_split;
     w.kb1 = min(p.num_kb, w.kb0 + p.kb_per_split);
     return w;
 }
 
+// Convert 32 FP32 accumulator columns of this thread's row to BF16 (times sab
+// for the per-tensor kind) into four 16-byte units.
+template <int KIND>
+PURO_DEV void pack_bf16x8(const uint32_t *src, float sab, uint32_t (&w)[4]) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        float lo = __uint_as_float(src[2 * j]), hi = __uint_as_float(src[2 * j + 1]);
+        if constexpr (KIND == kGemmFP8Tensor) {
+            lo = __fmul_rn(lo, sab);
+            hi = __fmul_rn(hi, sab);
+        }
+        __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+        w[j] = *reinterpret_cast<uint32_t *>(&v);
+    }
+}
+
 // OUT_F32: write FP32 partial tiles of a split reduction to the workspace
 // [splits * Mp, N], Mp = num_m * 256 (rows split * Mp + m), instead of the
-// BF16 output; a ragged last pair tile then stays inside its chunk.
+// BF16 output; a ragged last pair tile then stays inside its chunk (BN = 256
+// only).  tm_d: D with box {64, 32} and the 128-byte swizzle (BN = 256) or
+// box {32, 32} and the 64-byte swizzle (BN = 224).
 // tm_sfa / tm_sfb (block kind only): the scale vectors of A / B viewed as
-// uint32 [chunks, 128] (one 512-byte chunk per row), box {128, 1}.
-template <int KIND, bool OUT_F32>
+// uint32 [chunks, 128] (one 512-byte chunk per row), box {128, 1}; tm_sfb is
+// read only with BN = 256.
+template <int KIND, bool OUT_F32, int BN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     gemm_tn_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
                    const __grid_constant__ CUtensorMap tm_d, const __grid_constant__ CUtensorMap tm_sfa,
                    const __grid_constant__ CUtensorMap tm_sfb, const GemmParams p) {
+    using Smem = GemmSmem<BN>;
+    constexpr int kBNHalf = Smem::kBNHalf;
     constexpr bool kMX = (KIND == kGemmFP8Block);
-    constexpr int kAccBufs = kMX ? 1 : 2;              // hand-off barrier pairs (tfull / tempty)
-    constexpr int kAccShift = kMX ? kBN / 2 : kBN;     // column offset between consecutive tiles' accumulators
-    constexpr int kSfBase = kBN + kAccShift;           // first scale-vector column (MX)
+    constexpr bool kHelper = kMX && Smem::kSfbByHelper;
+    constexpr bool kShifted = kMX && BN == 256;         // shared-half accumulators
+    constexpr int kAccBufs = kShifted ? 1 : 2;          // hand-off barrier pairs (tfull / tempty)
+    constexpr int kAccShift = kShifted ? 128 : 256;     // column offset between consecutive tiles' accumulators
+    constexpr int kSfBase = kShifted ? 384 : 480;       // first scale-vector column (MX)
     constexpr int kElemBytes = (KIND == kGemmBF16) ? 2 : 1;
-    constexpr int kBK = kBKBytes / kElemBytes;         // elements of K per stage
-    constexpr int kAtomK = kAtomBytes / kElemBytes;    // elements of K per 128-byte atom
-    constexpr int kKSteps = kAtomBytes / 32;           // MMAs per atom (32 bytes of K each)
+    constexpr int kBK = kBKBytes / kElemBytes;          // elements of K per stage
+    constexpr int kAtomK = kAtomBytes / kElemBytes;     // elements of K per 128-byte atom
+    constexpr int kKSteps = kAtomBytes / 32;            // MMAs per atom (32 bytes of K each)
     constexpr uint32_t kStageBytes = (kBM + kBNHalf) * kBKBytes;  // one CTA's operand bytes per stage
-    constexpr uint32_t kSfBytes = 512 + 1024;                     // one CTA's scale-vector bytes per group
+    constexpr uint32_t kSfBytes = kHelper ? 512u : 512u + 1024u;  // one CTA's TMA scale bytes per group
+    static_assert(BN == 256 || (BN == 224 && kMX && !OUT_F32), "the 224-wide form is block-scaled, BF16 out");
     static_assert(!kMX || kSfBase + kSfSets * kSfColsPerSet <= kTmemCols, "TMEM budget");
+    static_assert(kAccShift + BN <= (kMX ? kSfBase : kTmemCols), "accumulators clear of the scale columns");
 
     extern __shared__ uint8_t smem_raw[];
-    GemmSmem &sm = *reinterpret_cast<GemmSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                                 ~static_cast<uintptr_t>(1023));
+    Smem &sm = *reinterpret_cast<Smem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const uint32_t rank = cluster_ctarank();  // 0: even CTA (issues the MMAs), 1: its peer
@@ -183,6 +223,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             mbar_init(&sm.tfull[b], 1);
             mbar_init(&sm.tempty[b], 8);  // four epilogue warps in each CTA
         }
+        for (int s = 0; s < kSfbSlots; ++s) {
+            mbar_init(&sm.sfb_full[s], 2);  // the helper warp of each CTA
+            mbar_init(&sm.sfb_empty[s], 1);
+        }
         mbar_init(&sm.drain, 1);
         sm.abort_flag = 0;
         fence_mbarrier_init();
@@ -191,7 +235,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         tma_prefetch_desc(&tm_d);
         if (kMX) {
             tma_prefetch_desc(&tm_sfa);
-            tma_prefetch_desc(&tm_sfb);
+            if (!kHelper) tma_prefetch_desc(&tm_sfb);
         }
     }
     if (warp == 1) {
@@ -212,7 +256,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             uint32_t issued = 0;  // stage fills started by this thread
             bool aborted = false;
             for (int u = pair; u < p.num_units && !aborted; u += num_pairs) {
-                const WorkUnit wu = work_unit(p, u);
+                const WorkUnit wu = work_unit<BN>(p, u);
                 const int a_row = wu.m0 + kBM * static_cast<int>(rank);
                 const int b_row = wu.n0 + kBNHalf * static_cast<int>(rank);
                 for (int kb = wu.kb0; kb < wu.kb1; ++kb) {
@@ -234,9 +278,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         // chunks beyond the operand's rows read as zero (their rows are zero too)
                         const int kg = kb / kStagesPerGroup;
                         tma_load_2d_pair(sm.sf_a[stage], &tm_sfa, full_bar, 0, (a_row / 128) * p.kgroups + kg);
-                        tma_load_2d_pair(sm.sf_b[stage], &tm_sfb, full_bar, 0, (wu.n0 / 128) * p.kgroups + kg);
-                        tma_load_2d_pair(sm.sf_b[stage] + 512, &tm_sfb, full_bar, 0,
-                                         (wu.n0 / 128 + 1) * p.kgroups + kg);
+                        if constexpr (!kHelper) {
+                            tma_load_2d_pair(sm.sf_b[stage], &tm_sfb, full_bar, 0, (wu.n0 / 128) * p.kgroups + kg);
+                            tma_load_2d_pair(sm.sf_b[stage] + 512, &tm_sfb, full_bar, 0,
+                                             (wu.n0 / 128 + 1) * p.kgroups + kg);
+                        }
                     }
                     ++issued;
                     if (++stage == kStages) {
@@ -265,10 +311,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     } else if (warp == 1 && rank == 0) {
         // ------------------------------------------------ MMA issuer (even CTA)
         uint32_t stage = 0, phase = 0;
+        uint32_t gseq = 0;  // groups of four k-blocks started (BN = 224: slot of the scale ring)
         bool aborted = false;
         int local = 0;
         for (int u = pair; u < p.num_units && !aborted; u += num_pairs, ++local) {
-            const WorkUnit wu = work_unit(p, u);
+            const WorkUnit wu = work_unit<BN>(p, u);
             const int buf = local % kAccBufs;
             const uint32_t acc_phase = static_cast<uint32_t>(local / kAccBufs) & 1u;
             bool ok = (sm.abort_flag == 0) && mbar_wait_bounded(&sm.tempty[buf], acc_phase ^ 1u, p.wait_ns);
@@ -281,7 +328,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             const uint32_t d_tmem = tmem + static_cast<uint32_t>((local & 1) * kAccShift);
 
             for (int kb = wu.kb0; kb < wu.kb1; ++kb) {
+                const bool group_start = kMX && (kb % kStagesPerGroup) == 0;
+                const uint32_t slot = gseq % kSfbSlots;
                 ok = (sm.abort_flag == 0) && mbar_wait_bounded(&sm.full[stage], phase, p.wait_ns);
+                if (kHelper && group_start)
+                    ok = ok && mbar_wait_bounded(&sm.sfb_full[slot], (gseq / kSfbSlots) & 1u, p.wait_ns);
                 if (!__all_sync(0xFFFFFFFFu, ok)) {
                     if (lane == 0) record_timeout(sm, p.status);
                     aborted = true;
@@ -292,13 +343,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     const uint32_t sfa_col = kSfBase + ((kb / kStagesPerGroup) & 1) * kSfColsPerSet;
                     const uint32_t sfb_col = sfa_col + 4;
                     if constexpr (kMX) {
-                        if (kb % kStagesPerGroup == 0) {  // new group of four k-blocks: its scale vectors
+                        if (group_start) {  // new group of four k-blocks: its scale vectors
+                            const uint8_t *sfb_src = kHelper ? sm.sf_b[slot] : sm.sf_b[stage];
                             tmem_cp_pair_32x128b_warpx4(tmem + sfa_col,
                                                         smem_desc_plain_16B_rows(smem_u32(sm.sf_a[stage])));
-                            tmem_cp_pair_32x128b_warpx4(tmem + sfb_col,
-                                                        smem_desc_plain_16B_rows(smem_u32(sm.sf_b[stage])));
+                            tmem_cp_pair_32x128b_warpx4(tmem + sfb_col, smem_desc_plain_16B_rows(smem_u32(sfb_src)));
                             tmem_cp_pair_32x128b_warpx4(tmem + sfb_col + 4,
-                                                        smem_desc_plain_16B_rows(smem_u32(sm.sf_b[stage] + 512)));
+                                                        smem_desc_plain_16B_rows(smem_u32(sfb_src + 512)));
                         }
                     }
 #pragma unroll
@@ -324,8 +375,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         }
                     }
                     tc_commit_pair_multicast(&sm.empty[stage], 0x3);  // stage reusable in both CTAs
+                    // the scale image is free once its copies (issued above) are done
+                    if (kHelper && group_start) tc_commit_pair_multicast(&sm.sfb_empty[slot], 0x3);
                 }
                 __syncwarp();
+                if (group_start) ++gseq;
                 if (++stage == kStages) {
                     stage = 0;
                     phase ^= 1u;
@@ -341,6 +395,53 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             mbar_wait_bounded(&sm.drain, 0, kDrainTimeoutNs);
         }
         __syncwarp();
+    } else if ((warp == 2 || warp == 3) && kHelper) {
+        // ------------------------------------------------ B scale images (BN = 224, both CTAs)
+        // A tile's rows of B start at a multiple of 32 that need not be a
+        // multiple of 128, so the 512-byte chunks of the scale-vector layout
+        // do not line up with the tile.  For each group of four k-blocks a
+        // helper warp gathers the words the MMA needs -- lane l, column j:
+        // row n0 + 32j + l -- into two 512-byte tcgen05.cp images.  Warps 2
+        // and 3 take alternate groups, so the L2 round trip of one group's
+        // loads overlaps the next.
+        const uint32_t sfb_full0 = mapa_shared(smem_u32(&sm.sfb_full[0]), 0);  // the even CTA's
+        const uint32_t *sfb_words = reinterpret_cast<const uint32_t *>(p.sfb);
+        const uint32_t mine = static_cast<uint32_t>(warp - 2);
+        uint32_t gseq = 0;
+        bool aborted = false;
+        for (int u = pair; u < p.num_units && !aborted; u += num_pairs) {
+            const WorkUnit wu = work_unit<BN>(p, u);
+            for (int kb = wu.kb0; kb < wu.kb1; kb += kStagesPerGroup, ++gseq) {
+                if ((gseq & 1u) != mine) continue;
+                const uint32_t slot = gseq % kSfbSlots;
+                const bool ok = (sm.abort_flag == 0) &&
+                                mbar_wait_bounded(&sm.sfb_empty[slot], ((gseq / kSfbSlots) & 1u) ^ 1u, p.wait_ns);
+                if (!__all_sync(0xFFFFFFFFu, ok)) {
+                    if (lane == 0) record_timeout(sm, p.status);
+                    aborted = true;
+                    break;
+                }
+                const int kg = kb / kStagesPerGroup;
+                uint32_t words[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const int grp = wu.n0 / 32 + j;  // 32-row group of B
+                    // rows past N (and the eighth column) hold no data: 2^0
+                    words[j] = (j < BN / 32 && 32 * grp < p.N)
+                                   ? __ldg(sfb_words + ((static_cast<int64_t>(grp / 4) * p.kgroups + kg) * 128 +
+                                                        4 * lane + (grp % 4)))
+                                   : 0x7F7F7F7Fu;
+                }
+                uint8_t *img = sm.sf_b[slot];
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+                    *reinterpret_cast<uint4 *>(img + 512 * h + 16 * lane) =
+                        make_uint4(words[4 * h], words[4 * h + 1], words[4 * h + 2], words[4 * h + 3]);
+                fence_proxy_async_smem();  // generic writes -> the tensor core's copy
+                __syncwarp();
+                if (lane == 0) mbar_arrive_cluster(sfb_full0 + 8u * slot);
+            }
+        }
     } else if (warp >= 4) {
         // ------------------------------------------------ epilogue (both CTAs)
         const int q = warp & 3;  // TMEM lane quarter of this warp
@@ -349,8 +450,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         uint8_t *stage_buf = sm.epi[q];
         const uint32_t tempty0 = mapa_shared(smem_u32(&sm.tempty[0]), 0);  // the even CTA's
         int local = 0;
+        uint32_t pieces = 0;  // BN = 224: 32-column pieces stored, alternating staging halves
         for (int u = pair; u < p.num_units; u += num_pairs, ++local) {
-            const WorkUnit wu = work_unit(p, u);
+            const WorkUnit wu = work_unit<BN>(p, u);
             const int m0 = wu.m0 + kBM * static_cast<int>(rank), n0 = wu.n0;  // this CTA's rows
             const int buf = local % kAccBufs;
             const uint32_t acc_phase = static_cast<uint32_t>(local / kAccBufs) & 1u;
@@ -366,7 +468,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 // FP32 partial tile: 8 chunks of 32 columns (128 bytes per row)
                 const int row0 = wu.split * p.num_m * kPairM + m0 + 32 * q;  // chunks pair-tile aligned
 #pragma unroll
-                for (int h = 0; h < kBN / 128; ++h) {
+                for (int h = 0; h < BN / 128; ++h) {
                     uint32_t r[4][32];
 #pragma unroll
                     for (int c = 0; c < 4; ++c) tmem_ld_32x32b_x32(t_row + 128 * h + 32 * c, r[c]);
@@ -400,12 +502,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 tc_fence_before_sync();
                 __syncwarp();
                 if (lane == 0) mbar_arrive_cluster(tempty0 + 8u * buf);
-            } else {
-                // Block kind: the half in the columns the next tile's
-                // accumulator shares ([128, 256) of tensor memory) first, and
-                // the accumulator released once it is in registers.  Dense
-                // kinds: halves in order, released after the second load.
-                const int h_first = kMX ? ((local & 1) ? 0 : 1) : 0;
+            } else if constexpr (BN == 256) {
+                // Shifted (block kind): the half in the columns the next
+                // tile's accumulator shares ([128, 256) of tensor memory)
+                // first, and the accumulator released once it is in
+                // registers.  Dense kinds: halves in order, released after
+                // the second load.
+                const int h_first = kShifted ? ((local & 1) ? 0 : 1) : 0;
 #pragma unroll 1
                 for (int hh = 0; hh < 2; ++hh) {
                     const int h = hh ^ h_first;
@@ -413,7 +516,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int c = 0; c < 4; ++c) tmem_ld_32x32b_x32(t_row + 128 * h + 32 * c, r[c]);
                     tmem_ld_wait();
-                    if (hh == (kMX ? 0 : 1)) {
+                    if (hh == (kShifted ? 0 : 1)) {
                         tc_fence_before_sync();
                         __syncwarp();
                         if (lane == 0) mbar_arrive_cluster(tempty0 + 8u * buf);  // accumulator free for the next tile
@@ -429,18 +532,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         uint8_t *row = stage_buf + 128 * lane;
 #pragma unroll
                         for (int i = 0; i < 8; ++i) {
-                            const uint32_t *src = &r[2 * ch + (i >> 2)][8 * (i & 3)];
                             uint32_t w[4];
-#pragma unroll
-                            for (int j = 0; j < 4; ++j) {
-                                float lo = __uint_as_float(src[2 * j]), hi = __uint_as_float(src[2 * j + 1]);
-                                if constexpr (KIND == kGemmFP8Tensor) {
-                                    lo = __fmul_rn(lo, sab);
-                                    hi = __fmul_rn(hi, sab);
-                                }
-                                __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-                                w[j] = *reinterpret_cast<uint32_t *>(&v);
-                            }
+                            pack_bf16x8<KIND>(&r[2 * ch + (i >> 2)][8 * (i & 3)], sab, w);
                             *reinterpret_cast<uint4 *>(row + 16 * (i ^ (lane & 7))) = make_uint4(w[0], w[1], w[2], w[3]);
                         }
                         fence_proxy_async_smem();
@@ -449,6 +542,49 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                             tma_store_2d(&tm_d, stage_buf, col, m0 + 32 * q);
                             bulk_commit_group();
                         }
+                    }
+                }
+            } else {
+                // BN = 224, double-buffered: columns [0, 128) then [128, 224),
+                // released after the second load; 32-column pieces (64 bytes
+                // per row, 64-byte swizzle: 16-byte unit i of row l at
+                // i ^ ((l / 2) % 4)) alternate between the two 2 KB halves of
+                // the staging tile, so a piece is written while the previous
+                // one is still being stored.
+#pragma unroll 1
+                for (int hh = 0; hh < 2; ++hh) {
+                    const int nc = hh == 0 ? 4 : (BN - 128) / 32;
+                    uint32_t r[4][32];
+#pragma unroll
+                    for (int c = 0; c < 4; ++c)
+                        if (c < nc) tmem_ld_32x32b_x32(t_row + 128 * hh + 32 * c, r[c]);
+                    tmem_ld_wait();
+                    if (hh == 1) {
+                        tc_fence_before_sync();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive_cluster(tempty0 + 8u * buf);  // accumulator free
+                    }
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        const int col = n0 + 128 * hh + 32 * c;
+                        if (c >= nc || col >= p.N) break;
+                        uint8_t *half = stage_buf + 2048 * (pieces & 1u);
+                        if (lane == 0) bulk_wait_group_read<1>();  // the store that last read this half is done
+                        __syncwarp();
+                        uint8_t *row = half + 64 * lane;
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            uint32_t w[4];
+                            pack_bf16x8<KIND>(&r[c][8 * i], sab, w);
+                            *reinterpret_cast<uint4 *>(row + 16 * (i ^ ((lane >> 1) & 3))) = make_uint4(w[0], w[1], w[2], w[3]);
+                        }
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) {
+                            tma_store_2d(&tm_d, half, col, m0 + 32 * q);
+                            bulk_commit_group();
+                        }
+                        ++pieces;
                     }
                 }
             }
@@ -485,7 +621,7 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const float4 *__rest
 
 int choose_splits(int64_t M, int64_t N, int64_t K, bool bf16) {
     if (bf16) return 1;
-    const int64_t tiles = ((M + kPairM - 1) / kPairM) * ((N + kBN - 1) / kBN);
+    const int64_t tiles = ((M + kPairM - 1) / kPairM) * ((N + 255) / 256);
     const int64_t kblocks = (K + 127) / 128;  // 128-byte k-blocks
     if (tiles >= kSplitRefPairs) return 1;
     // Modelled time = waves x k-blocks per chunk; chunks keep >= 16 k-blocks
@@ -509,6 +645,23 @@ int choose_splits(int64_t M, int64_t N, int64_t K, bool bf16) {
     return (best_cost * 100 <= base * 85) ? best : 1;
 }
 
+// Tile width of an unsplit block-scaled GEMM.  Modelled pair time = waves x
+// per-tile cycles, with constants fitted to measured GB300 times of both
+// forms: about 163 cycles per pair MMA plus a 2500-cycle accumulator hand-off
+// per tile for the 256-wide form, 170 cycles per MMA plus 350 per tile for
+// the 224-wide one.  The narrower form has more tiles, so it pays off only
+// where the hand-off dominates (short reductions) and the extra tiles do not
+// add a wave; it is taken only for a modelled gain above 5.5%, the margin the
+// fit needed to match every measured shape.
+int choose_tile_n(int64_t M, int64_t N, int64_t K) {
+    const int64_t stages = (K + kBKBytes - 1) / kBKBytes;
+    const int64_t m_tiles = (M + kPairM - 1) / kPairM;
+    auto waves = [&](int64_t bn) { return (m_tiles * ((N + bn - 1) / bn) + kSplitRefPairs - 1) / kSplitRefPairs; };
+    const int64_t c256 = waves(256) * (stages * kAtoms * 4 * 163 + 2500);
+    const int64_t c224 = waves(224) * (stages * kAtoms * 4 * 170 + 350);
+    return c224 * 1000 < c256 * 945 ? 224 : 256;
+}
+
 int64_t splitk_rows_per_chunk(int64_t M) { return (M + kPairM - 1) / kPairM * kPairM; }
 
 size_t splitk_workspace_bytes(int64_t M, int64_t N, int64_t K, bool bf16) {
@@ -520,7 +673,7 @@ size_t splitk_workspace_bytes(int64_t M, int64_t N, int64_t K, bool bf16) {
 
 // Pairs that can be resident at once for this kernel (the persistent grid
 // size), cached per device and kernel.
-template <int KIND, bool OUT_F32>
+template <int KIND, bool OUT_F32, int BN>
 static int max_resident_pairs(int num_sms, size_t smem) {
     static int cache[64] = {0};
     int dev = 0;
@@ -538,7 +691,7 @@ static int max_resident_pairs(int num_sms, size_t smem) {
     cfg.attrs = &attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, gemm_tn_kernel<KIND, OUT_F32>, &cfg) != cudaSuccess || n <= 0) {
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tn_kernel<KIND, OUT_F32, BN>, &cfg) != cudaSuccess || n <= 0) {
         (void)cudaGetLastError();
         n = num_sms / 2;
     }
@@ -546,7 +699,7 @@ static int max_resident_pairs(int num_sms, size_t smem) {
     return n;
 }
 
-template <int KIND, bool OUT_F32>
+template <int KIND, bool OUT_F32, int BN>
 static cudaError_t launch_kind(const GemmArgs &g, const GemmMaps &m, int splits, cudaStream_t s) {
     constexpr int kElemBytes = (KIND == kGemmBF16) ? 2 : 1;
     constexpr int kBK = kBKBytes / kElemBytes;
@@ -555,7 +708,7 @@ static cudaError_t launch_kind(const GemmArgs &g, const GemmMaps &m, int splits,
     p.N = static_cast<int>(g.N);
     p.K = static_cast<int>(g.K);
     p.num_m = static_cast<int>((g.M + kPairM - 1) / kPairM);
-    p.num_n = static_cast<int>((g.N + kBN - 1) / kBN);
+    p.num_n = static_cast<int>((g.N + BN - 1) / BN);
     p.num_kb = static_cast<int>((g.K + kBK - 1) / kBK);
     p.num_tiles = p.num_m * p.num_n;
     p.splits = splits;
@@ -564,22 +717,23 @@ static cudaError_t launch_kind(const GemmArgs &g, const GemmMaps &m, int splits,
     p.num_units = p.num_tiles * p.splits;
     p.m_fastest = g.M < g.N ? 1 : 0;  // re-read the smaller operand, stream the larger once
     if (KIND == kGemmBF16)
-        p.idesc = idesc_dense(1u, 1u);
+        p.idesc = idesc_dense(1u, 1u, BN);
     else if (KIND == kGemmFP8Tensor)
-        p.idesc = idesc_dense(static_cast<uint32_t>(g.a_fmt), static_cast<uint32_t>(g.b_fmt));
+        p.idesc = idesc_dense(static_cast<uint32_t>(g.a_fmt), static_cast<uint32_t>(g.b_fmt), BN);
     else
-        p.idesc = idesc_mx(static_cast<uint32_t>(g.a_fmt), static_cast<uint32_t>(g.b_fmt));
+        p.idesc = idesc_mx(static_cast<uint32_t>(g.a_fmt), static_cast<uint32_t>(g.b_fmt), BN);
     p.kgroups = static_cast<int>((g.K / 128 + 3) / 4);
+    p.sfb = g.sfb;
     p.sia = g.sia;
     p.sib = g.sib;
     p.status = g.status;
     p.wait_ns = g.wait_timeout_ns;
 
-    auto kern = gemm_tn_kernel<KIND, OUT_F32>;
-    const size_t smem = sizeof(GemmSmem) + 1024;
+    auto kern = gemm_tn_kernel<KIND, OUT_F32, BN>;
+    const size_t smem = sizeof(GemmSmem<BN>) + 1024;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    const int pairs_max = max_resident_pairs<KIND, OUT_F32>(g.num_sms, smem);
+    const int pairs_max = max_resident_pairs<KIND, OUT_F32, BN>(g.num_sms, smem);
     const int pairs = p.num_units < pairs_max ? p.num_units : pairs_max;
     kern<<<2 * pairs, kThreads, smem, s>>>(m.a, m.b, OUT_F32 ? m.ws : m.d, m.sfa, m.sfb, p);
     return cudaGetLastError();
@@ -587,8 +741,12 @@ static cudaError_t launch_kind(const GemmArgs &g, const GemmMaps &m, int splits,
 
 template <int KIND>
 static cudaError_t launch_split_or_not(const GemmArgs &g, const GemmMaps &m, cudaStream_t s) {
-    if (g.splits <= 1) return launch_kind<KIND, false>(g, m, 1, s);
-    cudaError_t e = launch_kind<KIND, true>(g, m, g.splits, s);
+    if (g.splits <= 1) {
+        if constexpr (KIND == kGemmFP8Block)
+            if (g.tile_n == 224) return launch_kind<KIND, false, 224>(g, m, 1, s);
+        return launch_kind<KIND, false, 256>(g, m, 1, s);
+    }
+    cudaError_t e = launch_kind<KIND, true, 256>(g, m, g.splits, s);
     if (e != cudaSuccess) return e;
     const int64_t n4 = g.M * g.N / 4;
     const int64_t stride4 = splitk_rows_per_chunk(g.M) * g.N / 4;
@@ -602,7 +760,7 @@ static cudaError_t launch_split_or_not(const GemmArgs &g, const GemmMaps &m, cud
 
 cudaError_t launch_gemm(const GemmArgs &g, const GemmMaps &m, cudaStream_t s) {
     switch (g.kind) {
-        case kGemmBF16: return launch_kind<kGemmBF16, false>(g, m, 1, s);
+        case kGemmBF16: return launch_kind<kGemmBF16, false, 256>(g, m, 1, s);
         case kGemmFP8Tensor: return launch_split_or_not<kGemmFP8Tensor>(g, m, s);
         default: return launch_split_or_not<kGemmFP8Block>(g, m, s);
     }

@@ -53,6 +53,10 @@ struct GemmArgs {
     GemmKind kind;
     int a_fmt, b_fmt;            // FP8 formats (0 = E4M3, 1 = E5M2)
     int64_t M, N, K;
+    int tile_n;                  // 256, or 224 (block kind, unsplit; see choose_tile_n)
+    // kGemmFP8Block: scale vectors of B (the 224-wide form gathers them
+    // itself; the 256-wide form loads them through GemmMaps::sfb).
+    const uint8_t *sfb;
     // kGemmFP8Tensor: dequantisation factors of A and B.
     const float *sia, *sib;
     int32_t *status;             // optional device status word
@@ -67,8 +71,9 @@ struct GemmArgs {
 
 // Tensor maps of one GEMM launch.
 //   a:   A [M, K] (128-byte swizzle, box {128 bytes, 128 rows})
-//   b:   B [N, K] (the same box: half of a 256-row tile per CTA)
-//   d:   D [M, N] bf16 (128-byte swizzle, box {64, 32})
+//   b:   B [N, K] (box {128 bytes, tile_n / 2 rows}: half of a tile per CTA)
+//   d:   D [M, N] bf16 (tile_n 256: 128-byte swizzle, box {64, 32};
+//        tile_n 224: 64-byte swizzle, box {32, 32})
 //   ws:  workspace [splits * splitk_rows_per_chunk(M), N] fp32 (128-byte
 //        swizzle, box {32, 32}); only read when g.splits > 1
 //   sfa, sfb (kGemmFP8Block only): the scale vectors of A / B,
@@ -90,6 +95,9 @@ puro_status_t fp8_gemm_entry(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t
 int choose_splits(int64_t M, int64_t N, int64_t K, bool bf16);
 size_t splitk_workspace_bytes(int64_t M, int64_t N, int64_t K, bool bf16);
 int64_t splitk_rows_per_chunk(int64_t M);  // M rounded up to a whole 256-row pair tile
+// Tile width (256 or 224) of an unsplit block-scaled GEMM: modelled waves x
+// per-tile time of the two forms.  Host-only, shape-only.
+int choose_tile_n(int64_t M, int64_t N, int64_t K);
 
 // Tile shape of the GEMM kernel: rows of A per CTA (a CTA pair computes
 // 2 * kGemmBM rows), columns of a tile (rows of B per pair), and the bytes

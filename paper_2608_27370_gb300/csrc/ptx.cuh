@@ -109,6 +109,9 @@ PURO_DEV void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *ba
 PURO_DEV void bulk_commit_group() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 // Wait until all committed bulk stores have finished reading shared memory.
 PURO_DEV void bulk_wait_group_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// Wait until at most N committed bulk stores still read shared memory.
+template <int N>
+PURO_DEV void bulk_wait_group_read() { asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory"); }
 // Wait until all committed bulk stores are complete.
 PURO_DEV void bulk_wait_group0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 

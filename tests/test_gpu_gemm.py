@@ -2,8 +2,10 @@
 against the oracle's fp64 products, element by element, within
 |gpu - ref| <= 2^-7 |ref| + 1e-3 rms(ref).
 
-Shapes span several output tiles (128 x 256) with ragged last tiles; the
-per-tensor and BF16 cases also have ragged reduction tails.
+Shapes span several output tiles (256 x 256 or 256 x 224 pair tiles) with
+ragged last tiles; the per-tensor and BF16 cases also have ragged reduction
+tails.  The block-scaled cases run with each tile form forced and with the
+per-shape choice.
 """
 import numpy as np
 import pytest
@@ -32,8 +34,16 @@ def _inputs(M, N, K, seed, t3=False):
     return x, w, dy
 
 
-@pytest.mark.parametrize("M,N,K", [(128, 128, 128), (384, 640, 384), (256, 1536, 1536), (512, 256, 1024)])
-def test_block_linear(M, N, K):
+@pytest.fixture(params=[0, 224, 256], ids=["tile_auto", "tile224", "tile256"])
+def tile_n(request):
+    P.puro_set_gemm_tile_n(request.param)
+    yield request.param
+    P.puro_set_gemm_tile_n(0)
+
+
+@pytest.mark.parametrize("M,N,K", [(128, 128, 128), (384, 640, 384), (256, 1536, 1536), (512, 256, 1024),
+                                   (640, 1152, 2560)])
+def test_block_linear(M, N, K, tile_n):
     x, w, dy = _inputs(M, N, K, 1000 + M + N + K, t3=True)
     out = run_linear(x, w, dy, P.SCALE_BLOCK)
     ref = oracle_linear(x, w, dy, P.SCALE_BLOCK)
@@ -43,7 +53,7 @@ def test_block_linear(M, N, K):
 
 
 @pytest.mark.parametrize("fmts", [(P.E4M3, P.E4M3, P.E5M2), (P.E5M2, P.E5M2, P.E5M2)])
-def test_block_linear_e5m2(fmts):
+def test_block_linear_e5m2(fmts, tile_n):
     M, N, K = 256, 384, 256
     x, w, dy = _inputs(M, N, K, 77)
     out = run_linear(x, w, dy, P.SCALE_BLOCK, *fmts)

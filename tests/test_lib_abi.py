@@ -162,3 +162,10 @@ def test_binding_refuses_host_tensors():
     x = torch.zeros(128, 128, dtype=torch.bfloat16)
     with pytest.raises(ValueError):
         P.puro_fp8_amax(x, torch.zeros(1, dtype=torch.int32))
+
+
+def test_gemm_tile_knob_validates_on_the_host(lib):
+    assert lib.puro_set_gemm_tile_n(192) == P.PURO_ERR_INVALID_ARG
+    assert lib.puro_set_gemm_tile_n(-1) == P.PURO_ERR_INVALID_ARG
+    for v in (224, 256, 0):
+        assert lib.puro_set_gemm_tile_n(v) == P.PURO_OK
