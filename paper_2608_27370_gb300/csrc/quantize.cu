@@ -255,10 +255,15 @@ __global__ void __launch_bounds__(kQThreads, 2)
         if (tid == 0) {
             const int next = tile + gridDim.x;
             if (next < ntiles) issue_load(next, buf ^ 1);  // its buffer was last read before (S2) of it-1
-            bulk_wait_group_read0();                        // previous tile's stores have read the staging
+            // The previous tile's TMA stores must have read the staging tiles
+            // before they are rewritten.  Per-tensor mode writes them right
+            // after (S1); the blockwise modes first spend phase A (and B) on
+            // the scales, so they wait just before the last barrier ahead of
+            // phase C and the stores' reads overlap that work.
+            if constexpr (KIND == kQuantTensor) bulk_wait_group_read0();
         }
         mbar_wait_bounded(&sm.full[buf], static_cast<uint32_t>(it >> 1) & 1u, kQuantWaitNs);
-        __syncthreads();                                    // (S1) staging free
+        __syncthreads();                                    // (S1) this tile's input landed
 
         // ---- the thread's 8x8 block: v[i] = row 8br+i, columns 8bc .. 8bc+7
         const uint16_t *in = sm.in[buf];
@@ -290,6 +295,7 @@ __global__ void __launch_bounds__(kQThreads, 2)
             for (int i = 0; i < 8; ++i) m = __vmaxu2(m, max_abs4(v[i]));
             m = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
             if (lane == 0) sm.red[warp] = m;
+            if (tid == 0) bulk_wait_group_read0();  // staging free (see above)
         }
         if constexpr (KIND != kQuantTensor) __syncthreads();  // (S2) partials written
 
@@ -314,7 +320,8 @@ __global__ void __launch_bounds__(kQThreads, 2)
                 sm.col_mul[c] = mul_of(g);
                 sm.col_g[c] = static_cast<uint8_t>(g);
             }
-            __syncthreads();  // (S3) scales ready
+            if (tid == 0) bulk_wait_group_read0();  // staging free (see above)
+            __syncthreads();  // (S3) scales ready, staging free
         }
 
         float rmul[8], cmul[8];
