@@ -92,6 +92,7 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-bf16", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--no-paper-model", action="store_true", help="skip the C6 (paper's own model shape) line")
     return ap.parse_args()
 
 
@@ -356,9 +357,59 @@ def bf16_layer_speedup(P, torch, stack):
     t_fp8 = timeit(run_fp8)
     flops = sum(6.0 * M * N * K for _, N, K in stack.wl.linears)
     del bufs
+
+    # Wgrad into an FP32 main-grad (the paper's FP32 gradient accumulation)
+    # against the BF16-output Wgrad, same operands
+    mains = [torch.zeros((N, K), dtype=torch.float32, device=dev) for _, N, K in stack.wl.linears]
+
+    def run_wgrad_bf16():
+        for j in range(len(stack.wl.linears)):
+            P.puro_fp8_linear_wgrad(stack.dyq[j].colwise, stack.xqt[0][j], stack.dw[j], stack.workspace)
+
+    def run_wgrad_main():
+        for j in range(len(stack.wl.linears)):
+            P.puro_fp8_linear_wgrad_main_grad(stack.dyq[j].colwise, stack.xqt[0][j], mains[j], stack.workspace)
+
+    t_wb = timeit(run_wgrad_bf16)
+    t_wm = timeit(run_wgrad_main)
+    wflops = sum(2.0 * M * N * K for _, N, K in stack.wl.linears)
+    del mains
     torch.cuda.empty_cache()
     return {"layer": 0, "bf16_gemm_tflops": flops / t_bf16 / 1e12, "fp8_gemm_tflops": flops / t_fp8 / 1e12,
-            "fp8_over_bf16": t_bf16 / t_fp8, "paper_fp8_over_bf16_whole_model_rtx5090": 1.36}
+            "fp8_over_bf16": t_bf16 / t_fp8, "paper_fp8_over_bf16_whole_model_rtx5090": 1.36,
+            "wgrad_bf16_out_tflops": wflops / t_wb / 1e12, "wgrad_fp32_main_grad_tflops": wflops / t_wm / 1e12}
+
+
+def paper_model_measure(P, W, torch, device, scaling, steps=5, warmup=3):
+    """The same step on the paper's own production model shape: C6, the
+    28-layer Qwen3-1.7B linear stack at its training micro-batch (2 x 4096
+    tokens).  Device-resident inputs, CUDA events around the timed steps."""
+    wl = W.WORKLOADS["C6"]
+    stack = LinearStack(P, W, torch, wl, device, scaling, wl.layers, wl.M)
+    torch.cuda.synchronize()
+    for _ in range(warmup):
+        stack.step()
+    torch.cuda.synchronize()
+    stack.timer.pending.clear()
+    stack.timer.enabled = True
+    s = torch.cuda.Event(enable_timing=True)
+    e = torch.cuda.Event(enable_timing=True)
+    s.record()
+    for _ in range(steps):
+        stack.step()
+    e.record()
+    torch.cuda.synchronize()
+    stack.timer.enabled = False
+    step_s = s.elapsed_time(e) * 1e-3 / steps
+    per = stack.timer.totals()
+    g, q = per["gemm"], per["quantize"]
+    out = {"workload": f"{wl.key}: " + wl.description, "value": stack.flops_per_step() / step_s / 1e12,
+           "unit": "TFLOP/s", "ms_per_step": step_s * 1e3, "tokens_per_s": wl.M / step_s, "steps": steps,
+           "warmup": warmup, "gemm_only_tflops": g["units"] / g["time_s"] / 1e12,
+           "quantize_gbs": q["units"] / q["time_s"] / 1e9}
+    del stack
+    torch.cuda.empty_cache()
+    return out
 
 
 def e2e_measure(P, torch, stack, steps):
@@ -629,6 +680,10 @@ def main():
             result["e2e"]["value"] = job_value(world, flops, ms * 1e-3) / 1e12
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(torch, stack)
+    if rank == 0 and world == 1 and not args.no_paper_model and args.config == "C5":
+        del stack
+        torch.cuda.empty_cache()
+        result["paper_model_shape"] = paper_model_measure(P, W, torch, device, args.scaling)
     if rank == 0:
         print(json.dumps(result), flush=True)
     if world > 1:

@@ -175,6 +175,21 @@ puro_status_t puro_fp8_linear_wgrad(const puro_fp8_tensor_t *dy_t, const puro_fp
                                     int32_t *dev_status, void *stream);
 
 /*
+ * Wgrad accumulated into an FP32 main-grad:
+ *     main_grad[n, k] += sum_m sA(n, m) sB(k, m) qA[n, m] qB[k, m]
+ * (appendix "FP8 implementation pipeline": the weight gradient is
+ * accumulated in FP32 across micro-batches, the main-grad of the optimizer).
+ * Same operands, scaling rules and workspace as puro_fp8_linear_wgrad;
+ * main_grad is FP32 [N, K], row-major, 16-byte aligned, read and written.
+ * Each element receives exactly one FP32 addition per call (of the FP32
+ * product, or of the fixed-order sum of the split partials), so results are
+ * deterministic.  A zero reduction extent leaves main_grad unchanged.
+ */
+puro_status_t puro_fp8_linear_wgrad_main_grad(const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t,
+                                              float *main_grad, void *workspace, size_t workspace_bytes,
+                                              int32_t *dev_status, void *stream);
+
+/*
  * Wgrad without allocation and without caller-supplied scratch.
  *
  * The paper has no counterpart to this entry point; it serves callers that

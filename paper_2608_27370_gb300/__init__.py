@@ -70,6 +70,7 @@ _SIGNATURES = {
     "puro_fp8_linear_fprop": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_dgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_wgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
+    "puro_fp8_linear_wgrad_main_grad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_wgrad_noalloc": (_I32, [_P, _P, _P, _P, _P]),
     "puro_fp8_workspace_size": (ctypes.c_size_t, [_I64, _I64, _I64]),
     "puro_fp8_scale_bytes": (ctypes.c_size_t, [_I64, _I64]),
@@ -176,12 +177,13 @@ class FP8Operand:
                                  self.data.shape[0], self.data.shape[1], self.fmt, self.scaling, self.role, 0)
 
 
-def _gemm(name: str, a: FP8Operand, b: FP8Operand, out: torch.Tensor, workspace, dev_status, stream) -> None:
+def _gemm(name: str, a: FP8Operand, b: FP8Operand, out: torch.Tensor, workspace, dev_status, stream,
+          out_dtype=torch.bfloat16) -> None:
     ca, cb = a.as_c(), b.as_c()
     ws_ptr = _ptr(workspace, None, "workspace")
     ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
     fn = getattr(load_library(), name)
-    st = fn(ctypes.byref(ca), ctypes.byref(cb), _ptr(out, torch.bfloat16, "out"), ws_ptr, ws_bytes,
+    st = fn(ctypes.byref(ca), ctypes.byref(cb), _ptr(out, out_dtype, "out"), ws_ptr, ws_bytes,
             _ptr(dev_status, torch.int32, "dev_status"), _stream(stream))
     _check(name, st)
 
@@ -202,6 +204,14 @@ def puro_fp8_linear_wgrad(dy_t: FP8Operand, x_t: FP8Operand, dw: torch.Tensor, w
                           stream=None) -> None:
     """dW [N,K] = dY^T [N,M] . X [M,K] (operands dY^T [N,M], X^T [K,M])."""
     _gemm("puro_fp8_linear_wgrad", dy_t, x_t, dw, workspace, dev_status, stream)
+
+
+def puro_fp8_linear_wgrad_main_grad(dy_t: FP8Operand, x_t: FP8Operand, main_grad: torch.Tensor, workspace=None,
+                                    dev_status=None, stream=None) -> None:
+    """main_grad [N,K] (FP32) += dY^T [N,M] . X [M,K]: the weight gradient
+    accumulated in FP32 (operands dY^T [N,M], X^T [K,M])."""
+    _gemm("puro_fp8_linear_wgrad_main_grad", dy_t, x_t, main_grad, workspace, dev_status, stream,
+          out_dtype=torch.float32)
 
 
 def puro_fp8_linear_wgrad_noalloc(dy_t: FP8Operand, x_t: FP8Operand, dw: torch.Tensor, dev_status=None,

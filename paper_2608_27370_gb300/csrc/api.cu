@@ -91,8 +91,9 @@ puro_status_t check_operand(const puro_fp8_tensor_t *t) {
 }
 
 // D[M,N] = A[M,K] * B[N,K]^T over quantised operands.
+// accumulate_f32: d is an FP32 [M, N] main-grad that receives d += A * B^T.
 puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, void *d, void *workspace,
-                       size_t workspace_bytes, int32_t *dev_status, void *stream) {
+                       size_t workspace_bytes, int32_t *dev_status, void *stream, bool accumulate_f32 = false) {
     puro_status_t st = check_operand(a);
     if (st != PURO_OK) return st;
     st = check_operand(b);
@@ -102,7 +103,8 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
     const int64_t M = a->rows, N = b->rows, K = a->red;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (M == 0 || N == 0) return PURO_OK;
-    if (K == 0) return cuda_status(cudaMemsetAsync(d, 0, static_cast<size_t>(M * N) * 2, s));
+    if (K == 0)  // an empty reduction: the product is zero
+        return accumulate_f32 ? PURO_OK : cuda_status(cudaMemsetAsync(d, 0, static_cast<size_t>(M * N) * 2, s));
     const bool block = a->scaling == PURO_SCALE_BLOCK;
 
     // Split the reduction across CTA pairs when the output has too few tiles
@@ -112,14 +114,16 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
     const bool split = sp > 1 && workspace && aligned16(workspace) &&
                        workspace_bytes >= splitk_workspace_bytes(M, N, K, false);
     const int forced = g_tile_n.load();
-    const int tile_n = (block && !split) ? (forced ? forced : choose_tile_n(M, N, K)) : 256;
+    const int tile_n = (block && !split && !accumulate_f32) ? (forced ? forced : choose_tile_n(M, N, K)) : 256;
 
     GemmMaps m{};
     if (!make_map(&m.a, CU_TENSOR_MAP_DATA_TYPE_UINT8, a->data, K, M, K, kGemmBKBytes, kGemmBM,
                   CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_map(&m.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, b->data, K, N, K, kGemmBKBytes,
                   static_cast<uint32_t>(tile_n / 2), CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !(tile_n == 256
+        !(accumulate_f32
+              ? make_map(&m.d, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, d, N, M, N * 4, 32, 32, CU_TENSOR_MAP_SWIZZLE_128B)
+          : tile_n == 256
               ? make_map(&m.d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B)
               : make_map(&m.d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B)))
         return PURO_ERR_CUDA;
@@ -147,6 +151,7 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
     if (g.num_sms <= 0) return PURO_ERR_CUDA;
     g.out = d;
     g.splits = 1;
+    g.accumulate_f32 = accumulate_f32;
     if (split) {
         const uint64_t rows = static_cast<uint64_t>(sp) * static_cast<uint64_t>(splitk_rows_per_chunk(M));
         if (!make_map(&m.ws, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, workspace, N, rows, N * 4, 32, 32,
@@ -285,6 +290,12 @@ PURO_API puro_status_t puro_fp8_linear_wgrad(const puro_fp8_tensor_t *dy_t, cons
                                              void *workspace, size_t workspace_bytes, int32_t *dev_status,
                                              void *stream) {
     return fp8_gemm(dy_t, x_t, dw, workspace, workspace_bytes, dev_status, stream);
+}
+
+PURO_API puro_status_t puro_fp8_linear_wgrad_main_grad(const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t,
+                                                       float *main_grad, void *workspace, size_t workspace_bytes,
+                                                       int32_t *dev_status, void *stream) {
+    return fp8_gemm(dy_t, x_t, main_grad, workspace, workspace_bytes, dev_status, stream, true);
 }
 
 PURO_API size_t puro_fp8_workspace_size(int64_t rows_out, int64_t cols_out, int64_t red) {

@@ -175,15 +175,17 @@ PURO_DEV void pack_bf16x8(const uint32_t *src, float sab, uint32_t (&w)[4]) {
     }
 }
 
-// OUT_F32: write FP32 partial tiles of a split reduction to the workspace
-// [splits * Mp, N], Mp = num_m * 256 (rows split * Mp + m), instead of the
-// BF16 output; a ragged last pair tile then stays inside its chunk (BN = 256
-// only).  tm_d: D with box {64, 32} and the 128-byte swizzle (BN = 256) or
+// OUT: kGemmOutBF16 writes D in BF16; kGemmOutF32Partial writes FP32
+// partial tiles of a split reduction to the workspace [splits * Mp, N],
+// Mp = num_m * 256 (rows split * Mp + m), so that a ragged last pair tile
+// stays inside its chunk; kGemmOutF32Add adds the FP32 tile to D (an FP32
+// main-grad, one TMA reduce-add per element, so the result is deterministic).
+// The FP32 forms are BN = 256 only.  tm_d: D with box {64, 32} and the 128-byte swizzle (BN = 256) or
 // box {32, 32} and the 64-byte swizzle (BN = 224).
 // tm_sfa / tm_sfb (block kind only): the scale vectors of A / B viewed as
 // uint32 [chunks, 128] (one 512-byte chunk per row), box {128, 1}; tm_sfb is
 // read only with BN = 256.
-template <int KIND, bool OUT_F32, int BN>
+template <int KIND, int OUT, int BN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     gemm_tn_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
                    const __grid_constant__ CUtensorMap tm_d, const __grid_constant__ CUtensorMap tm_sfa,
@@ -202,6 +204,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     constexpr int kKSteps = kAtomBytes / 32;            // MMAs per atom (32 bytes of K each)
     constexpr uint32_t kStageBytes = (kBM + kBNHalf) * kBKBytes;  // one CTA's operand bytes per stage
     constexpr uint32_t kSfBytes = kHelper ? 512u : 512u + 1024u;  // one CTA's TMA scale bytes per group
+    constexpr bool OUT_F32 = (OUT != kGemmOutBF16);
     static_assert(BN == 256 || (BN == 224 && kMX && !OUT_F32), "the 224-wide form is block-scaled, BF16 out");
     static_assert(!kMX || kSfBase + kSfSets * kSfColsPerSet <= kTmemCols, "TMEM budget");
     static_assert(kAccShift + BN <= (kMX ? kSfBase : kTmemCols), "accumulators clear of the scale columns");
@@ -465,8 +468,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             const uint32_t t_row =
                 tmem + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>((local & 1) * kAccShift);
             if constexpr (OUT_F32) {
-                // FP32 partial tile: 8 chunks of 32 columns (128 bytes per row)
-                const int row0 = wu.split * p.num_m * kPairM + m0 + 32 * q;  // chunks pair-tile aligned
+                // FP32 tile: 8 chunks of 32 columns (128 bytes per row), stored
+                // as a split partial or added to D
+                const int row0 = (OUT == kGemmOutF32Partial ? wu.split * p.num_m * kPairM : 0) + m0 + 32 * q;
 #pragma unroll
                 for (int h = 0; h < BN / 128; ++h) {
                     uint32_t r[4][32];
@@ -494,7 +498,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         fence_proxy_async_smem();
                         __syncwarp();
                         if (lane == 0) {
-                            tma_store_2d(&tm_d, stage_buf, col, row0);
+                            if constexpr (OUT == kGemmOutF32Add)
+                                tma_reduce_add_2d(&tm_d, stage_buf, col, row0);
+                            else
+                                tma_store_2d(&tm_d, stage_buf, col, row0);
                             bulk_commit_group();
                         }
                     }
@@ -619,6 +626,30 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const float4 *__rest
     }
 }
 
+// The same sum added to an FP32 main-grad: out[i] += sum_s ws[s][i] (one
+// add per element, fixed order).
+__global__ void __launch_bounds__(256) splitk_reduce_add_f32_kernel(const float4 *__restrict__ ws, int splits,
+                                                                    int64_t n4, int64_t split_stride4,
+                                                                    float4 *__restrict__ out) {
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
+        float4 a = ws[i];
+        for (int sp = 1; sp < splits; ++sp) {
+            const float4 b = ws[sp * split_stride4 + i];
+            a.x += b.x;
+            a.y += b.y;
+            a.z += b.z;
+            a.w += b.w;
+        }
+        float4 o = out[i];
+        o.x += a.x;
+        o.y += a.y;
+        o.z += a.z;
+        o.w += a.w;
+        out[i] = o;
+    }
+}
+
 int choose_splits(int64_t M, int64_t N, int64_t K, bool bf16) {
     if (bf16) return 1;
     const int64_t tiles = ((M + kPairM - 1) / kPairM) * ((N + 255) / 256);
@@ -673,7 +704,7 @@ size_t splitk_workspace_bytes(int64_t M, int64_t N, int64_t K, bool bf16) {
 
 // Pairs that can be resident at once for this kernel (the persistent grid
 // size), cached per device and kernel.
-template <int KIND, bool OUT_F32, int BN>
+template <int KIND, int OUT, int BN>
 static int max_resident_pairs(int num_sms, size_t smem) {
     static int cache[64] = {0};
     int dev = 0;
@@ -691,7 +722,7 @@ static int max_resident_pairs(int num_sms, size_t smem) {
     cfg.attrs = &attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, gemm_tn_kernel<KIND, OUT_F32, BN>, &cfg) != cudaSuccess || n <= 0) {
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tn_kernel<KIND, OUT, BN>, &cfg) != cudaSuccess || n <= 0) {
         (void)cudaGetLastError();
         n = num_sms / 2;
     }
@@ -699,7 +730,7 @@ static int max_resident_pairs(int num_sms, size_t smem) {
     return n;
 }
 
-template <int KIND, bool OUT_F32, int BN>
+template <int KIND, int OUT, int BN>
 static cudaError_t launch_kind(const GemmArgs &g, const GemmMaps &m, int splits, cudaStream_t s) {
     constexpr int kElemBytes = (KIND == kGemmBF16) ? 2 : 1;
     constexpr int kBK = kBKBytes / kElemBytes;
@@ -729,38 +760,43 @@ static cudaError_t launch_kind(const GemmArgs &g, const GemmMaps &m, int splits,
     p.status = g.status;
     p.wait_ns = g.wait_timeout_ns;
 
-    auto kern = gemm_tn_kernel<KIND, OUT_F32, BN>;
+    auto kern = gemm_tn_kernel<KIND, OUT, BN>;
     const size_t smem = sizeof(GemmSmem<BN>) + 1024;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    const int pairs_max = max_resident_pairs<KIND, OUT_F32, BN>(g.num_sms, smem);
+    const int pairs_max = max_resident_pairs<KIND, OUT, BN>(g.num_sms, smem);
     const int pairs = p.num_units < pairs_max ? p.num_units : pairs_max;
-    kern<<<2 * pairs, kThreads, smem, s>>>(m.a, m.b, OUT_F32 ? m.ws : m.d, m.sfa, m.sfb, p);
+    kern<<<2 * pairs, kThreads, smem, s>>>(m.a, m.b, OUT == kGemmOutF32Partial ? m.ws : m.d, m.sfa, m.sfb, p);
     return cudaGetLastError();
 }
 
 template <int KIND>
 static cudaError_t launch_split_or_not(const GemmArgs &g, const GemmMaps &m, cudaStream_t s) {
     if (g.splits <= 1) {
+        if (g.accumulate_f32) return launch_kind<KIND, kGemmOutF32Add, 256>(g, m, 1, s);
         if constexpr (KIND == kGemmFP8Block)
-            if (g.tile_n == 224) return launch_kind<KIND, false, 224>(g, m, 1, s);
-        return launch_kind<KIND, false, 256>(g, m, 1, s);
+            if (g.tile_n == 224) return launch_kind<KIND, kGemmOutBF16, 224>(g, m, 1, s);
+        return launch_kind<KIND, kGemmOutBF16, 256>(g, m, 1, s);
     }
-    cudaError_t e = launch_kind<KIND, true, 256>(g, m, g.splits, s);
+    cudaError_t e = launch_kind<KIND, kGemmOutF32Partial, 256>(g, m, g.splits, s);
     if (e != cudaSuccess) return e;
     const int64_t n4 = g.M * g.N / 4;
     const int64_t stride4 = splitk_rows_per_chunk(g.M) * g.N / 4;
     int64_t want = (n4 + 255) / 256;
     const int64_t cap = static_cast<int64_t>(g.num_sms) * 8;
     const int grid = static_cast<int>(want < cap ? want : cap);
-    splitk_reduce_kernel<<<grid, 256, 0, s>>>(reinterpret_cast<const float4 *>(g.workspace), g.splits, n4, stride4,
-                                              reinterpret_cast<uint2 *>(g.out));
+    if (g.accumulate_f32)
+        splitk_reduce_add_f32_kernel<<<grid, 256, 0, s>>>(reinterpret_cast<const float4 *>(g.workspace), g.splits, n4,
+                                                          stride4, reinterpret_cast<float4 *>(g.out));
+    else
+        splitk_reduce_kernel<<<grid, 256, 0, s>>>(reinterpret_cast<const float4 *>(g.workspace), g.splits, n4, stride4,
+                                                  reinterpret_cast<uint2 *>(g.out));
     return cudaGetLastError();
 }
 
 cudaError_t launch_gemm(const GemmArgs &g, const GemmMaps &m, cudaStream_t s) {
     switch (g.kind) {
-        case kGemmBF16: return launch_kind<kGemmBF16, false, 256>(g, m, 1, s);
+        case kGemmBF16: return launch_kind<kGemmBF16, kGemmOutBF16, 256>(g, m, 1, s);
         case kGemmFP8Tensor: return launch_split_or_not<kGemmFP8Tensor>(g, m, s);
         default: return launch_split_or_not<kGemmFP8Block>(g, m, s);
     }

@@ -49,6 +49,13 @@ enum GemmKind : int {
     kGemmFP8Block = 2,   // kind::mxf8f6f4 with E8M0 group scales
 };
 
+// Output forms of the GEMM kernel.
+enum GemmOut : int {
+    kGemmOutBF16 = 0,        // D in BF16
+    kGemmOutF32Partial = 1,  // FP32 partial tiles of a split reduction (workspace)
+    kGemmOutF32Add = 2,      // D (FP32) += the product (main-grad accumulation)
+};
+
 struct GemmArgs {
     GemmKind kind;
     int a_fmt, b_fmt;            // FP8 formats (0 = E4M3, 1 = E5M2)
@@ -67,13 +74,17 @@ struct GemmArgs {
     int splits;
     void *workspace;
     void *out;
+    // out is an FP32 main-grad [M, N] that receives out += A * B^T (block
+    // or per-tensor kinds; 256-wide tiles)
+    bool accumulate_f32;
 };
 
 // Tensor maps of one GEMM launch.
 //   a:   A [M, K] (128-byte swizzle, box {128 bytes, 128 rows})
 //   b:   B [N, K] (box {128 bytes, tile_n / 2 rows}: half of a tile per CTA)
 //   d:   D [M, N] bf16 (tile_n 256: 128-byte swizzle, box {64, 32};
-//        tile_n 224: 64-byte swizzle, box {32, 32})
+//        tile_n 224: 64-byte swizzle, box {32, 32}); with accumulate_f32, the
+//        FP32 main-grad [M, N] (128-byte swizzle, box {32, 32})
 //   ws:  workspace [splits * splitk_rows_per_chunk(M), N] fp32 (128-byte
 //        swizzle, box {32, 32}); only read when g.splits > 1
 //   sfa, sfb (kGemmFP8Block only): the scale vectors of A / B,

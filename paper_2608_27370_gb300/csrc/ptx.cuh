@@ -96,6 +96,16 @@ PURO_DEV void tma_store_2d(const CUtensorMap *map, const void *src, int32_t x, i
                  : "memory");
 }
 
+// 2-D tiled element-wise add shared -> global (bulk-group completion): each
+// element of the box is added to the global tensor's element (the tensor
+// map's type; f32 adds round to nearest).
+PURO_DEV void tma_reduce_add_2d(const CUtensorMap *map, const void *src, int32_t x, int32_t y) {
+    asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(smem_u32(src)), "r"(x), "r"(y)
+                 : "memory");
+}
+
 // Contiguous bulk copy global -> shared; both addresses 16-byte aligned,
 // bytes a multiple of 16.
 PURO_DEV void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {

@@ -1,8 +1,9 @@
-"""GPU parity at the full sizes of the five benchmark workloads, in the
-launch configuration the benchmark times.
+"""GPU parity at the full sizes of the benchmark workloads, in the launch
+configuration the benchmark times.
 
 C1 (one linear, M=256) is compared element by element in both scaling
-modes.  C2-C5 use the paper's blockwise recipe and are compared on sampled
+modes.  C2-C6 (C6: the paper's own Qwen3-1.7B-shaped model) use the
+paper's blockwise recipe and are compared on sampled
 outputs the oracle computes one by one: every quantised byte and scale on
 sampled rows and columns, and every GEMM output on the cross product of
 sampled rows and columns (which contains the four corner 128x128 tiles).
@@ -74,3 +75,10 @@ def test_c4_decoder_layer(idx):
 @pytest.mark.parametrize("idx", [0, 1, 2, 3])
 def test_c5_layers(layer, idx):
     _sampled("C5", layer, idx, 500 + 4 * layer + idx)
+
+
+@pytest.mark.parametrize("layer", [0, 27])
+@pytest.mark.parametrize("idx", [0, 1, 2, 3])
+def test_c6_paper_model_layers(layer, idx):
+    """The paper's own model shape (Qwen3-1.7B linears, M = 8192)."""
+    _sampled("C6", layer, idx, 600 + 4 * layer + idx)

@@ -152,3 +152,53 @@ def test_wgrad_split_reduction(scaling, M, N, K):
     P.puro_fp8_linear_wgrad(dyq.colwise, xq.colwise, dw_small, workspace=ws[: ws_bytes // 2])
     torch.cuda.synchronize()
     assert torch.equal(dw_small.view(torch.int16), dw_plain.view(torch.int16))
+
+
+@pytest.mark.parametrize("M,N,K,split", [(512, 384, 640, False), (640, 1152, 2560, False), (8192, 256, 256, True),
+                                         (4096, 384, 1536, True)])
+def test_wgrad_main_grad_accumulates_in_fp32(M, N, K, split):
+    """main_grad += dY^T X, twice from the same FP32 start: the result is the
+    start plus twice the oracle's product (within the GEMM tolerance), it is
+    deterministic, and the split schedule (with a workspace) agrees."""
+    x, w, dy = _inputs(M, N, K, 5000 + M + N + K, t3=True)
+    xq = P.quantize(x, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT)
+    dyq = P.quantize(dy, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT)
+    ws = None
+    if split:
+        ws_bytes = P.puro_fp8_workspace_size(N, K, M)
+        assert ws_bytes > 0, "this shape should take the split schedule"
+        ws = torch.full((ws_bytes,), 0xFF, dtype=torch.uint8, device=DEV)
+    main0 = W.normal_f32((N, K), 0.05, DEV, 6000 + M)
+    runs = []
+    for _ in range(2):
+        main = main0.clone()
+        P.puro_fp8_linear_wgrad_main_grad(dyq.colwise, xq.colwise, main, workspace=ws)
+        P.puro_fp8_linear_wgrad_main_grad(dyq.colwise, xq.colwise, main, workspace=ws)
+        runs.append(main)
+    torch.cuda.synchronize()
+    assert torch.equal(runs[0], runs[1]), "main-grad accumulation is not deterministic"
+    dw_ref = oracle_linear(x, w, dy, P.SCALE_BLOCK)["dw"]
+    start = main0.double().cpu().numpy()
+    got = runs[0].double().cpu().numpy()
+    ok, ratio = O.within_tolerance(got - start, 2.0 * dw_ref)
+    assert ok, f"main-grad increment outside tolerance (worst ratio {ratio:.3g})"
+    # and the FP32 sum keeps far more than BF16's precision: typical error
+    # well below a BF16 ulp of the increment
+    rel = np.abs((got - start) - 2.0 * dw_ref) / np.maximum(np.abs(2.0 * dw_ref), 1e-30)
+    assert float(np.median(rel)) < 2.0 ** -12, f"median relative error {float(np.median(rel)):.3g}"
+
+
+def test_wgrad_main_grad_zero_reduction_leaves_it_unchanged():
+    import ctypes
+    lib = P.load_library()
+    stream = torch.cuda.current_stream().cuda_stream
+    buf = torch.zeros(4096, dtype=torch.uint8, device=DEV)
+    p = buf.data_ptr()
+    a = P.puro_fp8_tensor_t(p, p, 256, 0, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT, 0)
+    b = P.puro_fp8_tensor_t(p, p, 384, 0, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT, 0)
+    main = W.normal_f32((256, 384), 1.0, DEV, 77)
+    before = main.clone()
+    assert lib.puro_fp8_linear_wgrad_main_grad(ctypes.byref(a), ctypes.byref(b), main.data_ptr(), None, 0, None,
+                                               stream) == 0
+    torch.cuda.synchronize()
+    assert torch.equal(main, before)
