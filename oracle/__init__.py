@@ -76,6 +76,8 @@ def _load():
         "oracle_fp8_encode_array": (None, [P, I64, I, P]),
         "oracle_bf16_from_double_array": (None, [P, I64, P]),
         "oracle_e8m0_from_amax_array": (None, [P, I64, I, P]),
+        "oracle_rmsnorm_rstd": (None, [P, I64, I64, ctypes.c_double, P]),
+        "oracle_rmsnorm_apply_f32": (None, [P, I64, I64, P, P, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -291,6 +293,27 @@ def linear_tensor(x, w, dy, fmt_x: int = E4M3, fmt_w: int = E4M3, fmt_g: int = E
         y=gemm_tn(X, W, nthreads), dx=gemm_tn(dY, np.ascontiguousarray(W.T), nthreads),
         dw=gemm_tn(np.ascontiguousarray(dY.T), np.ascontiguousarray(X.T), nthreads),
     )
+
+
+def rmsnorm_rstd(h, eps: float) -> np.ndarray:
+    """Per-row 1/sqrt(mean(h^2) + eps) of a bf16 [rows, cols] matrix, fp64."""
+    hb = np.ascontiguousarray(_bits(h))
+    rows, cols = hb.shape
+    out = np.empty(rows, np.float64)
+    _load().oracle_rmsnorm_rstd(_p(hb), rows, cols, ctypes.c_double(eps), _p(out))
+    return out
+
+
+def rmsnorm_apply_f32(h, rstd_f32, gamma=None) -> np.ndarray:
+    """bf16 bits of (h * rstd) * gamma in fp32 (gamma None: no gain)."""
+    hb = np.ascontiguousarray(_bits(h))
+    rows, cols = hb.shape
+    r = np.ascontiguousarray(np.asarray(rstd_f32, np.float32))
+    assert r.shape == (rows,)
+    g = None if gamma is None else np.ascontiguousarray(_bits(gamma))
+    out = np.empty((rows, cols), np.uint16)
+    _load().oracle_rmsnorm_apply_f32(_p(hb), rows, cols, _p(r), None if g is None else _p(g), _p(out))
+    return out
 
 
 def within_tolerance(gpu, ref):

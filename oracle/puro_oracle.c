@@ -28,6 +28,10 @@
  *   - Per-tensor current scaling (the contrast drawn in the same section:
  *     "one scale for an entire tensor"): scale = fp32(fmt_max / amax),
  *     codes = RNE_sat(fp32(x * scale)), scale_inv = fp32(1 / scale).
+ *   - RMSNorm ahead of the quantiser (the model's normalisation before the
+ *     attention and MLP projections, section "Model architecture and
+ *     pretraining system": the Qwen3 architecture): rstd = 1/sqrt(mean h^2
+ *     + eps) per row, y = bf16((h * rstd) * gamma).
  *
  * Build: gcc -std=c11 -O2 -ffp-contract=off -fPIC -shared -pthread.
  * No fast-math: every float/double operation below is an IEEE operation in
@@ -435,4 +439,41 @@ void oracle_bf16_from_double_array(const double *v, int64_t n, uint16_t *out)
 void oracle_e8m0_from_amax_array(const uint16_t *amax_bits, int64_t n, int fmt, uint8_t *out)
 {
     for (int64_t i = 0; i < n; ++i) out[i] = oracle_e8m0_from_amax(amax_bits[i], fmt);
+}
+
+/* ---------------------------------------------------------------------- */
+/* RMSNorm producer                                                        */
+/* ---------------------------------------------------------------------- */
+/*
+ * Per-row reciprocal RMS of h [rows, cols] (bf16): rstd[r] = 1 /
+ * sqrt(sum_k h[r,k]^2 / cols + eps), in fp64 (each square is exact in fp64;
+ * the sum is taken in k order).
+ */
+void oracle_rmsnorm_rstd(const uint16_t *h, int64_t rows, int64_t cols, double eps, double *rstd)
+{
+    for (int64_t r = 0; r < rows; ++r) {
+        double ss = 0.0;
+        for (int64_t k = 0; k < cols; ++k) {
+            const double v = bf16_to_double(h[r * cols + k]);
+            ss += v * v;
+        }
+        rstd[r] = 1.0 / sqrt(ss / (double)cols + eps);
+    }
+}
+
+/*
+ * The normalised activation the quantiser receives, given an fp32 rstd per
+ * row: y[r,k] = bf16_rne(fp32(fp32(h[r,k] * rstd[r]) * gamma[k])), the two
+ * products in fp32 round-to-nearest in that order; gamma NULL means no gain
+ * (the second product is skipped).
+ */
+void oracle_rmsnorm_apply_f32(const uint16_t *h, int64_t rows, int64_t cols, const float *rstd,
+                              const uint16_t *gamma, uint16_t *y)
+{
+    for (int64_t r = 0; r < rows; ++r)
+        for (int64_t k = 0; k < cols; ++k) {
+            float p = bf16_to_float(h[r * cols + k]) * rstd[r];
+            if (gamma) p = p * bf16_to_float(gamma[k]);
+            y[r * cols + k] = oracle_bf16_from_double((double)p);
+        }
 }
