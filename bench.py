@@ -380,6 +380,55 @@ def bf16_layer_speedup(P, torch, stack):
             "wgrad_bf16_out_tflops": wflops / t_wb / 1e12, "wgrad_fp32_main_grad_tflops": wflops / t_wm / 1e12}
 
 
+def rmsnorm_fusion_measure(P, W, torch, device):
+    """RMSNorm fused ahead of the activation quantiser against RMSNorm (bf16
+    y written and read back) followed by the quantiser, on the inputs of the
+    qkv / gate_up projections of C5 ([32768, 1536]) and C6 ([8192, 2048])."""
+
+    def timeit(fn, reps=20):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        s = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        s.record()
+        for _ in range(reps):
+            fn()
+        e.record()
+        torch.cuda.synchronize()
+        return s.elapsed_time(e) * 1e-3 / reps
+
+    out = []
+    for key, (M, K) in (("C5", (32768, 1536)), ("C6", (8192, 2048))):
+        hs = [W.normal_bf16((M, K), 1.0, device, 31 + i) for i in range(2)]  # alternate: no L2 reuse across calls
+        gamma = W.normal_bf16((K,), 0.1, device, 33).add_(1.0)
+        rstd = torch.empty(M, dtype=torch.float32, device=device)
+        y = torch.empty((M, K), dtype=torch.bfloat16, device=device)
+        q = P.quantize(hs[0])
+        it = [0]
+
+        def fused():
+            it[0] ^= 1
+            P.puro_fp8_quantize_rmsnorm(hs[it[0]], gamma, 1e-6, P.E4M3, rstd, None, q.rowwise.data, q.rowwise.scale,
+                                        q.colwise.data, q.colwise.scale)
+
+        def unfused():
+            it[0] ^= 1
+            P.puro_rmsnorm_bf16(hs[it[0]], gamma, 1e-6, rstd, y)
+            P.quantize(y, out=q)
+
+        tf, tu = timeit(fused), timeit(unfused)
+        n = M * K
+        # algorithmic bytes of the fused op: read h, write both FP8 copies,
+        # their scales and rstd
+        fused_bytes = 2 * n + 2 * n + 2 * n // 128 + 4 * M
+        out.append({"input": f"{key} qkv/gate_up input [{M}, {K}]", "fused_us": tf * 1e6, "unfused_us": tu * 1e6,
+                    "fused_over_unfused_time": tf / tu, "fused_algorithmic_gbs": fused_bytes / tf / 1e9})
+        del hs, y, q
+        torch.cuda.empty_cache()
+    return out
+
+
 def paper_model_measure(P, W, torch, device, scaling, steps=5, warmup=3):
     """The same step on the paper's own production model shape: C6, the
     28-layer Qwen3-1.7B linear stack at its training micro-batch (2 x 4096
@@ -684,6 +733,7 @@ def main():
         del stack
         torch.cuda.empty_cache()
         result["paper_model_shape"] = paper_model_measure(P, W, torch, device, args.scaling)
+        result["rmsnorm_quantize_fusion"] = rmsnorm_fusion_measure(P, W, torch, device)
     if rank == 0:
         print(json.dumps(result), flush=True)
     if world > 1:

@@ -138,6 +138,39 @@ puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t cols,
                                 void *stream);
 
 /*
+ * RMSNorm fused ahead of the blockwise activation quantiser.
+ *
+ * The model normalises the hidden states with RMSNorm before the attention
+ * and MLP projections (section "Model architecture and pretraining system":
+ * the Qwen3 architecture); this entry point takes the pre-norm rows h and
+ * emits the FP8 operands of the projection directly:
+ *     rstd[r] = 1 / sqrt(mean_k h[r,k]^2 + eps)     (fp32, written)
+ *     y[r,k]  = bf16((h[r,k] * rstd[r]) * gamma[k])  (fp32 products)
+ * and then quantises y exactly as puro_fp8_quantize does with
+ * PURO_SCALE_BLOCK / PURO_ROLE_ACT (1x128 groups, optional transposed copy).
+ *   h: bf16 [rows, cols]; rows and cols multiples of 128; 16-byte aligned.
+ *   gamma: bf16 [cols] gain, or NULL for none.
+ *   eps >= 0.
+ *   rstd: fp32 [rows], written (kept for the RMSNorm backward).
+ *   y: bf16 [rows, cols], or NULL: y itself is written only when asked.
+ *   q, scale, q_t, scale_t: as in puro_fp8_quantize.
+ * rstd is an fp32 sum of squares in a fixed order, so it agrees with an
+ * exact computation to within a few fp32 ulps; y and every code and scale
+ * are then exactly determined by rstd.  Two kernels on `stream`; h is read
+ * twice (the second time largely from L2).
+ */
+puro_status_t puro_fp8_quantize_rmsnorm(const void *h, int64_t rows, int64_t cols, const void *gamma, float eps,
+                                        int32_t fmt, float *rstd, void *y, uint8_t *q, void *scale, uint8_t *q_t,
+                                        void *scale_t, void *stream);
+
+/*
+ * The same RMSNorm without the quantiser: rstd and y (bf16) as above, cols
+ * a multiple of 8.  The unfused comparison for the fused entry point.
+ */
+puro_status_t puro_rmsnorm_bf16(const void *h, int64_t rows, int64_t cols, const void *gamma, float eps,
+                                float *rstd, void *y, void *stream);
+
+/*
  * The three FP8 GEMMs of a linear layer with weight W [N, K], input X [M, K]
  * and output gradient dY [M, N] (appendix "FP8 implementation pipeline":
  * Fprop, Dgrad and Wgrad all use blockwise E4M3 operands).  Each computes

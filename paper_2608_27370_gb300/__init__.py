@@ -67,6 +67,8 @@ _I32 = ctypes.c_int32
 _SIGNATURES = {
     "puro_fp8_amax": (_I32, [_P, _I64, _I64, _P, _P]),
     "puro_fp8_quantize": (_I32, [_P, _I64, _I64, _I32, _I32, _I32, _P, _P, _P, _P, _P, _P]),
+    "puro_fp8_quantize_rmsnorm": (_I32, [_P, _I64, _I64, _P, ctypes.c_float, _I32, _P, _P, _P, _P, _P, _P, _P]),
+    "puro_rmsnorm_bf16": (_I32, [_P, _I64, _I64, _P, ctypes.c_float, _P, _P, _P]),
     "puro_fp8_linear_fprop": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_dgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_wgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
@@ -153,6 +155,33 @@ def puro_fp8_quantize(x: torch.Tensor, fmt: int, scaling: int, role: int, amax_b
         _ptr(amax_bits, (torch.int32, torch.uint32), "amax_bits"), _ptr(q, u8, "q"), _ptr(scale, sdt, "scale"),
         _ptr(q_t, u8, "q_t"), _ptr(scale_t, sdt, "scale_t"), _stream(stream))
     _check("puro_fp8_quantize", st)
+
+
+def puro_fp8_quantize_rmsnorm(h: torch.Tensor, gamma: Optional[torch.Tensor], eps: float, fmt: int,
+                              rstd: torch.Tensor, y: Optional[torch.Tensor], q: torch.Tensor, scale: torch.Tensor,
+                              q_t: Optional[torch.Tensor] = None, scale_t: Optional[torch.Tensor] = None,
+                              stream=None) -> None:
+    """RMSNorm of the rows of h (bf16, optional bf16 gain) fused ahead of the
+    blockwise activation quantiser: writes rstd (fp32 [rows]), optionally y
+    (bf16), and the codes and scales as puro_fp8_quantize does."""
+    rows, cols = h.shape
+    u8 = torch.uint8
+    st = load_library().puro_fp8_quantize_rmsnorm(
+        _ptr(h, torch.bfloat16, "h"), rows, cols, _ptr(gamma, torch.bfloat16, "gamma"), float(eps), fmt,
+        _ptr(rstd, torch.float32, "rstd"), _ptr(y, torch.bfloat16, "y"), _ptr(q, u8, "q"), _ptr(scale, u8, "scale"),
+        _ptr(q_t, u8, "q_t"), _ptr(scale_t, u8, "scale_t"), _stream(stream))
+    _check("puro_fp8_quantize_rmsnorm", st)
+
+
+def puro_rmsnorm_bf16(h: torch.Tensor, gamma: Optional[torch.Tensor], eps: float, rstd: torch.Tensor,
+                      y: torch.Tensor, stream=None) -> None:
+    """The same RMSNorm without the quantiser (rstd fp32, y bf16)."""
+    rows, cols = h.shape
+    st = load_library().puro_rmsnorm_bf16(_ptr(h, torch.bfloat16, "h"), rows, cols,
+                                          _ptr(gamma, torch.bfloat16, "gamma"), float(eps),
+                                          _ptr(rstd, torch.float32, "rstd"), _ptr(y, torch.bfloat16, "y"),
+                                          _stream(stream))
+    _check("puro_rmsnorm_bf16", st)
 
 
 @dataclass

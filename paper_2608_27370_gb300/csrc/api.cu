@@ -274,6 +274,64 @@ PURO_API puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t co
     return cuda_status(launch_quantize(a, tm_x, tm_q, tm_qt, static_cast<cudaStream_t>(stream)));
 }
 
+// RMSNorm (rows of h, optional bf16 gain) fused ahead of the blockwise
+// activation quantiser; see the header.
+PURO_API puro_status_t puro_fp8_quantize_rmsnorm(const void *h, int64_t rows, int64_t cols, const void *gamma,
+                                                 float eps, int32_t fmt, float *rstd, void *y, uint8_t *q, void *scale,
+                                                 uint8_t *q_t, void *scale_t, void *stream) {
+    if (!valid_fmt(fmt) || rows < 0 || cols < 0 || !(eps >= 0.0f)) return PURO_ERR_INVALID_ARG;
+    if (rows % 128 || cols % 128) return PURO_ERR_INVALID_ARG;
+    if ((q_t == nullptr) != (scale_t == nullptr)) return PURO_ERR_INVALID_ARG;
+    if (rows > INT32_MAX || cols > INT32_MAX) return PURO_ERR_UNSUPPORTED;
+    if (rows == 0 || cols == 0) return PURO_OK;
+    if (!h || !rstd || !q || !scale) return PURO_ERR_INVALID_ARG;
+    if (!aligned16(h) || !aligned16(gamma) || !aligned16(y) || !aligned16(q) || !aligned16(scale) ||
+        !aligned16(q_t) || !aligned16(scale_t) || (reinterpret_cast<uintptr_t>(rstd) & 3u))
+        return PURO_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    QuantArgs a{};
+    a.fmt = fmt;
+    a.rows = rows;
+    a.cols = cols;
+    a.has_t = q_t != nullptr;
+    a.kind = kQuantBlockAct;
+    a.scale_u8 = static_cast<uint8_t *>(scale);
+    a.scale_t_u8 = static_cast<uint8_t *>(scale_t);
+    a.x = static_cast<const uint16_t *>(h);
+    CUtensorMap tm_x, tm_q, tm_qt, tm_y;
+    if (!make_map(&tm_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h, cols, rows, cols * 2, 128, 128,
+                  CU_TENSOR_MAP_SWIZZLE_NONE) ||
+        !make_map(&tm_q, CU_TENSOR_MAP_DATA_TYPE_UINT8, q, cols, rows, cols, 128, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
+        return PURO_ERR_CUDA;
+    tm_qt = tm_q;
+    if (a.has_t && !make_map(&tm_qt, CU_TENSOR_MAP_DATA_TYPE_UINT8, q_t, rows, cols, rows, 128, 128,
+                             CU_TENSOR_MAP_SWIZZLE_128B))
+        return PURO_ERR_CUDA;
+    tm_y = tm_x;
+    if (y && !make_map(&tm_y, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, y, cols, rows, cols * 2, 128, 128,
+                       CU_TENSOR_MAP_SWIZZLE_NONE))
+        return PURO_ERR_CUDA;
+    cudaError_t e = launch_rmsnorm_rstd(static_cast<const uint16_t *>(h), rows, cols, eps, rstd, s);
+    if (e != cudaSuccess) return cuda_status(e);
+    ProdArgs prod{rstd, static_cast<const uint16_t *>(gamma), y != nullptr};
+    return cuda_status(launch_quantize_rmsnorm(a, tm_x, tm_q, tm_qt, tm_y, prod, s));
+}
+
+// The same RMSNorm without the quantiser (the unfused comparison).
+PURO_API puro_status_t puro_rmsnorm_bf16(const void *h, int64_t rows, int64_t cols, const void *gamma, float eps,
+                                         float *rstd, void *y, void *stream) {
+    if (rows < 0 || cols < 0 || cols % 8 || !(eps >= 0.0f)) return PURO_ERR_INVALID_ARG;
+    if (rows == 0 || cols == 0) return PURO_OK;
+    if (!h || !rstd || !y || !aligned16(h) || !aligned16(gamma) || !aligned16(y) ||
+        (reinterpret_cast<uintptr_t>(rstd) & 3u))
+        return PURO_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = launch_rmsnorm_rstd(static_cast<const uint16_t *>(h), rows, cols, eps, rstd, s);
+    if (e != cudaSuccess) return cuda_status(e);
+    return cuda_status(launch_rmsnorm_apply(static_cast<const uint16_t *>(h), rows, cols, rstd,
+                                            static_cast<const uint16_t *>(gamma), static_cast<uint16_t *>(y), s));
+}
+
 PURO_API puro_status_t puro_fp8_linear_fprop(const puro_fp8_tensor_t *x, const puro_fp8_tensor_t *w, void *y,
                                              void *workspace, size_t workspace_bytes, int32_t *dev_status,
                                              void *stream) {

@@ -33,11 +33,35 @@ struct QuantArgs {
 
 cudaError_t launch_amax(const uint16_t *x, int64_t n, uint32_t *amax, cudaStream_t s);
 
+// Producers fused ahead of the activation quantiser.
+enum QuantProd : int {
+    kProdNone = 0,
+    kProdRmsNorm = 1,  // y = bf16((h * rstd[row]) * gamma[col])
+};
+struct ProdArgs {
+    const float *rstd;      // kProdRmsNorm: [rows]
+    const uint16_t *gamma;  // kProdRmsNorm: bf16 [cols], or null (no gain)
+    bool write_y;           // also store y (through tm_y)
+};
+
+// rstd[r] = 1 / sqrt(mean(h[r,:]^2) + eps) (cols a multiple of 8).
+cudaError_t launch_rmsnorm_rstd(const uint16_t *h, int64_t rows, int64_t cols, float eps, float *rstd, cudaStream_t s);
+// y = bf16((h * rstd) * gamma), the unfused application.
+cudaError_t launch_rmsnorm_apply(const uint16_t *h, int64_t rows, int64_t cols, const float *rstd,
+                                 const uint16_t *gamma, uint16_t *y, cudaStream_t s);
+
 // tm_x: bf16 [rows, cols], box {128, 128}, no swizzle.
 // tm_q: u8 [rows, cols], box {128, 128}, no swizzle.
 // tm_qt: u8 [cols, rows], box {128, 128}, 128-byte swizzle (only if has_t).
 cudaError_t launch_quantize(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
                             const CUtensorMap &tm_qt, cudaStream_t s);
+
+// The activation quantiser fed by RMSNorm (a.kind must be kQuantBlockAct):
+// tm_x maps h; tm_y (bf16 [rows, cols], box {128, 128}, no swizzle) is
+// written only when prod.write_y.
+cudaError_t launch_quantize_rmsnorm(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
+                                    const CUtensorMap &tm_qt, const CUtensorMap &tm_y, const ProdArgs &prod,
+                                    cudaStream_t s);
 
 // Writes only the per-tensor scale_inv (used for empty tensors).
 cudaError_t launch_tensor_scale_only(const QuantArgs &a, cudaStream_t s);

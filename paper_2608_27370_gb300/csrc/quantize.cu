@@ -171,6 +171,124 @@ PURO_DEV void store_scale_vec(uint8_t *__restrict__ base, int64_t row, int64_t k
         for (int pb = b + 1; pb < 4; ++pb) chunk[pb] = 127;
 }
 
+// ------------------------------------------------------ RMSNorm producer
+// RMSNorm of the activation the quantiser receives (the model's
+// normalisation ahead of the attention and MLP projections): per row
+// rstd = 1 / sqrt(mean(h^2) + eps), then y = bf16((h * rstd) * gamma).
+
+// rstd of each row of h [rows, cols] (cols a multiple of 8), one warp per
+// row: fp32 sums of squares in a fixed order (lane-strided 8-value chunks,
+// then a butterfly), then an IEEE division and square root.
+__global__ void __launch_bounds__(256) rmsnorm_rstd_kernel(const uint16_t *__restrict__ h, int64_t rows, int64_t cols,
+                                                           float eps, float *__restrict__ rstd) {
+    const int lane = threadIdx.x & 31;
+    const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
+    for (int64_t r = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5); r < rows; r += nwarps) {
+        const uint4 *row = reinterpret_cast<const uint4 *>(h + r * cols);
+        float a = 0.0f, b = 0.0f;
+        for (int64_t c = lane; c < cols / 8; c += 32) {
+            const uint4 w = __ldg(row + c);
+            const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const float lo = __uint_as_float(ws[j] << 16), hi = __uint_as_float(ws[j] & 0xFFFF0000u);
+                a = __fmaf_rn(lo, lo, a);
+                b = __fmaf_rn(hi, hi, b);
+            }
+        }
+        float ss = a + b;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
+        if (lane == 0) rstd[r] = __fdiv_rn(1.0f, __fsqrt_rn(__fdiv_rn(ss, static_cast<float>(cols)) + eps));
+    }
+}
+
+// y = bf16((h * rstd) * gamma) for an 8-value chunk (gm unused without gamma).
+PURO_DEV uint4 rmsnorm_chunk(uint4 w, float rs, const float (&gm)[8], bool has_gamma) {
+    uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        float lo = __fmul_rn(__uint_as_float(ws[j] << 16), rs), hi = __fmul_rn(__uint_as_float(ws[j] & 0xFFFF0000u), rs);
+        if (has_gamma) {
+            lo = __fmul_rn(lo, gm[2 * j]);
+            hi = __fmul_rn(hi, gm[2 * j + 1]);
+        }
+        __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+        ws[j] = *reinterpret_cast<uint32_t *>(&v);
+    }
+    return make_uint4(ws[0], ws[1], ws[2], ws[3]);
+}
+
+PURO_DEV void load_gamma8(const uint16_t *gamma, int64_t c, int64_t cols, float (&gm)[8]) {
+    if (c + 8 <= cols) {
+        const uint4 g = __ldg(reinterpret_cast<const uint4 *>(gamma + c));
+        const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            gm[2 * j] = __uint_as_float(gw[j] << 16);
+            gm[2 * j + 1] = __uint_as_float(gw[j] & 0xFFFF0000u);
+        }
+    } else {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) gm[j] = 0.0f;  // columns past the end hold zeros
+    }
+}
+
+// Unfused comparison: y = bf16((h * rstd) * gamma), one 8-value chunk per
+// thread and step.
+__global__ void __launch_bounds__(256) rmsnorm_apply_kernel(const uint16_t *__restrict__ h, int64_t rows, int64_t cols,
+                                                            const float *__restrict__ rstd,
+                                                            const uint16_t *__restrict__ gamma, uint16_t *__restrict__ y) {
+    const int64_t per_row = cols / 8;
+    const int64_t chunks = rows * per_row;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < chunks; i += stride) {
+        const int64_t r = i / per_row, c = (i - r * per_row) * 8;
+        float gm[8];
+        if (gamma) load_gamma8(gamma, c, cols, gm);
+        reinterpret_cast<uint4 *>(y)[i] =
+            rmsnorm_chunk(__ldg(reinterpret_cast<const uint4 *>(h) + i), __ldg(rstd + r), gm, gamma != nullptr);
+    }
+}
+
+static int sm_count_here() {
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    return sms;
+}
+
+cudaError_t launch_rmsnorm_rstd(const uint16_t *h, int64_t rows, int64_t cols, float eps, float *rstd, cudaStream_t s) {
+    const int sms = sm_count_here();
+    const int64_t want = (rows + 7) / 8;
+    const int grid = static_cast<int>(want < 8 * sms ? want : 8 * sms);
+    rmsnorm_rstd_kernel<<<grid > 0 ? grid : 1, 256, 0, s>>>(h, rows, cols, eps, rstd);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_rmsnorm_apply(const uint16_t *h, int64_t rows, int64_t cols, const float *rstd,
+                                 const uint16_t *gamma, uint16_t *y, cudaStream_t s) {
+    const int sms = sm_count_here();
+    const int64_t want = (rows * (cols / 8) + 255) / 256;
+    const int grid = static_cast<int>(want < 8 * sms ? want : 8 * sms);
+    rmsnorm_apply_kernel<<<grid > 0 ? grid : 1, 256, 0, s>>>(h, rows, cols, rstd, gamma, y);
+    return cudaGetLastError();
+}
+
+// The thread's 8x8 block of h -> y in registers (rows from row0, columns
+// from col0; rows past the end read rstd as 0 and hold zeros anyway).
+PURO_DEV void rmsnorm_block(uint4 (&v)[8], const ProdArgs &prod, int64_t row0, int64_t col0, int64_t rows,
+                            int64_t cols) {
+    float gm[8];
+    const bool has_gamma = prod.gamma != nullptr;
+    if (has_gamma) load_gamma8(prod.gamma, col0, cols, gm);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const float rs = (row0 + i < rows) ? __ldg(prod.rstd + row0 + i) : 0.0f;
+        v[i] = rmsnorm_chunk(v[i], rs, gm, has_gamma);
+    }
+}
+
 // ------------------------------------------------------ cast kernel
 constexpr int kQT = 128;          // tile edge
 constexpr int kQThreads = 256;
@@ -204,12 +322,18 @@ PURO_DEV float mul_of(uint32_t g) { return g == 0xFFu ? __uint_as_float(0x7FC000
 //   A  partial maxima of its 8 rows and 8 columns -> shared memory
 //   B  128 threads finish the 128 row scales and 128 column scales
 //   C  every thread quantises its block twice (row scales, column scales)
-template <int FMT, int KIND, bool HAS_T>
+// PROD = kProdRmsNorm: the tile holds h, and the kernel quantises the
+// RMSNorm output y = bf16((h * rstd[row]) * gamma[col]) (fp32 products,
+// gamma optional), which it forms in place in shared memory before phase A;
+// with prod.write_y it also stores y through tm_y.  Activation kind only.
+template <int FMT, int KIND, bool HAS_T, int PROD>
 __global__ void __launch_bounds__(kQThreads, 2)
     quant_tile_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_q,
-                      const __grid_constant__ CUtensorMap tm_qt, int64_t rows, int64_t cols,
-                      uint8_t *__restrict__ scale_u8, uint8_t *__restrict__ scale_t_u8, float *scale_f,
-                      float *scale_t_f, const uint32_t *__restrict__ amax_bits, int tiles_n, int ntiles) {
+                      const __grid_constant__ CUtensorMap tm_qt, const __grid_constant__ CUtensorMap tm_y,
+                      int64_t rows, int64_t cols, uint8_t *__restrict__ scale_u8, uint8_t *__restrict__ scale_t_u8,
+                      float *scale_f, float *scale_t_f, const uint32_t *__restrict__ amax_bits, ProdArgs prod,
+                      int tiles_n, int ntiles) {
+    static_assert(PROD == kProdNone || KIND == kQuantBlockAct, "producers feed the activation quantiser");
     extern __shared__ uint8_t smem_raw[];
     QuantSmem &sm = *reinterpret_cast<QuantSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                    ~static_cast<uintptr_t>(1023));
@@ -254,6 +378,9 @@ __global__ void __launch_bounds__(kQThreads, 2)
         const int64_t c0 = static_cast<int64_t>(tile % tiles_n) * kQT;
         if (tid == 0) {
             const int next = tile + gridDim.x;
+            // with a y output, the buffer's last reader was the y store of
+            // tile it-1: all but the newest bulk group (its code stores) done
+            if (PROD != kProdNone && prod.write_y) bulk_wait_group_read<1>();
             if (next < ntiles) issue_load(next, buf ^ 1);  // its buffer was last read before (S2) of it-1
             // The previous tile's TMA stores must have read the staging tiles
             // before they are rewritten.  Per-tensor mode writes them right
@@ -270,6 +397,14 @@ __global__ void __launch_bounds__(kQThreads, 2)
         uint4 v[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) v[i] = *reinterpret_cast<const uint4 *>(in + (8 * br + i) * kQT + 8 * bc);
+        if constexpr (PROD == kProdRmsNorm) {
+            // y = bf16((h * rstd) * gamma), formed in place (each thread its
+            // own block; the y store waits for (S2)).
+            rmsnorm_block(v, prod, r0 + 8 * br, c0 + 8 * bc, rows, cols);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) *reinterpret_cast<uint4 *>(sm.in[buf] + (8 * br + i) * kQT + 8 * bc) = v[i];
+            if (prod.write_y) fence_proxy_async_smem();
+        }
 
         // ---- A: partial maxima
         if constexpr (KIND == kQuantBlockAct) {
@@ -298,6 +433,12 @@ __global__ void __launch_bounds__(kQThreads, 2)
             if (tid == 0) bulk_wait_group_read0();  // staging free (see above)
         }
         if constexpr (KIND != kQuantTensor) __syncthreads();  // (S2) partials written
+        if constexpr (PROD != kProdNone) {
+            if (prod.write_y && tid == 0) {  // every block's y is in shared memory
+                tma_store_2d(&tm_y, sm.in[buf], static_cast<int32_t>(c0), static_cast<int32_t>(r0));
+                bulk_commit_group();
+            }
+        }
 
         // ---- B: finish the scales (thread t < 128: row t; t >= 128: column t - 128)
         if constexpr (KIND == kQuantBlockAct) {
@@ -320,7 +461,12 @@ __global__ void __launch_bounds__(kQThreads, 2)
                 sm.col_mul[c] = mul_of(g);
                 sm.col_g[c] = static_cast<uint8_t>(g);
             }
-            if (tid == 0) bulk_wait_group_read0();  // staging free (see above)
+            if (tid == 0) {  // staging free (see above); a y store issued after (S2) may still run
+                if (PROD != kProdNone && prod.write_y)
+                    bulk_wait_group_read<1>();
+                else
+                    bulk_wait_group_read0();
+            }
             __syncthreads();  // (S3) scales ready, staging free
         }
 
@@ -449,10 +595,11 @@ cudaError_t launch_tensor_scale_only(const QuantArgs &a, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-template <int FMT, int KIND, bool HAS_T>
+template <int FMT, int KIND, bool HAS_T, int PROD = kProdNone>
 static cudaError_t launch_quant_t(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
-                                  const CUtensorMap &tm_qt, cudaStream_t s) {
-    auto kern = quant_tile_kernel<FMT, KIND, HAS_T>;
+                                  const CUtensorMap &tm_qt, cudaStream_t s, const CUtensorMap *tm_y = nullptr,
+                                  ProdArgs prod = ProdArgs{}) {
+    auto kern = quant_tile_kernel<FMT, KIND, HAS_T, PROD>;
     const size_t smem = sizeof(QuantSmem) + 1024;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
@@ -463,8 +610,8 @@ static cudaError_t launch_quant_t(const QuantArgs &a, const CUtensorMap &tm_x, c
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int grid = ntiles < 2 * sms ? ntiles : 2 * sms;  // persistent: two CTAs per SM
-    kern<<<grid, kQThreads, smem, s>>>(tm_x, tm_q, tm_qt, a.rows, a.cols, a.scale_u8, a.scale_t_u8, a.scale_f,
-                                       a.scale_t_f, a.amax, tiles_n, ntiles);
+    kern<<<grid, kQThreads, smem, s>>>(tm_x, tm_q, tm_qt, tm_y ? *tm_y : tm_x, a.rows, a.cols, a.scale_u8,
+                                       a.scale_t_u8, a.scale_f, a.scale_t_f, a.amax, prod, tiles_n, ntiles);
     return cudaGetLastError();
 }
 
@@ -488,6 +635,21 @@ static cudaError_t launch_quant_f(const QuantArgs &a, const CUtensorMap &tm_x, c
 cudaError_t launch_quantize(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
                             const CUtensorMap &tm_qt, cudaStream_t s) {
     return a.fmt == 0 ? launch_quant_f<0>(a, tm_x, tm_q, tm_qt, s) : launch_quant_f<1>(a, tm_x, tm_q, tm_qt, s);
+}
+
+template <int FMT>
+static cudaError_t launch_rms_f(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
+                                const CUtensorMap &tm_qt, const CUtensorMap &tm_y, const ProdArgs &prod,
+                                cudaStream_t s) {
+    return a.has_t ? launch_quant_t<FMT, kQuantBlockAct, true, kProdRmsNorm>(a, tm_x, tm_q, tm_qt, s, &tm_y, prod)
+                   : launch_quant_t<FMT, kQuantBlockAct, false, kProdRmsNorm>(a, tm_x, tm_q, tm_qt, s, &tm_y, prod);
+}
+
+cudaError_t launch_quantize_rmsnorm(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
+                                    const CUtensorMap &tm_qt, const CUtensorMap &tm_y, const ProdArgs &prod,
+                                    cudaStream_t s) {
+    return a.fmt == 0 ? launch_rms_f<0>(a, tm_x, tm_q, tm_qt, tm_y, prod, s)
+                      : launch_rms_f<1>(a, tm_x, tm_q, tm_qt, tm_y, prod, s);
 }
 
 }  // namespace puro

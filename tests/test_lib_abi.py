@@ -169,3 +169,23 @@ def test_gemm_tile_knob_validates_on_the_host(lib):
     assert lib.puro_set_gemm_tile_n(-1) == P.PURO_ERR_INVALID_ARG
     for v in (224, 256, 0):
         assert lib.puro_set_gemm_tile_n(v) == P.PURO_OK
+
+
+def test_fused_rmsnorm_validates_on_the_host(lib):
+    fake = 0x100000  # never dereferenced: every call below is refused before any CUDA call
+    args = dict(gamma=None, eps=ctypes.c_float(1e-6), fmt=P.E4M3, rstd=fake, y=None, q=fake, scale=fake,
+                q_t=None, scale_t=None, stream=None)
+
+    def call(rows, cols, **kw):
+        a = dict(args, **kw)
+        return lib.puro_fp8_quantize_rmsnorm(fake, rows, cols, a["gamma"], a["eps"], a["fmt"], a["rstd"], a["y"],
+                                             a["q"], a["scale"], a["q_t"], a["scale_t"], a["stream"])
+
+    assert call(200, 256) == P.PURO_ERR_INVALID_ARG            # rows not a multiple of 128
+    assert call(256, 200) == P.PURO_ERR_INVALID_ARG            # cols not a multiple of 128
+    assert call(256, 256, fmt=7) == P.PURO_ERR_INVALID_ARG     # unknown format
+    assert call(256, 256, eps=ctypes.c_float(-1.0)) == P.PURO_ERR_INVALID_ARG
+    assert call(256, 256, q_t=fake) == P.PURO_ERR_INVALID_ARG  # transposed codes without their scales
+    assert call(256, 256, rstd=fake + 2) == P.PURO_ERR_INVALID_ARG  # misaligned rstd
+    assert call(0, 256) == P.PURO_OK                           # empty: nothing to do
+    assert lib.puro_rmsnorm_bf16(fake, 4, 12, None, ctypes.c_float(1e-6), fake, fake, None) == P.PURO_ERR_INVALID_ARG
