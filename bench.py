@@ -400,7 +400,9 @@ def rmsnorm_fusion_measure(P, W, torch, device):
 
     out = []
     for key, (M, K) in (("C5", (32768, 1536)), ("C6", (8192, 2048))):
-        hs = [W.normal_bf16((M, K), 1.0, device, 31 + i) for i in range(2)]  # alternate: no L2 reuse across calls
+        # rotate over inputs totalling more than twice L2: no reuse across calls
+        nbuf = max(2, -(-300_000_000 // (M * K * 2)))
+        hs = [W.normal_bf16((M, K), 1.0, device, 31 + i) for i in range(nbuf)]
         gamma = W.normal_bf16((K,), 0.1, device, 33).add_(1.0)
         rstd = torch.empty(M, dtype=torch.float32, device=device)
         y = torch.empty((M, K), dtype=torch.bfloat16, device=device)
@@ -408,12 +410,12 @@ def rmsnorm_fusion_measure(P, W, torch, device):
         it = [0]
 
         def fused():
-            it[0] ^= 1
+            it[0] = (it[0] + 1) % nbuf
             P.puro_fp8_quantize_rmsnorm(hs[it[0]], gamma, 1e-6, P.E4M3, rstd, None, q.rowwise.data, q.rowwise.scale,
                                         q.colwise.data, q.colwise.scale)
 
         def unfused():
-            it[0] ^= 1
+            it[0] = (it[0] + 1) % nbuf
             P.puro_rmsnorm_bf16(hs[it[0]], gamma, 1e-6, rstd, y)
             P.quantize(y, out=q)
 
