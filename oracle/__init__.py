@@ -78,6 +78,7 @@ def _load():
         "oracle_e8m0_from_amax_array": (None, [P, I64, I, P]),
         "oracle_rmsnorm_rstd": (None, [P, I64, I64, ctypes.c_double, P]),
         "oracle_rmsnorm_apply_f32": (None, [P, I64, I64, P, P, P]),
+        "oracle_swiglu": (None, [P, P, I64, I64, I64, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -313,6 +314,31 @@ def rmsnorm_apply_f32(h, rstd_f32, gamma=None) -> np.ndarray:
     g = None if gamma is None else np.ascontiguousarray(_bits(gamma))
     out = np.empty((rows, cols), np.uint16)
     _load().oracle_rmsnorm_apply_f32(_p(hb), rows, cols, _p(r), None if g is None else _p(g), _p(out))
+    return out
+
+
+def swiglu(g, u) -> np.ndarray:
+    """bf16 bits of silu(g) * u (fp64, one rounding) for bf16 [rows, cols]
+    matrices g and u.  Row-strided views (e.g. the two halves of one
+    [rows, 2 cols] array) are passed with their row stride, not copied."""
+    gb, ub = _bits(g), _bits(u)
+    assert gb.shape == ub.shape and gb.ndim == 2
+    rows, cols = gb.shape
+
+    def strided(a):
+        if a.strides[1] == 2 and a.strides[0] % 2 == 0 and a.strides[0] >= 2 * cols:
+            return a, a.strides[0] // 2
+        a = np.ascontiguousarray(a)
+        return a, cols
+
+    gb, ldg = strided(gb)
+    ub, ldu = strided(ub)
+    if ldg != ldu:
+        gb, ub, ldg = np.ascontiguousarray(gb), np.ascontiguousarray(ub), cols
+    out = np.empty((rows, cols), np.uint16)
+    if rows and cols:
+        _load().oracle_swiglu(ctypes.c_void_p(gb.ctypes.data), ctypes.c_void_p(ub.ctypes.data), rows, cols, ldg,
+                              _p(out))
     return out
 
 

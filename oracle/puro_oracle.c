@@ -32,6 +32,8 @@
  *     attention and MLP projections, section "Model architecture and
  *     pretraining system": the Qwen3 architecture): rstd = 1/sqrt(mean h^2
  *     + eps) per row, y = bf16((h * rstd) * gamma).
+ *   - SwiGLU ahead of the quantiser (the same architecture's MLP: the down
+ *     projection receives silu(gate) * up): h = bf16(g * u / (1 + e^-g)).
  *
  * Build: gcc -std=c11 -O2 -ffp-contract=off -fPIC -shared -pthread.
  * No fast-math: every float/double operation below is an IEEE operation in
@@ -475,5 +477,26 @@ void oracle_rmsnorm_apply_f32(const uint16_t *h, int64_t rows, int64_t cols, con
             float p = bf16_to_float(h[r * cols + k]) * rstd[r];
             if (gamma) p = p * bf16_to_float(gamma[k]);
             y[r * cols + k] = oracle_bf16_from_double((double)p);
+        }
+}
+
+/* ---------------------------------------------------------------------- */
+/* SwiGLU producer                                                         */
+/* ---------------------------------------------------------------------- */
+/*
+ * The down projection's input in the gated MLP: h[r,k] = bf16_rne(silu(g) * u)
+ * with silu(g) = g / (1 + e^-g), evaluated in fp64 (libm exp) and rounded
+ * once to bf16.  g and u are bf16 [rows, cols] with rows ld elements apart
+ * (ld >= cols; views into the gate/up halves of one [rows, 2*cols] output
+ * have ld = 2*cols); h is contiguous [rows, cols].
+ */
+void oracle_swiglu(const uint16_t *g, const uint16_t *u, int64_t rows, int64_t cols, int64_t ld, uint16_t *h)
+{
+    for (int64_t r = 0; r < rows; ++r)
+        for (int64_t k = 0; k < cols; ++k) {
+            const double gv = bf16_to_double(g[r * ld + k]);
+            const double uv = bf16_to_double(u[r * ld + k]);
+            const double silu = gv / (1.0 + exp(-gv));
+            h[r * cols + k] = oracle_bf16_from_double(silu * uv);
         }
 }
