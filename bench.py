@@ -92,7 +92,7 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-bf16", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
-    ap.add_argument("--no-paper-model", action="store_true", help="skip the C6 (paper's own model shape) line")
+    ap.add_argument("--no-paper-model", action="store_true", help="skip the C6 (paper model shape), E5M2-gradient and RMSNorm-fusion lines")
     return ap.parse_args()
 
 
@@ -249,6 +249,7 @@ class LinearStack:
             self.dx.append(torch.empty((M, K), dtype=bf, device=device))
             self.dw.append(torch.empty((N, K), dtype=bf, device=device))
         self.xamax = [torch.zeros(1, dtype=torch.int32, device=device) for _ in wl.linears]
+        self.grad_fmt = P.E4M3
         # scratch for split reductions of small-output GEMMs (Wgrad of qkv / o_proj)
         ws = max([P.puro_fp8_workspace_size(N, K, M) for _, N, K in wl.linears] +
                  [P.puro_fp8_workspace_size(M, N, K) for _, N, K in wl.linears] +
@@ -265,13 +266,22 @@ class LinearStack:
             return 4 * n + 2 * (rows // 128) * (cols // 128)
         return 4 * n + 2 * n // 128
 
-    def _quant(self, x, role, q: "object"):
+    def set_grad_format(self, fmt):
+        """FP8 format of the output-gradient operands (E4M3 by default; E5M2
+        is the wider-range variant the FP8 section contrasts it with)."""
+        self.grad_fmt = fmt
+        for q in self.dyq:
+            q.rowwise.fmt = fmt
+            q.colwise.fmt = fmt
+
+    def _quant(self, x, role, q: "object", fmt=None):
         P, T = self.P, self.timer
         rows, cols = x.shape
         if self.scaling == P.SCALE_TENSOR:
             T.run("amax", 2 * rows * cols, P.puro_fp8_amax, x, q.amax)
             self.launches_per_step += 1
-        T.run("quantize", self._qbytes(rows, cols, role), P.puro_fp8_quantize, x, P.E4M3, self.scaling, role,
+        fmt = P.E4M3 if fmt is None else fmt
+        T.run("quantize", self._qbytes(rows, cols, role), P.puro_fp8_quantize, x, fmt, self.scaling, role,
               q.amax if self.scaling == P.SCALE_TENSOR else None, q.rowwise.data, q.rowwise.scale,
               q.colwise.data, q.colwise.scale)
         self.launches_per_step += 1
@@ -297,7 +307,7 @@ class LinearStack:
             for j in reversed(range(len(self.wl.linears))):
                 _, N, K = self.wl.linears[j]
                 li = self.inputs[l][j]
-                self._quant(li.dy, P.ROLE_ACT, self.dyq[j])
+                self._quant(li.dy, P.ROLE_ACT, self.dyq[j], self.grad_fmt)
                 T.run("gemm", 2.0 * self.M * N * K, P.puro_fp8_linear_dgrad, self.dyq[j].rowwise,
                       self.wq[l][j].colwise, self.dx[j], self.workspace)
                 T.run("gemm", 2.0 * self.M * N * K, P.puro_fp8_linear_wgrad, self.dyq[j].colwise, self.xqt[l][j],
@@ -429,6 +439,41 @@ def rmsnorm_fusion_measure(P, W, torch, device):
         del hs, y, q
         torch.cuda.empty_cache()
     return out
+
+
+def timed_steps(torch, stack, steps, warmup):
+    """Step time of `stack` (CUDA events around `steps` steps after `warmup`)
+    and the per-category launch totals of the timed steps."""
+    for _ in range(warmup):
+        stack.step()
+    torch.cuda.synchronize()
+    stack.timer.pending.clear()
+    stack.timer.enabled = True
+    s = torch.cuda.Event(enable_timing=True)
+    e = torch.cuda.Event(enable_timing=True)
+    s.record()
+    for _ in range(steps):
+        stack.step()
+    e.record()
+    torch.cuda.synchronize()
+    stack.timer.enabled = False
+    return s.elapsed_time(e) * 1e-3 / steps, stack.timer.totals()
+
+
+def grad_format_measure(P, torch, stack, steps=3, warmup=2):
+    """The same step with E5M2 output-gradient operands (weights and
+    activations stay E4M3): the quantiser writes E5M2 codes for dY and its
+    transposed copy, and Dgrad / Wgrad take one E5M2 operand."""
+    stack.set_grad_format(P.E5M2)
+    try:
+        step_s, per = timed_steps(torch, stack, steps, warmup)
+    finally:
+        stack.set_grad_format(P.E4M3)
+    g, q = per["gemm"], per["quantize"]
+    return {"variant": "dY and dY^T in E5M2, X and W in E4M3 (block scaling)",
+            "value": stack.flops_per_step() / step_s / 1e12, "unit": "TFLOP/s", "ms_per_step": step_s * 1e3,
+            "steps": steps, "warmup": warmup, "gemm_only_tflops": g["units"] / g["time_s"] / 1e12,
+            "quantize_gbs": q["units"] / q["time_s"] / 1e9}
 
 
 def paper_model_measure(P, W, torch, device, scaling, steps=5, warmup=3):
@@ -723,6 +768,8 @@ def main():
             result["bf16_comparison"] = bf16_layer_speedup(P, torch, stack)
         except (RuntimeError, torch.cuda.OutOfMemoryError) as exc:  # report, do not hide
             result["bf16_comparison"] = {"error": str(exc)}
+    if rank == 0 and world == 1 and not args.no_paper_model and args.scaling == "block":
+        result["e5m2_gradients"] = grad_format_measure(P, torch, stack)
     if not args.no_e2e:
         result["e2e"] = e2e_measure(P, torch, stack, max(1, min(args.steps, 3)))
         if world > 1:
