@@ -92,7 +92,7 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-bf16", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
-    ap.add_argument("--no-paper-model", action="store_true", help="skip the C6 (paper model shape), E5M2-gradient and RMSNorm-fusion lines")
+    ap.add_argument("--no-paper-model", action="store_true", help="skip the C6 (paper model shape), E5M2-gradient and producer-fusion lines")
     return ap.parse_args()
 
 
@@ -441,6 +441,59 @@ def rmsnorm_fusion_measure(P, W, torch, device):
     return out
 
 
+def swiglu_fusion_measure(P, W, torch, device):
+    """SwiGLU fused ahead of the activation quantiser against SwiGLU (bf16 h
+    written and read back) followed by the quantiser, on the down-projection
+    inputs of C5 (F = 8960) and C6 (F = 6144): gate and up are the two halves
+    of one [M, 2F] gate/up output."""
+
+    def timeit(fn, reps=20):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        s = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        s.record()
+        for _ in range(reps):
+            fn()
+        e.record()
+        torch.cuda.synchronize()
+        return s.elapsed_time(e) * 1e-3 / reps
+
+    out = []
+    for key, (M, F) in (("C5", (32768, 8960)), ("C6", (8192, 6144))):
+        # rotate over inputs totalling more than twice L2: no reuse across calls
+        nbuf = max(2, -(-300_000_000 // (M * 2 * F * 2)))
+        gus = [W.student_t3_f32((M, 2 * F), device, 41 + i).to(torch.bfloat16) for i in range(nbuf)]
+        h = torch.empty((M, F), dtype=torch.bfloat16, device=device)
+        q = P.quantize(h)
+        it = [0]
+
+        def fused():
+            it[0] = (it[0] + 1) % nbuf
+            gu = gus[it[0]]
+            P.puro_fp8_quantize_swiglu(gu[:, :F], gu[:, F:], P.E4M3, None, q.rowwise.data, q.rowwise.scale,
+                                       q.colwise.data, q.colwise.scale)
+
+        def unfused():
+            it[0] = (it[0] + 1) % nbuf
+            gu = gus[it[0]]
+            P.puro_swiglu_bf16(gu[:, :F], gu[:, F:], h)
+            P.quantize(h, out=q)
+
+        tf, tu = timeit(fused), timeit(unfused)
+        n = M * F
+        # algorithmic bytes of the fused op: read gate and up, write both FP8
+        # copies and their scales
+        fused_bytes = 4 * n + 2 * n + 2 * n // 128
+        out.append({"input": f"{key} down-projection input [{M}, {F}] from gate/up [{M}, {2 * F}]",
+                    "fused_us": tf * 1e6, "unfused_us": tu * 1e6, "fused_over_unfused_time": tf / tu,
+                    "fused_algorithmic_gbs": fused_bytes / tf / 1e9})
+        del gus, h, q
+        torch.cuda.empty_cache()
+    return out
+
+
 def timed_steps(torch, stack, steps, warmup):
     """Step time of `stack` (CUDA events around `steps` steps after `warmup`)
     and the per-category launch totals of the timed steps."""
@@ -783,6 +836,7 @@ def main():
         torch.cuda.empty_cache()
         result["paper_model_shape"] = paper_model_measure(P, W, torch, device, args.scaling)
         result["rmsnorm_quantize_fusion"] = rmsnorm_fusion_measure(P, W, torch, device)
+        result["swiglu_quantize_fusion"] = swiglu_fusion_measure(P, W, torch, device)
     if rank == 0:
         print(json.dumps(result), flush=True)
     if world > 1:

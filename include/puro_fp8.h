@@ -171,6 +171,42 @@ puro_status_t puro_rmsnorm_bf16(const void *h, int64_t rows, int64_t cols, const
                                 float *rstd, void *y, void *stream);
 
 /*
+ * SwiGLU fused ahead of the blockwise activation quantiser.
+ *
+ * The model's MLP is gated (section "Model architecture and pretraining
+ * system": the Qwen3 architecture): the down projection receives
+ *     y[r,k] = bf16(silu(gate[r,k]) * up[r,k]),   silu(g) = g / (1 + e^-g),
+ * evaluated in fp32 (sigmoid from e^-|g|, so nothing overflows; the
+ * exponential and the reciprocal are single special-function instructions,
+ * with subnormal values of e^-|g| kept by an exact power-of-two scaling).
+ * This entry
+ * point quantises y exactly as puro_fp8_quantize does with PURO_SCALE_BLOCK /
+ * PURO_ROLE_ACT (1x128 groups, optional transposed copy) without writing y,
+ * which the MLP's backward does not need (it keeps gate and up).
+ *   gate, up: bf16 [rows, cols] with rows ld elements apart (ld >= cols, a
+ *     multiple of 8): the two halves of one [rows, 2*cols] gate/up output are
+ *     passed as gate = out, up = out + cols, ld = 2*cols.  16-byte aligned.
+ *   rows and cols multiples of 128.
+ *   y: bf16 [rows, cols] contiguous, or NULL: written only when asked.
+ *   q, scale, q_t, scale_t: as in puro_fp8_quantize.
+ * Every code and scale is an exact function of y.  y itself agrees with the
+ * exactly rounded silu(gate) * up to within one bf16 ulp, and equals it for
+ * all but about 1e-5 of typical inputs.  One kernel on `stream`; gate and up
+ * are each read once.
+ */
+puro_status_t puro_fp8_quantize_swiglu(const void *gate, const void *up, int64_t rows, int64_t cols, int64_t ld,
+                                       int32_t fmt, void *y, uint8_t *q, void *scale, uint8_t *q_t, void *scale_t,
+                                       void *stream);
+
+/*
+ * The same SwiGLU without the quantiser: y (bf16, contiguous [rows, cols]) as
+ * above, cols a multiple of 8.  The unfused comparison for the fused entry
+ * point.
+ */
+puro_status_t puro_swiglu_bf16(const void *gate, const void *up, int64_t rows, int64_t cols, int64_t ld, void *y,
+                               void *stream);
+
+/*
  * The three FP8 GEMMs of a linear layer with weight W [N, K], input X [M, K]
  * and output gradient dY [M, N] (appendix "FP8 implementation pipeline":
  * Fprop, Dgrad and Wgrad all use blockwise E4M3 operands).  Each computes

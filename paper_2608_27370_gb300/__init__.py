@@ -69,6 +69,8 @@ _SIGNATURES = {
     "puro_fp8_quantize": (_I32, [_P, _I64, _I64, _I32, _I32, _I32, _P, _P, _P, _P, _P, _P]),
     "puro_fp8_quantize_rmsnorm": (_I32, [_P, _I64, _I64, _P, ctypes.c_float, _I32, _P, _P, _P, _P, _P, _P, _P]),
     "puro_rmsnorm_bf16": (_I32, [_P, _I64, _I64, _P, ctypes.c_float, _P, _P, _P]),
+    "puro_fp8_quantize_swiglu": (_I32, [_P, _P, _I64, _I64, _I64, _I32, _P, _P, _P, _P, _P, _P]),
+    "puro_swiglu_bf16": (_I32, [_P, _P, _I64, _I64, _I64, _P, _P]),
     "puro_fp8_linear_fprop": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_dgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_wgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
@@ -171,6 +173,43 @@ def puro_fp8_quantize_rmsnorm(h: torch.Tensor, gamma: Optional[torch.Tensor], ep
         _ptr(rstd, torch.float32, "rstd"), _ptr(y, torch.bfloat16, "y"), _ptr(q, u8, "q"), _ptr(scale, u8, "scale"),
         _ptr(q_t, u8, "q_t"), _ptr(scale_t, u8, "scale_t"), _stream(stream))
     _check("puro_fp8_quantize_rmsnorm", st)
+
+
+def _gate_up(gate: torch.Tensor, up: torch.Tensor):
+    """Pointers and the shared row stride of gate / up (bf16 [rows, cols]
+    CUDA tensors with unit column stride, e.g. the halves of one output)."""
+    for name, t in (("gate", gate), ("up", up)):
+        if not t.is_cuda or t.dtype != torch.bfloat16 or t.dim() != 2:
+            raise ValueError(f"{name} must be a 2-D bf16 CUDA tensor")
+        if t.numel() and t.stride(1) != 1:
+            raise ValueError(f"{name} must have unit column stride")
+    if gate.shape != up.shape:
+        raise ValueError("gate and up differ in shape")
+    rows, cols = gate.shape
+    ld = gate.stride(0) if rows > 1 else cols
+    if rows > 1 and up.stride(0) != ld:
+        raise ValueError("gate and up must share one row stride")
+    return gate.data_ptr() or None, up.data_ptr() or None, rows, cols, ld
+
+
+def puro_fp8_quantize_swiglu(gate: torch.Tensor, up: torch.Tensor, fmt: int, y: Optional[torch.Tensor],
+                             q: torch.Tensor, scale: torch.Tensor, q_t: Optional[torch.Tensor] = None,
+                             scale_t: Optional[torch.Tensor] = None, stream=None) -> None:
+    """SwiGLU (silu(gate) * up, bf16) fused ahead of the blockwise activation
+    quantiser: writes the codes and scales as puro_fp8_quantize does, and y
+    (bf16) only when given.  gate and up may be row-strided views."""
+    g, u, rows, cols, ld = _gate_up(gate, up)
+    u8 = torch.uint8
+    st = load_library().puro_fp8_quantize_swiglu(
+        g, u, rows, cols, ld, fmt, _ptr(y, torch.bfloat16, "y"), _ptr(q, u8, "q"), _ptr(scale, u8, "scale"),
+        _ptr(q_t, u8, "q_t"), _ptr(scale_t, u8, "scale_t"), _stream(stream))
+    _check("puro_fp8_quantize_swiglu", st)
+
+
+def puro_swiglu_bf16(gate: torch.Tensor, up: torch.Tensor, y: torch.Tensor, stream=None) -> None:
+    g, u, rows, cols, ld = _gate_up(gate, up)
+    st = load_library().puro_swiglu_bf16(g, u, rows, cols, ld, _ptr(y, torch.bfloat16, "y"), _stream(stream))
+    _check("puro_swiglu_bf16", st)
 
 
 def puro_rmsnorm_bf16(h: torch.Tensor, gamma: Optional[torch.Tensor], eps: float, rstd: torch.Tensor,

@@ -317,6 +317,60 @@ PURO_API puro_status_t puro_fp8_quantize_rmsnorm(const void *h, int64_t rows, in
     return cuda_status(launch_quantize_rmsnorm(a, tm_x, tm_q, tm_qt, tm_y, prod, s));
 }
 
+// SwiGLU fused ahead of the activation quantiser.
+PURO_API puro_status_t puro_fp8_quantize_swiglu(const void *gate, const void *up, int64_t rows, int64_t cols,
+                                                int64_t ld, int32_t fmt, void *y, uint8_t *q, void *scale,
+                                                uint8_t *q_t, void *scale_t, void *stream) {
+    if (!valid_fmt(fmt) || rows < 0 || cols < 0 || ld < cols || ld % 8) return PURO_ERR_INVALID_ARG;
+    if (rows % 128 || cols % 128) return PURO_ERR_INVALID_ARG;
+    if ((q_t == nullptr) != (scale_t == nullptr)) return PURO_ERR_INVALID_ARG;
+    if (rows > INT32_MAX || cols > INT32_MAX || ld > INT32_MAX) return PURO_ERR_UNSUPPORTED;
+    if (rows == 0 || cols == 0) return PURO_OK;
+    if (!gate || !up || !q || !scale) return PURO_ERR_INVALID_ARG;
+    if (!aligned16(gate) || !aligned16(up) || !aligned16(y) || !aligned16(q) || !aligned16(scale) ||
+        !aligned16(q_t) || !aligned16(scale_t))
+        return PURO_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    QuantArgs a{};
+    a.fmt = fmt;
+    a.rows = rows;
+    a.cols = cols;
+    a.has_t = q_t != nullptr;
+    a.kind = kQuantBlockAct;
+    a.scale_u8 = static_cast<uint8_t *>(scale);
+    a.scale_t_u8 = static_cast<uint8_t *>(scale_t);
+    a.x = static_cast<const uint16_t *>(gate);
+    CUtensorMap tm_x, tm_q, tm_qt, tm_y;
+    if (!make_map(&tm_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, gate, cols, rows, ld * 2, 128, 128,
+                  CU_TENSOR_MAP_SWIZZLE_NONE) ||
+        !make_map(&tm_q, CU_TENSOR_MAP_DATA_TYPE_UINT8, q, cols, rows, cols, 128, 128, CU_TENSOR_MAP_SWIZZLE_NONE))
+        return PURO_ERR_CUDA;
+    tm_qt = tm_q;
+    if (a.has_t && !make_map(&tm_qt, CU_TENSOR_MAP_DATA_TYPE_UINT8, q_t, rows, cols, rows, 128, 128,
+                             CU_TENSOR_MAP_SWIZZLE_128B))
+        return PURO_ERR_CUDA;
+    tm_y = tm_x;
+    if (y && !make_map(&tm_y, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, y, cols, rows, cols * 2, 128, 128,
+                       CU_TENSOR_MAP_SWIZZLE_NONE))
+        return PURO_ERR_CUDA;
+    ProdArgs prod{};
+    prod.write_y = y != nullptr;
+    prod.up = static_cast<const uint16_t *>(up);
+    prod.ld = ld;
+    return cuda_status(launch_quantize_swiglu(a, tm_x, tm_q, tm_qt, tm_y, prod, s));
+}
+
+// The same SwiGLU without the quantiser (the unfused comparison).
+PURO_API puro_status_t puro_swiglu_bf16(const void *gate, const void *up, int64_t rows, int64_t cols, int64_t ld,
+                                        void *y, void *stream) {
+    if (rows < 0 || cols < 0 || cols % 8 || ld < cols || ld % 8) return PURO_ERR_INVALID_ARG;
+    if (rows == 0 || cols == 0) return PURO_OK;
+    if (!gate || !up || !y || !aligned16(gate) || !aligned16(up) || !aligned16(y)) return PURO_ERR_INVALID_ARG;
+    return cuda_status(launch_swiglu_apply(static_cast<const uint16_t *>(gate), static_cast<const uint16_t *>(up),
+                                           rows, cols, ld, static_cast<uint16_t *>(y),
+                                           static_cast<cudaStream_t>(stream)));
+}
+
 // The same RMSNorm without the quantiser (the unfused comparison).
 PURO_API puro_status_t puro_rmsnorm_bf16(const void *h, int64_t rows, int64_t cols, const void *gamma, float eps,
                                          float *rstd, void *y, void *stream) {

@@ -37,11 +37,14 @@ cudaError_t launch_amax(const uint16_t *x, int64_t n, uint32_t *amax, cudaStream
 enum QuantProd : int {
     kProdNone = 0,
     kProdRmsNorm = 1,  // y = bf16((h * rstd[row]) * gamma[col])
+    kProdSwiGlu = 2,   // y = bf16(silu(gate) * up)
 };
 struct ProdArgs {
     const float *rstd;      // kProdRmsNorm: [rows]
     const uint16_t *gamma;  // kProdRmsNorm: bf16 [cols], or null (no gain)
     bool write_y;           // also store y (through tm_y)
+    const uint16_t *up;     // kProdSwiGlu: bf16 [rows, cols], rows ld elements apart
+    int64_t ld;             // kProdSwiGlu: row stride of up (and of the gate tm_x maps)
 };
 
 // rstd[r] = 1 / sqrt(mean(h[r,:]^2) + eps) (cols a multiple of 8).
@@ -62,6 +65,17 @@ cudaError_t launch_quantize(const QuantArgs &a, const CUtensorMap &tm_x, const C
 cudaError_t launch_quantize_rmsnorm(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
                                     const CUtensorMap &tm_qt, const CUtensorMap &tm_y, const ProdArgs &prod,
                                     cudaStream_t s);
+
+// The activation quantiser fed by SwiGLU (a.kind must be kQuantBlockAct, rows
+// and cols multiples of 128): tm_x maps the gate (bf16 [rows, cols], row
+// stride prod.ld elements), prod.up the up projection with the same stride.
+cudaError_t launch_quantize_swiglu(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
+                                   const CUtensorMap &tm_qt, const CUtensorMap &tm_y, const ProdArgs &prod,
+                                   cudaStream_t s);
+// y = bf16(silu(gate) * up), the unfused application (cols a multiple of 8;
+// gate and up rows ld elements apart, y contiguous).
+cudaError_t launch_swiglu_apply(const uint16_t *gate, const uint16_t *up, int64_t rows, int64_t cols, int64_t ld,
+                                uint16_t *y, cudaStream_t s);
 
 // Writes only the per-tensor scale_inv (used for empty tensors).
 cudaError_t launch_tensor_scale_only(const QuantArgs &a, cudaStream_t s);

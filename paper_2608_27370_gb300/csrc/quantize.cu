@@ -289,6 +289,87 @@ PURO_DEV void rmsnorm_block(uint4 (&v)[8], const ProdArgs &prod, int64_t row0, i
     }
 }
 
+// ------------------------------------------------------ SwiGLU producer
+// 2^x and 1/x by the special-function unit (PTX ex2.approx / rcp.approx:
+// relative error around 2^-22; subnormal results flush to zero).
+PURO_DEV float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+PURO_DEV float rcp_approx(float x) {
+    float y;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// silu(g) = g * sigmoid(g) in fp32, with sigmoid from t = e^-|g| (in (0, 1],
+// so nothing overflows): sigmoid(g) = r = 1 / (1 + t) for g >= 0, t * r
+// otherwise.  t = 2^(64 - |g| log2 e) * 2^-64: the special-function
+// exponent stays in the normal range for |g| < 131.7, and the exact IEEE
+// scaling by 2^-64 (and t * r) keep subnormal values of e^-|g|.  The
+// special-function forms cost one instruction each; their few-ulp fp32
+// error is far below the bf16 rounding that follows (with correctly rounded
+// exp and division the fused kernel is bound by those instructions, not by
+// memory).  Below g ~ -131.7 t is zero, where the exact product
+// silu(g) * u is below 1e-55 |u|.  NaN stays NaN; -inf gives NaN (-inf * 0).
+PURO_DEV float silu_f32(float g) {
+    const float a = fabsf(g);
+    const float t = __fmul_rn(ex2_approx(fmaf(a, -1.44269504f, 64.0f)), 0x1p-64f);
+    const float r = rcp_approx(__fadd_rn(1.0f, t));
+    return __fmul_rn(g, g >= 0.0f ? r : __fmul_rn(t, r));
+}
+
+// y = bf16(silu(g) * u) for an 8-value chunk.
+PURO_DEV uint4 swiglu_chunk(uint4 g, uint4 u) {
+    const uint32_t gw[4] = {g.x, g.y, g.z, g.w}, uw[4] = {u.x, u.y, u.z, u.w};
+    uint32_t out[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const float lo = __fmul_rn(silu_f32(__uint_as_float(gw[j] << 16)), __uint_as_float(uw[j] << 16));
+        const float hi = __fmul_rn(silu_f32(__uint_as_float(gw[j] & 0xFFFF0000u)), __uint_as_float(uw[j] & 0xFFFF0000u));
+        __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+        out[j] = *reinterpret_cast<uint32_t *>(&v);
+    }
+    return make_uint4(out[0], out[1], out[2], out[3]);
+}
+
+// Unfused comparison: y = bf16(silu(gate) * up), one 8-value chunk per thread
+// and step; gate and up rows ld elements apart, y contiguous.
+__global__ void __launch_bounds__(256) swiglu_apply_kernel(const uint16_t *__restrict__ gate,
+                                                           const uint16_t *__restrict__ up, int64_t rows,
+                                                           int64_t cols, int64_t ld, uint16_t *__restrict__ y) {
+    const int64_t per_row = cols / 8;
+    const int64_t chunks = rows * per_row;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < chunks; i += stride) {
+        const int64_t r = i / per_row, c = (i - r * per_row) * 8;
+        const uint4 g = __ldg(reinterpret_cast<const uint4 *>(gate + r * ld + c));
+        const uint4 u = __ldg(reinterpret_cast<const uint4 *>(up + r * ld + c));
+        reinterpret_cast<uint4 *>(y)[i] = swiglu_chunk(g, u);
+    }
+}
+
+cudaError_t launch_swiglu_apply(const uint16_t *gate, const uint16_t *up, int64_t rows, int64_t cols, int64_t ld,
+                                uint16_t *y, cudaStream_t s) {
+    const int sms = sm_count_here();
+    const int64_t want = (rows * (cols / 8) + 255) / 256;
+    const int grid = static_cast<int>(want < 8 * sms ? want : 8 * sms);
+    swiglu_apply_kernel<<<grid > 0 ? grid : 1, 256, 0, s>>>(gate, up, rows, cols, ld, y);
+    return cudaGetLastError();
+}
+
+// The thread's 8x8 block of the up projection for a tile (rows and columns
+// are whole tiles: the SwiGLU entry point requires multiples of 128).  Each
+// row's 16 bytes are one of 16 consecutive chunks a half-warp reads together.
+PURO_DEV void load_up_block(uint4 (&u)[8], const ProdArgs &prod, int tile, int tiles_n, int br, int bc) {
+    const int64_t row0 = static_cast<int64_t>(tile / tiles_n) * 128 + 8 * br;
+    const int64_t col0 = static_cast<int64_t>(tile % tiles_n) * 128 + 8 * bc;
+    const uint16_t *p = prod.up + row0 * prod.ld + col0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) u[i] = __ldg(reinterpret_cast<const uint4 *>(p + i * prod.ld));
+}
+
 // ------------------------------------------------------ cast kernel
 constexpr int kQT = 128;          // tile edge
 constexpr int kQThreads = 256;
@@ -326,6 +407,10 @@ PURO_DEV float mul_of(uint32_t g) { return g == 0xFFu ? __uint_as_float(0x7FC000
 // RMSNorm output y = bf16((h * rstd[row]) * gamma[col]) (fp32 products,
 // gamma optional), which it forms in place in shared memory before phase A;
 // with prod.write_y it also stores y through tm_y.  Activation kind only.
+// PROD = kProdSwiGlu: the tile holds the gate g, and the kernel quantises
+// y = bf16(silu(g) * u); each thread reads its 8x8 block of the up
+// projection u straight into registers one tile ahead, so those loads are in
+// flight while the previous tile is quantised.
 template <int FMT, int KIND, bool HAS_T, int PROD>
 __global__ void __launch_bounds__(kQThreads, 2)
     quant_tile_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_q,
@@ -372,6 +457,10 @@ __global__ void __launch_bounds__(kQThreads, 2)
     };
     int tile = blockIdx.x;
     if (tid == 0 && tile < ntiles) issue_load(tile, 0);
+    uint4 un[8];  // kProdSwiGlu: this thread's block of u for the current tile
+    if constexpr (PROD == kProdSwiGlu) {
+        if (tile < ntiles) load_up_block(un, prod, tile, tiles_n, br, bc);
+    }
     for (int it = 0; tile < ntiles; ++it, tile += gridDim.x) {
         const int buf = it & 1;
         const int64_t r0 = static_cast<int64_t>(tile / tiles_n) * kQT;
@@ -404,6 +493,16 @@ __global__ void __launch_bounds__(kQThreads, 2)
 #pragma unroll
             for (int i = 0; i < 8; ++i) *reinterpret_cast<uint4 *>(sm.in[buf] + (8 * br + i) * kQT + 8 * bc) = v[i];
             if (prod.write_y) fence_proxy_async_smem();
+        } else if constexpr (PROD == kProdSwiGlu) {
+            // y = bf16(silu(g) * u), formed in place like the RMSNorm output
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                v[i] = swiglu_chunk(v[i], un[i]);
+                *reinterpret_cast<uint4 *>(sm.in[buf] + (8 * br + i) * kQT + 8 * bc) = v[i];
+            }
+            if (prod.write_y) fence_proxy_async_smem();
+            const int next = tile + gridDim.x;
+            if (next < ntiles) load_up_block(un, prod, next, tiles_n, br, bc);
         }
 
         // ---- A: partial maxima
@@ -650,6 +749,21 @@ cudaError_t launch_quantize_rmsnorm(const QuantArgs &a, const CUtensorMap &tm_x,
                                     cudaStream_t s) {
     return a.fmt == 0 ? launch_rms_f<0>(a, tm_x, tm_q, tm_qt, tm_y, prod, s)
                       : launch_rms_f<1>(a, tm_x, tm_q, tm_qt, tm_y, prod, s);
+}
+
+template <int FMT>
+static cudaError_t launch_swiglu_f(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
+                                   const CUtensorMap &tm_qt, const CUtensorMap &tm_y, const ProdArgs &prod,
+                                   cudaStream_t s) {
+    return a.has_t ? launch_quant_t<FMT, kQuantBlockAct, true, kProdSwiGlu>(a, tm_x, tm_q, tm_qt, s, &tm_y, prod)
+                   : launch_quant_t<FMT, kQuantBlockAct, false, kProdSwiGlu>(a, tm_x, tm_q, tm_qt, s, &tm_y, prod);
+}
+
+cudaError_t launch_quantize_swiglu(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
+                                   const CUtensorMap &tm_qt, const CUtensorMap &tm_y, const ProdArgs &prod,
+                                   cudaStream_t s) {
+    return a.fmt == 0 ? launch_swiglu_f<0>(a, tm_x, tm_q, tm_qt, tm_y, prod, s)
+                      : launch_swiglu_f<1>(a, tm_x, tm_q, tm_qt, tm_y, prod, s);
 }
 
 }  // namespace puro

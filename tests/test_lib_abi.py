@@ -189,3 +189,23 @@ def test_fused_rmsnorm_validates_on_the_host(lib):
     assert call(256, 256, rstd=fake + 2) == P.PURO_ERR_INVALID_ARG  # misaligned rstd
     assert call(0, 256) == P.PURO_OK                           # empty: nothing to do
     assert lib.puro_rmsnorm_bf16(fake, 4, 12, None, ctypes.c_float(1e-6), fake, fake, None) == P.PURO_ERR_INVALID_ARG
+
+
+def test_fused_swiglu_validates_on_the_host(lib):
+    fake = 0x100000  # never dereferenced: every call below is refused before any CUDA call
+
+    def call(rows, cols, ld, fmt=P.E4M3, gate=fake, up=fake, y=None, q_t=None, scale_t=None):
+        return lib.puro_fp8_quantize_swiglu(gate, up, rows, cols, ld, fmt, y, fake, fake, q_t, scale_t, None)
+
+    assert call(200, 256, 512) == P.PURO_ERR_INVALID_ARG            # rows not a multiple of 128
+    assert call(256, 200, 400) == P.PURO_ERR_INVALID_ARG            # cols not a multiple of 128
+    assert call(256, 256, 128) == P.PURO_ERR_INVALID_ARG            # row stride shorter than a row
+    assert call(256, 256, 260) == P.PURO_ERR_INVALID_ARG            # row stride not 16-byte aligned
+    assert call(256, 256, 512, fmt=7) == P.PURO_ERR_INVALID_ARG     # unknown format
+    assert call(256, 256, 512, q_t=fake) == P.PURO_ERR_INVALID_ARG  # transposed codes without their scales
+    assert call(256, 256, 512, up=fake + 2) == P.PURO_ERR_INVALID_ARG  # misaligned up
+    assert call(256, 256, 512, up=None) == P.PURO_ERR_INVALID_ARG
+    assert call(0, 256, 512) == P.PURO_OK                           # empty: nothing to do
+    assert lib.puro_swiglu_bf16(fake, fake, 4, 12, 16, fake, None) == P.PURO_ERR_INVALID_ARG  # cols % 8
+    assert lib.puro_swiglu_bf16(fake, fake, 4, 16, 8, fake, None) == P.PURO_ERR_INVALID_ARG   # ld < cols
+    assert lib.puro_swiglu_bf16(fake, fake, 0, 16, 16, fake, None) == P.PURO_OK
