@@ -79,6 +79,8 @@ def _load():
         "oracle_rmsnorm_rstd": (None, [P, I64, I64, ctypes.c_double, P]),
         "oracle_rmsnorm_apply_f32": (None, [P, I64, I64, P, P, P]),
         "oracle_swiglu": (None, [P, P, I64, I64, I64, P]),
+        "oracle_frobenius_norm": (ctypes.c_double, [P, I64]),
+        "oracle_muonh_step": (None, [P, P, I64, ctypes.c_double, ctypes.c_double, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -339,6 +341,23 @@ def swiglu(g, u) -> np.ndarray:
     if rows and cols:
         _load().oracle_swiglu(ctypes.c_void_p(gb.ctypes.data), ctypes.c_void_p(ub.ctypes.data), rows, cols, ldg,
                               _p(out))
+    return out
+
+
+def frobenius_norm(x) -> float:
+    """||x||_F of an fp32 array (any shape), accumulated in fp64."""
+    a = np.ascontiguousarray(np.asarray(x, np.float32))
+    return float(_load().oracle_frobenius_norm(_p(a), a.size))
+
+
+def muonh_step(w, u, eta: float, radius: float) -> np.ndarray:
+    """The hyperball update of fp32 W along the Muon direction u (same
+    shape): R W~ / ||W~||_F with W~ = W - eta R u / ||u||_F, in fp64."""
+    wa = np.ascontiguousarray(np.asarray(w, np.float32))
+    ua = np.ascontiguousarray(np.asarray(u, np.float32))
+    assert wa.shape == ua.shape
+    out = np.empty(wa.shape, np.float64)
+    _load().oracle_muonh_step(_p(wa), _p(ua), wa.size, ctypes.c_double(eta), ctypes.c_double(radius), _p(out))
     return out
 
 

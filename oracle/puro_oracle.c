@@ -34,6 +34,9 @@
  *     + eps) per row, y = bf16((h * rstd) * gamma).
  *   - SwiGLU ahead of the quantiser (the same architecture's MLP: the down
  *     projection receives silu(gate) * up): h = bf16(g * u / (1 + e^-g)).
+ *   - The MuonH hyperball step (section "Hyperball Optimization", Eq.
+ *     hyperball-update): u_hat = u / ||u||_F, W~ = W - eta R u_hat,
+ *     W <- R W~ / ||W~||_F with R = ||W_0||_F fixed.
  *
  * Build: gcc -std=c11 -O2 -ffp-contract=off -fPIC -shared -pthread.
  * No fast-math: every float/double operation below is an IEEE operation in
@@ -499,4 +502,36 @@ void oracle_swiglu(const uint16_t *g, const uint16_t *u, int64_t rows, int64_t c
             const double silu = gv / (1.0 + exp(-gv));
             h[r * cols + k] = oracle_bf16_from_double(silu * uv);
         }
+}
+
+/* ---------------------------------------------------------------------- */
+/* MuonH hyperball step                                                    */
+/* ---------------------------------------------------------------------- */
+/* Frobenius norm of n fp32 values, in fp64 (index order). */
+double oracle_frobenius_norm(const float *x, int64_t n)
+{
+    double ss = 0.0;
+    for (int64_t i = 0; i < n; ++i) ss += (double)x[i] * (double)x[i];
+    return sqrt(ss);
+}
+
+/*
+ * One hyperball update of a wrapped matrix (n values, any shape: the
+ * Frobenius norm is that of the flattened matrix), in the order of the
+ * equation: normalise the Muon direction, step by eta * R along it, then
+ * project back onto the sphere of radius R.  w_new is fp64 (the fp32 master
+ * weight the kernels write is compared against it within a tolerance).
+ */
+void oracle_muonh_step(const float *w, const float *u, int64_t n, double eta, double radius, double *w_new)
+{
+    const double unorm = oracle_frobenius_norm(u, n);
+    double tnorm2 = 0.0;
+    for (int64_t i = 0; i < n; ++i) {
+        const double u_hat = (double)u[i] / unorm;
+        const double wt = (double)w[i] - eta * radius * u_hat;
+        w_new[i] = wt;
+        tnorm2 += wt * wt;
+    }
+    const double tnorm = sqrt(tnorm2);
+    for (int64_t i = 0; i < n; ++i) w_new[i] = radius * (w_new[i] / tnorm);
 }
