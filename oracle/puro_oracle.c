@@ -521,13 +521,15 @@ double oracle_frobenius_norm(const float *x, int64_t n)
  * equation: normalise the Muon direction, step by eta * R along it, then
  * project back onto the sphere of radius R.  w_new is fp64 (the fp32 master
  * weight the kernels write is compared against it within a tolerance).
+ * Reading where the equation is undefined: a zero Muon direction (||u|| = 0)
+ * takes no step (u_hat = 0), so W is only projected.
  */
 void oracle_muonh_step(const float *w, const float *u, int64_t n, double eta, double radius, double *w_new)
 {
     const double unorm = oracle_frobenius_norm(u, n);
     double tnorm2 = 0.0;
     for (int64_t i = 0; i < n; ++i) {
-        const double u_hat = (double)u[i] / unorm;
+        const double u_hat = unorm > 0.0 ? (double)u[i] / unorm : 0.0;
         const double wt = (double)w[i] - eta * radius * u_hat;
         w_new[i] = wt;
         tnorm2 += wt * wt;

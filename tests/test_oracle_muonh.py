@@ -50,6 +50,14 @@ def test_zero_step_is_the_projection():
     assert np.allclose(got, want, rtol=1e-13, atol=0)
 
 
+def test_zero_direction_takes_no_step():
+    # the equation divides by ||u|| = 0; the reading taken: no step
+    rng = np.random.default_rng(6)
+    w = rng.standard_normal(300).astype(np.float32)
+    got = O.muonh_step(w, np.zeros(300, np.float32), 0.1, 2.0)
+    assert np.array_equal(got, O.muonh_step(w, np.ones(300, np.float32), 0.0, 2.0))
+
+
 def test_orthogonal_update_closed_form():
     # <W, u> = 0 and ||W|| = R:  ||W~||^2 = R^2 (1 + eta^2), so
     # W_new = (W - eta R u_hat) / sqrt(1 + eta^2)
