@@ -92,7 +92,7 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-bf16", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
-    ap.add_argument("--no-paper-model", action="store_true", help="skip the C6 (paper model shape), E5M2-gradient and producer-fusion lines")
+    ap.add_argument("--no-paper-model", action="store_true", help="skip the C6 (paper model shape), E5M2-gradient, producer-fusion and MuonH lines")
     return ap.parse_args()
 
 
@@ -494,6 +494,50 @@ def swiglu_fusion_measure(P, W, torch, device):
     return out
 
 
+def muonh_measure(P, W, torch, device, peaks, steps=3, warmup=2):
+    """The MuonH hyperball step over every wrapped matrix of C5 (the 112
+    linear weights of the 28 layers, 1.30 G parameters): fp32 master weights
+    and Muon directions resident in HBM, the bf16 weight copy written."""
+    import math
+
+    wl = W.WORKLOADS["C5"]
+    mats = []
+    for l in range(wl.layers):
+        for j, (_, N, K) in enumerate(wl.linears):
+            w = W.normal_f32((N, K), 0.02, device, 7000 + 16 * l + j)
+            u = W.normal_f32((N, K), 1.0 / math.sqrt(K), device, 9000 + 16 * l + j)
+            mats.append((w, u, torch.empty((N, K), dtype=torch.bfloat16, device=device),
+                         float(torch.linalg.vector_norm(w.double()))))
+    sums = torch.empty((len(mats), 3), dtype=torch.float64, device=device)
+    ws = torch.empty(P.puro_muonh_grouped_workspace_size(mats), dtype=torch.uint8, device=device)
+
+    def step():  # every matrix in one grouped step: three launches
+        P.puro_muonh_step_grouped(mats, 4.08e-4, sums, ws)
+
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize()
+    s = torch.cuda.Event(enable_timing=True)
+    e = torch.cuda.Event(enable_timing=True)
+    s.record()
+    for _ in range(steps):
+        step()
+    e.record()
+    torch.cuda.synchronize()
+    t = s.elapsed_time(e) * 1e-3 / steps
+    n = sum(w.numel() for w, _, _, _ in mats)
+    # algorithmic bytes per element: read W and u (reduce), read W and u,
+    # write W and the bf16 copy (apply)
+    gbs = 22.0 * n / t / 1e9
+    out = {"workload": f"MuonH hyperball step over C5's {len(mats)} linear weights ({n / 1e9:.2f} G fp32 parameters)",
+           "ms_per_step": t * 1e3, "params_per_s": n / t, "algorithmic_gbs": gbs,
+           "hbm_frac": gbs / peaks["hbm_gbs"], "launches_per_step": 3 * (-(-len(mats) // 128)), "steps": steps,
+           "warmup": warmup}
+    del mats, sums, ws
+    torch.cuda.empty_cache()
+    return out
+
+
 def timed_steps(torch, stack, steps, warmup):
     """Step time of `stack` (CUDA events around `steps` steps after `warmup`)
     and the per-category launch totals of the timed steps."""
@@ -837,6 +881,7 @@ def main():
         result["paper_model_shape"] = paper_model_measure(P, W, torch, device, args.scaling)
         result["rmsnorm_quantize_fusion"] = rmsnorm_fusion_measure(P, W, torch, device)
         result["swiglu_quantize_fusion"] = swiglu_fusion_measure(P, W, torch, device)
+        result["muonh_step"] = muonh_measure(P, W, torch, device, peaks)
     if rank == 0:
         print(json.dumps(result), flush=True)
     if world > 1:

@@ -347,6 +347,67 @@ void puro_set_wait_timeout_ns(uint64_t ns);
  */
 puro_status_t puro_set_gemm_tile_n(int32_t tile_n);
 
+/*
+ * MuonH hyperball step (section "Hyperball Optimization", Eq.
+ * hyperball-update), for one wrapped matrix W (FP32 master weight) and its
+ * Muon update direction u:
+ *     u_hat = u / ||u||_F,   W~ = W - eta R u_hat,   W <- R W~ / ||W~||_F,
+ * R = ||W_0||_F being the matrix's fixed radius (puro_muonh_reduce of W_0
+ * with itself gives R^2 as sums[0]).  The Muon orthogonalisation that
+ * produces u is not part of this step (the paper does not specify it).
+ *
+ * The step is two passes over memory: a reduction of the three sums
+ *     sums = {S_ww, S_wu, S_uu} = {sum W^2, sum W u, sum u^2}   (fp64)
+ * and an update W <- s (W - c u), c = eta R / sqrt(S_uu),
+ * s = R / sqrt(S_ww - 2 c S_wu + c^2 S_uu), with c and s rounded to fp32.
+ * The sums are additive over any partition of the matrix: a caller that
+ * shards W across devices runs puro_muonh_reduce on each shard, all-reduces
+ * the three doubles, then runs puro_muonh_apply on each shard.
+ *   w, u: fp32, n values (any shape; the Frobenius norm is that of the
+ *     flattened matrix), n a multiple of 4, 16-byte aligned; w updated in place.
+ *   sums: device double[3], 8-byte aligned (written by reduce, read by apply).
+ *   workspace: device scratch of puro_muonh_workspace_size(n) bytes, 8-byte
+ *     aligned (per-block partial sums).
+ *   eta >= 0 (the Hyperball learning rate), radius > 0, both finite.
+ *   w_bf16: optional bf16 [n] copy of the updated W (8-byte aligned), or NULL.
+ * A zero direction (S_uu = 0) takes no step: W is only projected (the
+ * equation is undefined there).  If W~ = 0 the result is NaN.  The
+ * reduction order is fixed by n alone, so results are deterministic and the
+ * same on every device.  n = 0 does nothing (reduce writes zero sums).
+ * Three kernels for the step: the chunk sums, their fixed-order total, and
+ * the update.
+ */
+size_t puro_muonh_workspace_size(int64_t n);
+puro_status_t puro_muonh_reduce(const float *w, const float *u, int64_t n, double *sums, void *workspace,
+                                size_t workspace_bytes, void *stream);
+puro_status_t puro_muonh_apply(float *w, const float *u, int64_t n, const double *sums, double eta, double radius,
+                               void *w_bf16, void *stream);
+/* reduce then apply, on one device (three kernels on `stream`). */
+puro_status_t puro_muonh_step(float *w, const float *u, int64_t n, double eta, double radius, double *sums,
+                              void *workspace, size_t workspace_bytes, void *w_bf16, void *stream);
+
+/*
+ * The same step for many matrices at once (every wrapped matrix of a model):
+ * three kernel launches per 128 matrices instead of three per matrix.  Each
+ * matrix is cut into chunks by its own size alone, so its result is bit for
+ * bit the one puro_muonh_step gives.
+ *   mats: host array of `count` descriptors (read during the call only).
+ *   sums: device double[count][3], written (the three sums of each matrix).
+ *   workspace: puro_muonh_grouped_workspace_size(mats, count) bytes.
+ * Every descriptor is checked before anything is enqueued.
+ */
+typedef struct {
+    float *w;           /* fp32 master weight [n], updated in place (16-byte aligned) */
+    const float *u;     /* fp32 Muon direction [n] (16-byte aligned) */
+    void *w_bf16;       /* bf16 copy [n] written after the update (8-byte aligned), or NULL */
+    int64_t n;          /* number of values, a multiple of 4 */
+    double radius;      /* R = ||W_0||_F > 0 */
+} puro_muonh_matrix_t;
+
+size_t puro_muonh_grouped_workspace_size(const puro_muonh_matrix_t *mats, int32_t count);
+puro_status_t puro_muonh_step_grouped(const puro_muonh_matrix_t *mats, int32_t count, double eta, double *sums,
+                                      void *workspace, size_t workspace_bytes, void *stream);
+
 /* Human-readable name of a status code (static string). */
 const char *puro_status_string(puro_status_t s);
 

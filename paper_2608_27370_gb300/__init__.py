@@ -70,6 +70,12 @@ _SIGNATURES = {
     "puro_fp8_quantize_rmsnorm": (_I32, [_P, _I64, _I64, _P, ctypes.c_float, _I32, _P, _P, _P, _P, _P, _P, _P]),
     "puro_rmsnorm_bf16": (_I32, [_P, _I64, _I64, _P, ctypes.c_float, _P, _P, _P]),
     "puro_fp8_quantize_swiglu": (_I32, [_P, _P, _I64, _I64, _I64, _I32, _P, _P, _P, _P, _P, _P]),
+    "puro_muonh_workspace_size": (ctypes.c_size_t, [_I64]),
+    "puro_muonh_reduce": (_I32, [_P, _P, _I64, _P, _P, ctypes.c_size_t, _P]),
+    "puro_muonh_apply": (_I32, [_P, _P, _I64, _P, ctypes.c_double, ctypes.c_double, _P, _P]),
+    "puro_muonh_step": (_I32, [_P, _P, _I64, ctypes.c_double, ctypes.c_double, _P, _P, ctypes.c_size_t, _P, _P]),
+    "puro_muonh_grouped_workspace_size": (ctypes.c_size_t, [_P, _I32]),
+    "puro_muonh_step_grouped": (_I32, [_P, _I32, ctypes.c_double, _P, _P, ctypes.c_size_t, _P]),
     "puro_swiglu_bf16": (_I32, [_P, _P, _I64, _I64, _I64, _P, _P]),
     "puro_fp8_linear_fprop": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_dgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
@@ -210,6 +216,83 @@ def puro_swiglu_bf16(gate: torch.Tensor, up: torch.Tensor, y: torch.Tensor, stre
     g, u, rows, cols, ld = _gate_up(gate, up)
     st = load_library().puro_swiglu_bf16(g, u, rows, cols, ld, _ptr(y, torch.bfloat16, "y"), _stream(stream))
     _check("puro_swiglu_bf16", st)
+
+
+def puro_muonh_workspace_size(n: int) -> int:
+    return int(load_library().puro_muonh_workspace_size(n))
+
+
+def puro_muonh_reduce(w: torch.Tensor, u: torch.Tensor, sums: torch.Tensor, workspace: torch.Tensor,
+                      stream=None) -> None:
+    """sums (fp64 [3], device) = {sum W^2, sum W u, sum u^2} of fp32 W and u."""
+    if w.numel() != u.numel():
+        raise ValueError("w and u differ in size")
+    st = load_library().puro_muonh_reduce(_ptr(w, torch.float32, "w"), _ptr(u, torch.float32, "u"), w.numel(),
+                                          _ptr(sums, torch.float64, "sums"), _ptr(workspace, None, "workspace"),
+                                          workspace.numel() * workspace.element_size(), _stream(stream))
+    _check("puro_muonh_reduce", st)
+
+
+def puro_muonh_apply(w: torch.Tensor, u: torch.Tensor, sums: torch.Tensor, eta: float, radius: float,
+                     w_bf16: Optional[torch.Tensor] = None, stream=None) -> None:
+    if w.numel() != u.numel() or (w_bf16 is not None and w_bf16.numel() != w.numel()):
+        raise ValueError("w, u and w_bf16 differ in size")
+    st = load_library().puro_muonh_apply(_ptr(w, torch.float32, "w"), _ptr(u, torch.float32, "u"), w.numel(),
+                                         _ptr(sums, torch.float64, "sums"), float(eta), float(radius),
+                                         _ptr(w_bf16, torch.bfloat16, "w_bf16"), _stream(stream))
+    _check("puro_muonh_apply", st)
+
+
+def puro_muonh_step(w: torch.Tensor, u: torch.Tensor, eta: float, radius: float, sums: torch.Tensor,
+                    workspace: torch.Tensor, w_bf16: Optional[torch.Tensor] = None, stream=None) -> None:
+    """One MuonH hyperball update of the fp32 master weight w (in place)
+    along the Muon direction u; optionally writes the bf16 copy."""
+    if w.numel() != u.numel() or (w_bf16 is not None and w_bf16.numel() != w.numel()):
+        raise ValueError("w, u and w_bf16 differ in size")
+    st = load_library().puro_muonh_step(_ptr(w, torch.float32, "w"), _ptr(u, torch.float32, "u"), w.numel(),
+                                        float(eta), float(radius), _ptr(sums, torch.float64, "sums"),
+                                        _ptr(workspace, None, "workspace"),
+                                        workspace.numel() * workspace.element_size(),
+                                        _ptr(w_bf16, torch.bfloat16, "w_bf16"), _stream(stream))
+    _check("puro_muonh_step", st)
+
+
+class puro_muonh_matrix_t(ctypes.Structure):
+    _fields_ = [("w", ctypes.c_void_p), ("u", ctypes.c_void_p), ("w_bf16", ctypes.c_void_p),
+                ("n", ctypes.c_int64), ("radius", ctypes.c_double)]
+
+
+def _muonh_table(mats):
+    """ctypes array of descriptors from (w, u, w_bf16 or None, radius) tuples."""
+    arr = (puro_muonh_matrix_t * max(1, len(mats)))()
+    for i, (w, u, wb, r) in enumerate(mats):
+        if w.numel() != u.numel() or (wb is not None and wb.numel() != w.numel()):
+            raise ValueError(f"matrix {i}: w, u and w_bf16 differ in size")
+        arr[i] = puro_muonh_matrix_t(_ptr(w, torch.float32, "w"), _ptr(u, torch.float32, "u"),
+                                     _ptr(wb, torch.bfloat16, "w_bf16"), w.numel(), float(r))
+    return arr
+
+
+def puro_muonh_grouped_workspace_size(mats) -> int:
+    return int(load_library().puro_muonh_grouped_workspace_size(_muonh_table(mats), len(mats)))
+
+
+def puro_muonh_step_grouped(mats, eta: float, sums: torch.Tensor, workspace: torch.Tensor, stream=None) -> None:
+    """The hyperball step for every (w, u, w_bf16 or None, radius) in mats;
+    sums: fp64 [len(mats), 3] on the device."""
+    table = _muonh_table(mats)
+    st = load_library().puro_muonh_step_grouped(table, len(mats), float(eta), _ptr(sums, torch.float64, "sums"),
+                                                _ptr(workspace, None, "workspace"),
+                                                workspace.numel() * workspace.element_size(), _stream(stream))
+    _check("puro_muonh_step_grouped", st)
+
+
+def muonh_radius(w0: torch.Tensor) -> float:
+    """R = ||W_0||_F (fp64, through puro_muonh_reduce; synchronises)."""
+    sums = torch.empty(3, dtype=torch.float64, device=w0.device)
+    ws = torch.empty(max(8, puro_muonh_workspace_size(w0.numel())), dtype=torch.uint8, device=w0.device)
+    puro_muonh_reduce(w0, w0, sums, ws)
+    return float(sums[0].sqrt().item())
 
 
 def puro_rmsnorm_bf16(h: torch.Tensor, gamma: Optional[torch.Tensor], eps: float, rstd: torch.Tensor,

@@ -1,6 +1,6 @@
 """Build the CUDA library libpuro_fp8.so in-tree with nvcc for sm_103a.
 
-Four translation units are compiled in parallel and linked into one shared
+Five translation units are compiled in parallel and linked into one shared
 object with the CUDA runtime linked statically, so the library loads on a
 machine without a GPU driver (only the first CUDA call needs one).
 """
@@ -17,7 +17,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libpuro_fp8.so")
-SOURCES = ["api.cu", "quantize.cu", "gemm.cu", "noalloc.cu"]
+SOURCES = ["api.cu", "quantize.cu", "gemm.cu", "noalloc.cu", "muonh.cu"]
 HEADERS = ["ptx.cuh", "internal.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",

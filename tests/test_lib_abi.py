@@ -209,3 +209,41 @@ def test_fused_swiglu_validates_on_the_host(lib):
     assert lib.puro_swiglu_bf16(fake, fake, 4, 12, 16, fake, None) == P.PURO_ERR_INVALID_ARG  # cols % 8
     assert lib.puro_swiglu_bf16(fake, fake, 4, 16, 8, fake, None) == P.PURO_ERR_INVALID_ARG   # ld < cols
     assert lib.puro_swiglu_bf16(fake, fake, 0, 16, 16, fake, None) == P.PURO_OK
+
+
+def test_muonh_validates_on_the_host(lib):
+    fake = 0x100000  # never dereferenced: every call below is refused before any CUDA call
+    ws = lib.puro_muonh_workspace_size(1 << 20)
+    assert ws > 0 and ws % 24 == 0 and lib.puro_muonh_workspace_size(0) == 0
+    # chunks of n/4096 values, clamped to [4096, 65536]: 24 bytes per chunk
+    assert lib.puro_muonh_workspace_size(4096) == 24
+    assert lib.puro_muonh_workspace_size(4100) == 48
+    assert lib.puro_muonh_workspace_size(1 << 24) == 24 * 1024
+    assert lib.puro_muonh_workspace_size(1 << 30) == 24 * (1 << 14)
+    assert lib.puro_muonh_reduce(fake, fake, 6, fake, fake, ws, None) == P.PURO_ERR_INVALID_ARG  # n % 4
+    assert lib.puro_muonh_reduce(fake + 8, fake, 1 << 20, fake, fake, ws, None) == P.PURO_ERR_INVALID_ARG
+    assert lib.puro_muonh_reduce(fake, fake, 1 << 20, fake, fake, ws - 8, None) == P.PURO_ERR_INVALID_ARG
+    assert lib.puro_muonh_apply(fake, fake, 1 << 20, fake, -1.0, 1.0, None, None) == P.PURO_ERR_INVALID_ARG
+    assert lib.puro_muonh_apply(fake, fake, 1 << 20, fake, 0.1, 0.0, None, None) == P.PURO_ERR_INVALID_ARG
+    assert lib.puro_muonh_apply(fake, fake, 1 << 20, fake, float("nan"), 1.0, None, None) == P.PURO_ERR_INVALID_ARG
+    assert lib.puro_muonh_apply(fake, fake, 1 << 20, fake, 0.1, 1.0, fake + 4, None) == P.PURO_ERR_INVALID_ARG
+    assert lib.puro_muonh_step(fake, fake, 0, 0.1, 1.0, fake, None, 0, None, None) == P.PURO_OK
+
+
+def test_muonh_grouped_validates_on_the_host(lib):
+    fake = 0x100000
+    M = P.puro_muonh_matrix_t
+    good = M(fake, fake + 0x10000, None, 1 << 16, 1.0)
+    arr = (M * 3)(good, M(fake, fake, None, 6, 1.0), good)            # the middle one has n % 4 != 0
+    assert lib.puro_muonh_step_grouped(arr, 3, 0.1, fake, fake, 1 << 20, None) == P.PURO_ERR_INVALID_ARG
+    arr = (M * 2)(good, M(fake, fake, None, 1024, -1.0))               # negative radius
+    assert lib.puro_muonh_step_grouped(arr, 2, 0.1, fake, fake, 1 << 20, None) == P.PURO_ERR_INVALID_ARG
+    arr = (M * 2)(good, good)
+    need = lib.puro_muonh_grouped_workspace_size(arr, 2)
+    assert need == 2 * lib.puro_muonh_workspace_size(1 << 16)
+    assert lib.puro_muonh_step_grouped(arr, 2, 0.1, fake, fake, need - 8, None) == P.PURO_ERR_INVALID_ARG
+    assert lib.puro_muonh_step_grouped(arr, 2, float("inf"), fake, fake, need, None) == P.PURO_ERR_INVALID_ARG
+    assert lib.puro_muonh_step_grouped(arr, 0, 0.1, None, None, 0, None) == P.PURO_OK
+    # launches of 128 matrices reuse the scratch: 200 matrices need the larger batch only
+    big = (M * 200)(*([good] * 200))
+    assert lib.puro_muonh_grouped_workspace_size(big, 200) == 128 * lib.puro_muonh_workspace_size(1 << 16)
