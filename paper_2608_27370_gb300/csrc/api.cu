@@ -123,8 +123,6 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
                   static_cast<uint32_t>(tile_n / 2), CU_TENSOR_MAP_SWIZZLE_128B) ||
         !(accumulate_f32
               ? make_map(&m.d, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, d, N, M, N * 4, 32, 32, CU_TENSOR_MAP_SWIZZLE_128B)
-          : tile_n == 256
-              ? make_map(&m.d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B)
               : make_map(&m.d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B)))
         return PURO_ERR_CUDA;
     m.ws = m.d;
@@ -176,7 +174,7 @@ puro_status_t bf16_gemm(const void *a, const void *b, void *d, int64_t M, int64_
                   CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_map(&m.b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, b, K, N, K * 2, kGemmBKBytes / 2, kGemmBN / 2,
                   CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&m.d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B))
+        !make_map(&m.d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d, N, M, N * 2, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B))
         return PURO_ERR_CUDA;
     m.ws = m.d;
     m.sfa = m.d;

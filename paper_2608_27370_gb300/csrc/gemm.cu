@@ -180,8 +180,9 @@ PURO_DEV void pack_bf16x8(const uint32_t *src, float sab, uint32_t (&w)[4]) {
 // Mp = num_m * 256 (rows split * Mp + m), so that a ragged last pair tile
 // stays inside its chunk; kGemmOutF32Add adds the FP32 tile to D (an FP32
 // main-grad, one TMA reduce-add per element, so the result is deterministic).
-// The FP32 forms are BN = 256 only.  tm_d: D with box {64, 32} and the 128-byte swizzle (BN = 256) or
-// box {32, 32} and the 64-byte swizzle (BN = 224).
+// The FP32 forms are BN = 256 only.  tm_d: BF16 D with box {32, 32} and the
+// 64-byte swizzle, or FP32 D / workspace with box {32, 32} and the 128-byte
+// swizzle.
 // tm_sfa / tm_sfb (block kind only): the scale vectors of A / B viewed as
 // uint32 [chunks, 128] (one 512-byte chunk per row), box {128, 1}; tm_sfb is
 // read only with BN = 256.
@@ -453,7 +454,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         uint8_t *stage_buf = sm.epi[q];
         const uint32_t tempty0 = mapa_shared(smem_u32(&sm.tempty[0]), 0);  // the even CTA's
         int local = 0;
-        uint32_t pieces = 0;  // BN = 224: 32-column pieces stored, alternating staging halves
+        uint32_t pieces = 0;  // BF16 output: 32-column pieces stored, alternating staging halves
         for (int u = pair; u < p.num_units; u += num_pairs, ++local) {
             const WorkUnit wu = work_unit<BN>(p, u);
             const int m0 = wu.m0 + kBM * static_cast<int>(rank), n0 = wu.n0;  // this CTA's rows
@@ -509,71 +510,36 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 tc_fence_before_sync();
                 __syncwarp();
                 if (lane == 0) mbar_arrive_cluster(tempty0 + 8u * buf);
-            } else if constexpr (BN == 256) {
-                // Shifted (block kind): the half in the columns the next
-                // tile's accumulator shares ([128, 256) of tensor memory)
-                // first, and the accumulator released once it is in
-                // registers.  Dense kinds: halves in order, released after
-                // the second load.
+            } else {
+                // BF16 tile in two halves of 128 columns (BN = 224: 128 + 96).
+                // Shifted (block kind, BN = 256): the half in the columns the
+                // next tile's accumulator shares ([128, 256) of tensor
+                // memory) first, and the accumulator released once it is in
+                // registers; otherwise halves in order, released after the
+                // second load.  Each half leaves in 32-column pieces (64
+                // bytes per row, 64-byte swizzle: 16-byte unit i of row l at
+                // i ^ ((l / 2) % 4)) that alternate between the two 2 KB
+                // halves of the staging tile, so a piece is written while the
+                // previous one is still being stored.
                 const int h_first = kShifted ? ((local & 1) ? 0 : 1) : 0;
+                constexpr int kReleaseAt = kShifted ? 0 : 1;
 #pragma unroll 1
                 for (int hh = 0; hh < 2; ++hh) {
                     const int h = hh ^ h_first;
+                    const int nc = h == 0 ? 4 : (BN - 128) / 32;
                     uint32_t r[4][32];
 #pragma unroll
-                    for (int c = 0; c < 4; ++c) tmem_ld_32x32b_x32(t_row + 128 * h + 32 * c, r[c]);
+                    for (int c = 0; c < 4; ++c)
+                        if (c < nc) tmem_ld_32x32b_x32(t_row + 128 * h + 32 * c, r[c]);
                     tmem_ld_wait();
-                    if (hh == (kShifted ? 0 : 1)) {
+                    if (hh == kReleaseAt) {
                         tc_fence_before_sync();
                         __syncwarp();
                         if (lane == 0) mbar_arrive_cluster(tempty0 + 8u * buf);  // accumulator free for the next tile
                     }
-                    // Two chunks of 64 columns (128 bytes per row) through the
-                    // per-warp staging tile, 16-byte unit i of row l at i ^ (l % 8).
-#pragma unroll
-                    for (int ch = 0; ch < 2; ++ch) {
-                        const int col = n0 + 128 * h + 64 * ch;
-                        if (col >= p.N) break;
-                        if (lane == 0) bulk_wait_group_read0();
-                        __syncwarp();
-                        uint8_t *row = stage_buf + 128 * lane;
-#pragma unroll
-                        for (int i = 0; i < 8; ++i) {
-                            uint32_t w[4];
-                            pack_bf16x8<KIND>(&r[2 * ch + (i >> 2)][8 * (i & 3)], sab, w);
-                            *reinterpret_cast<uint4 *>(row + 16 * (i ^ (lane & 7))) = make_uint4(w[0], w[1], w[2], w[3]);
-                        }
-                        fence_proxy_async_smem();
-                        __syncwarp();
-                        if (lane == 0) {
-                            tma_store_2d(&tm_d, stage_buf, col, m0 + 32 * q);
-                            bulk_commit_group();
-                        }
-                    }
-                }
-            } else {
-                // BN = 224, double-buffered: columns [0, 128) then [128, 224),
-                // released after the second load; 32-column pieces (64 bytes
-                // per row, 64-byte swizzle: 16-byte unit i of row l at
-                // i ^ ((l / 2) % 4)) alternate between the two 2 KB halves of
-                // the staging tile, so a piece is written while the previous
-                // one is still being stored.
-#pragma unroll 1
-                for (int hh = 0; hh < 2; ++hh) {
-                    const int nc = hh == 0 ? 4 : (BN - 128) / 32;
-                    uint32_t r[4][32];
-#pragma unroll
-                    for (int c = 0; c < 4; ++c)
-                        if (c < nc) tmem_ld_32x32b_x32(t_row + 128 * hh + 32 * c, r[c]);
-                    tmem_ld_wait();
-                    if (hh == 1) {
-                        tc_fence_before_sync();
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive_cluster(tempty0 + 8u * buf);  // accumulator free
-                    }
 #pragma unroll
                     for (int c = 0; c < 4; ++c) {
-                        const int col = n0 + 128 * hh + 32 * c;
+                        const int col = n0 + 128 * h + 32 * c;
                         if (c >= nc || col >= p.N) break;
                         uint8_t *half = stage_buf + 2048 * (pieces & 1u);
                         if (lane == 0) bulk_wait_group_read<1>();  // the store that last read this half is done

@@ -178,22 +178,33 @@ PURO_DEV void store_scale_vec(uint8_t *__restrict__ base, int64_t row, int64_t k
 
 // rstd of each row of h [rows, cols] (cols a multiple of 8), one warp per
 // row: fp32 sums of squares in a fixed order (lane-strided 8-value chunks,
-// then a butterfly), then an IEEE division and square root.
+// then a butterfly), then an IEEE division and square root.  A lane loads
+// up to eight of its chunks before it adds any (in chunk order), so a
+// row's loads are in flight together.
 __global__ void __launch_bounds__(256) rmsnorm_rstd_kernel(const uint16_t *__restrict__ h, int64_t rows, int64_t cols,
                                                            float eps, float *__restrict__ rstd) {
+    constexpr int kBatch = 8;
     const int lane = threadIdx.x & 31;
     const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
+    const int64_t n8 = cols / 8;
     for (int64_t r = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5); r < rows; r += nwarps) {
         const uint4 *row = reinterpret_cast<const uint4 *>(h + r * cols);
         float a = 0.0f, b = 0.0f;
-        for (int64_t c = lane; c < cols / 8; c += 32) {
-            const uint4 w = __ldg(row + c);
-            const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+        for (int64_t c0 = lane; c0 < n8; c0 += 32 * kBatch) {
+            uint4 w[kBatch];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const float lo = __uint_as_float(ws[j] << 16), hi = __uint_as_float(ws[j] & 0xFFFF0000u);
-                a = __fmaf_rn(lo, lo, a);
-                b = __fmaf_rn(hi, hi, b);
+            for (int k = 0; k < kBatch; ++k)
+                w[k] = c0 + 32 * k < n8 ? __ldg(row + c0 + 32 * k) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+            for (int k = 0; k < kBatch; ++k) {
+                if (c0 + 32 * k >= n8) break;
+                const uint32_t ws[4] = {w[k].x, w[k].y, w[k].z, w[k].w};
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float lo = __uint_as_float(ws[j] << 16), hi = __uint_as_float(ws[j] & 0xFFFF0000u);
+                    a = __fmaf_rn(lo, lo, a);
+                    b = __fmaf_rn(hi, hi, b);
+                }
             }
         }
         float ss = a + b;

@@ -1,0 +1,58 @@
+"""Launch one of the library's fused or optimizer kernels a few times on a
+fixed synthetic input, for profiling with ncu (one kernel per run, small
+enough that a full capture ends in seconds).  Not part of the library.
+
+    python -m paper_2608_27370_gb300.microbench.kernels swiglu   # [8192, 6144] from gate/up [8192, 12288]
+    python -m paper_2608_27370_gb300.microbench.kernels rmsnorm  # [32768, 1536] with a gain
+    python -m paper_2608_27370_gb300.microbench.kernels muonh    # gate_up [17920, 1536] + down [1536, 8960]
+
+Each input is larger than L2.  Every call is made twice: the second is the
+one to capture (ncu -s skips the first).
+"""
+import math
+import sys
+
+import torch
+
+import paper_2608_27370_gb300 as P
+from paper_2608_27370_gb300 import workloads as W
+
+
+def main(which: str) -> None:
+    dev = "cuda"
+    P.load_library()
+    if which == "swiglu":
+        M, F = 8192, 6144
+        gu = W.student_t3_f32((M, 2 * F), dev, 41).to(torch.bfloat16)
+        q = P.quantize(torch.empty((M, F), dtype=torch.bfloat16, device=dev))
+        for _ in range(2):
+            P.puro_fp8_quantize_swiglu(gu[:, :F], gu[:, F:], P.E4M3, None, q.rowwise.data, q.rowwise.scale,
+                                       q.colwise.data, q.colwise.scale)
+    elif which == "rmsnorm":
+        M, K = 32768, 1536
+        h = W.normal_bf16((M, K), 1.0, dev, 31)
+        g = W.normal_bf16((K,), 0.1, dev, 33).add_(1.0)
+        rstd = torch.empty(M, dtype=torch.float32, device=dev)
+        q = P.quantize(h)
+        for _ in range(2):
+            P.puro_fp8_quantize_rmsnorm(h, g, 1e-6, P.E4M3, rstd, None, q.rowwise.data, q.rowwise.scale,
+                                        q.colwise.data, q.colwise.scale)
+    elif which == "muonh":
+        mats = []
+        for j, (N, K) in enumerate(((17920, 1536), (1536, 8960))):
+            w = W.normal_f32((N, K), 0.02, dev, 70 + j)
+            u = W.normal_f32((N, K), 1.0 / math.sqrt(K), dev, 90 + j)
+            mats.append((w, u, torch.empty((N, K), dtype=torch.bfloat16, device=dev),
+                         float(torch.linalg.vector_norm(w.double()))))
+        sums = torch.empty((len(mats), 3), dtype=torch.float64, device=dev)
+        ws = torch.empty(P.puro_muonh_grouped_workspace_size(mats), dtype=torch.uint8, device=dev)
+        for _ in range(2):
+            P.puro_muonh_step_grouped(mats, 4.08e-4, sums, ws)
+    else:
+        raise SystemExit(f"unknown kernel {which!r}: swiglu, rmsnorm or muonh")
+    torch.cuda.synchronize()
+    print("ok", which)
+
+
+if __name__ == "__main__":
+    main(sys.argv[1] if len(sys.argv) > 1 else "swiglu")
