@@ -5,6 +5,7 @@ enough that a full capture ends in seconds).  Not part of the library.
     python -m paper_2608_27370_gb300.microbench.kernels swiglu   # [8192, 6144] from gate/up [8192, 12288]
     python -m paper_2608_27370_gb300.microbench.kernels rmsnorm  # [32768, 1536] with a gain
     python -m paper_2608_27370_gb300.microbench.kernels muonh    # gate_up [17920, 1536] + down [1536, 8960]
+    python -m paper_2608_27370_gb300.microbench.kernels gemm     # down Fprop, M = 8192, N = 1536, K = 8960
 
 Each input is larger than L2.  Every call is made twice: the second is the
 one to capture (ncu -s skips the first).
@@ -48,8 +49,15 @@ def main(which: str) -> None:
         ws = torch.empty(P.puro_muonh_grouped_workspace_size(mats), dtype=torch.uint8, device=dev)
         for _ in range(2):
             P.puro_muonh_step_grouped(mats, 4.08e-4, sums, ws)
+    elif which == "gemm":
+        M, N, K = 8192, 1536, 8960
+        a = P.quantize(W.normal_bf16((M, K), 1.0, dev, 1), transpose=False)
+        b = P.quantize(W.normal_bf16((N, K), 0.02, dev, 2), P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT, transpose=False)
+        d = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
+        for _ in range(2):
+            P.puro_fp8_linear_fprop(a.rowwise, b.rowwise, d)
     else:
-        raise SystemExit(f"unknown kernel {which!r}: swiglu, rmsnorm or muonh")
+        raise SystemExit(f"unknown kernel {which!r}: swiglu, rmsnorm, muonh or gemm")
     torch.cuda.synchronize()
     print("ok", which)
 
