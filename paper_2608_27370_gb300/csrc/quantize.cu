@@ -489,8 +489,14 @@ __global__ void __launch_bounds__(kQThreads, 2)
             // phase C and the stores' reads overlap that work.
             if constexpr (KIND == kQuantTensor) bulk_wait_group_read0();
         }
+        // Every thread waits on the tile's barrier itself, which makes the
+        // TMA-written tile visible to it.  The blockwise kinds need no CTA
+        // barrier here: the shared buffers they write before (S2) were last
+        // read before (S4) of the previous tile.  Per-tensor mode writes the
+        // staging tiles right away, so it waits (S1) for thread 0 to have
+        // seen the previous stores read them.
         mbar_wait_bounded(&sm.full[buf], static_cast<uint32_t>(it >> 1) & 1u, kQuantWaitNs);
-        __syncthreads();                                    // (S1) this tile's input landed
+        if constexpr (KIND == kQuantTensor) __syncthreads();  // (S1) staging free
 
         // ---- the thread's 8x8 block: v[i] = row 8br+i, columns 8bc .. 8bc+7
         const uint16_t *in = sm.in[buf];
