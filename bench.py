@@ -47,9 +47,9 @@ FP8_PER_BF16 = 2.0  # nominal dense ratio (4.5 / 2.25 PFLOP/s)
 # reported as null once they change or for another workload.
 CAPTURED_TRAFFIC = {
     "gemm": {"files": ["gemm.cu", "ptx.cuh", "internal.h", "api.cu"], "sha1": "2a776834d7abc2f7",
-             "bytes_per_call": 455678485, "algorithmic_bytes_per_call": 417016966},
-    "quantize": {"files": ["quantize.cu", "ptx.cuh", "internal.h", "api.cu"], "sha1": "d18172d57b272c3c",
-                 "bytes_per_call": 379282837, "algorithmic_bytes_per_call": 417016966},
+             "bytes_per_call": 456054720, "algorithmic_bytes_per_call": 417016966},
+    "quantize": {"files": ["quantize.cu", "ptx.cuh", "internal.h", "api.cu"], "sha1": "8948c135ca23107f",
+                 "bytes_per_call": 375261034, "algorithmic_bytes_per_call": 417016966},
 }
 CAPTURED_TRAFFIC_WORKLOAD = ("C5", 32768, "block")
 CAPTURED_TRAFFIC_PROFILE = "profiles/dram_traffic_C5_layer_M32768.md"
@@ -849,7 +849,7 @@ def main():
                      "peak_source": f"2 x bf16_tflops_sustained ({peak_src}); kernel timed inside a long step",
                      "traffic": captured_traffic("gemm", traffic_wl),
                      "traffic_note": "DRAM bytes per GEMM call (avg of one layer's 12), " + CAPTURED_TRAFFIC_PROFILE},
-        "roofline_quantize": {"bound": "hbm", "kernel": "quant_tile_kernel", "achieved": quant_gbs,
+        "roofline_quantize": {"bound": "hbm", "kernel": "quant_act_kernel (X, dY) + quant_tile_kernel (W)", "achieved": quant_gbs,
                               "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": quant_gbs / peaks["hbm_gbs"],
                               "peak_source": f"hbm_gbs ({peak_src})",
                               "traffic": captured_traffic("quantize", traffic_wl),

@@ -4,14 +4,17 @@
 // the GEMM reduction dimension for activations and activation gradients,
 // 128x128 blocks for weights -- each a power of two).
 //
-// Both kernels are HBM-bandwidth bound.  The cast kernel reads each 128x128
-// BF16 tile once (one TMA load per tile, double buffered), computes the row-group and the
-// column-group scales from the same shared-memory copy, and writes the
-// rowwise codes and the transposed codes through shared memory with TMA
-// stores (the transposed staging tile uses the 128-byte swizzle so the
-// column pass stores without bank conflicts).  The arithmetic per value is
-// kept to a widening shift, half a packed fp32 multiply and half a paired
-// cvt, since at HBM rates the kernel is otherwise instruction bound.
+// The kernels are HBM-bandwidth bound.  The cast kernels read each 128x128
+// BF16 tile once (one TMA load per tile, double buffered), compute the
+// scales from the same shared-memory copy, and write the rowwise codes and
+// the transposed codes through shared memory with TMA stores (the
+// transposed staging tile uses the 128-byte swizzle so the column pass
+// stores without bank conflicts).  Activations and gradients (1x128 groups
+// both ways, optionally behind a fused RMSNorm or SwiGLU producer) use a
+// 512-thread kernel; weights (128x128 blocks) and per-tensor scaling use a
+// 256-thread one.  The arithmetic per value is kept to a widening shift,
+// half a packed fp32 multiply and half a paired cvt, since at HBM rates the
+// kernels are otherwise instruction bound.
 #include <cfloat>
 #include <cuda_bf16.h>
 
@@ -286,20 +289,6 @@ cudaError_t launch_rmsnorm_apply(const uint16_t *h, int64_t rows, int64_t cols, 
     return cudaGetLastError();
 }
 
-// The thread's 8x8 block of h -> y in registers (rows from row0, columns
-// from col0; rows past the end read rstd as 0 and hold zeros anyway).
-PURO_DEV void rmsnorm_block(uint4 (&v)[8], const ProdArgs &prod, int64_t row0, int64_t col0, int64_t rows,
-                            int64_t cols) {
-    float gm[8];
-    const bool has_gamma = prod.gamma != nullptr;
-    if (has_gamma) load_gamma8(prod.gamma, col0, cols, gm);
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        const float rs = (row0 + i < rows) ? __ldg(prod.rstd + row0 + i) : 0.0f;
-        v[i] = rmsnorm_chunk(v[i], rs, gm, has_gamma);
-    }
-}
-
 // ------------------------------------------------------ SwiGLU producer
 // 2^x and 1/x by the special-function unit (PTX ex2.approx / rcp.approx:
 // relative error around 2^-22; subnormal results flush to zero).
@@ -370,17 +359,6 @@ cudaError_t launch_swiglu_apply(const uint16_t *gate, const uint16_t *up, int64_
     return cudaGetLastError();
 }
 
-// The thread's 8x8 block of the up projection for a tile (rows and columns
-// are whole tiles: the SwiGLU entry point requires multiples of 128).  Each
-// row's 16 bytes are one of 16 consecutive chunks a half-warp reads together.
-PURO_DEV void load_up_block(uint4 (&u)[8], const ProdArgs &prod, int tile, int tiles_n, int br, int bc) {
-    const int64_t row0 = static_cast<int64_t>(tile / tiles_n) * 128 + 8 * br;
-    const int64_t col0 = static_cast<int64_t>(tile % tiles_n) * 128 + 8 * bc;
-    const uint16_t *p = prod.up + row0 * prod.ld + col0;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) u[i] = __ldg(reinterpret_cast<const uint4 *>(p + i * prod.ld));
-}
-
 // ------------------------------------------------------ cast kernel
 constexpr int kQT = 128;          // tile edge
 constexpr int kQThreads = 256;
@@ -391,15 +369,9 @@ constexpr int kQThreads = 256;
 struct QuantSmem {
     alignas(1024) uint8_t q_stage[kQT * kQT];    // rowwise codes, plain rows
     alignas(1024) uint8_t qt_stage[kQT * kQT];   // transposed codes, 128B-swizzled rows
-    alignas(128) uint16_t in[2][kQT * kQT];                // bf16 tile, double buffered
-    uint32_t row_part[kQT / 2][16];   // [row pair][column block]: 16-bit row maxima, two rows per word
-    uint32_t col_part[16][kQT / 2];   // [row block][column pair]: 16-bit column maxima, two columns per word
-    alignas(16) float row_mul[kQT];   // 2^(127-g) per row (NaN marks a non-finite group)
-    alignas(16) float col_mul[kQT];   // 2^(127-g) per column
-    uint32_t red[8];
-    alignas(16) uint8_t row_g[kQT];
-    alignas(16) uint8_t col_g[kQT];
-    uint64_t full[2];                 // TMA tile loads into in[0], in[1]
+    alignas(128) uint16_t in[2][kQT * kQT];      // bf16 tile, double buffered
+    uint32_t red[8];                             // weight kind: per-warp block maxima
+    uint64_t full[2];                            // TMA tile loads into in[0], in[1]
 };
 
 constexpr uint64_t kQuantWaitNs = 2000000000ull;  // a TMA load always lands long before this
@@ -407,29 +379,20 @@ constexpr uint64_t kQuantWaitNs = 2000000000ull;  // a TMA load always lands lon
 // 2^(127-g) for a scale exponent, NaN for the non-finite marker 0xFF.
 PURO_DEV float mul_of(uint32_t g) { return g == 0xFFu ? __uint_as_float(0x7FC00000u) : pow2_inv_scale(g); }
 
-// Tile kernel: each thread owns one 8x8 block of the 128x128 tile (rows
-// 8*br .. 8*br+7, columns 8*bc .. 8*bc+7; a warp holds two block rows of 16
-// blocks).  It loads the block once and produces both its rowwise codes
-// (q) and its transposed codes (q_t) from the same registers:
-//   A  partial maxima of its 8 rows and 8 columns -> shared memory
-//   B  128 threads finish the 128 row scales and 128 column scales
-//   C  every thread quantises its block twice (row scales, column scales)
-// PROD = kProdRmsNorm: the tile holds h, and the kernel quantises the
-// RMSNorm output y = bf16((h * rstd[row]) * gamma[col]) (fp32 products,
-// gamma optional), which it forms in place in shared memory before phase A;
-// with prod.write_y it also stores y through tm_y.  Activation kind only.
-// PROD = kProdSwiGlu: the tile holds the gate g, and the kernel quantises
-// y = bf16(silu(g) * u); each thread reads its 8x8 block of the up
-// projection u straight into registers one tile ahead, so those loads are in
-// flight while the previous tile is quantised.
-template <int FMT, int KIND, bool HAS_T, int PROD>
+// Weight (128x128 blocks) and per-tensor cast kernel: one scale per tile
+// (the block's or the tensor's), so every thread owns one 8x8 block of the
+// 128x128 tile (rows 8*br .. 8*br+7, columns 8*bc .. 8*bc+7; a warp holds
+// two block rows of 16 blocks) and produces both its rowwise codes (q) and
+// its transposed codes (q_t) from the same registers.  The weight kind
+// reduces the block maximum through the warps (one barrier); the per-tensor
+// kind reads its scale from the device amax.
+template <int FMT, int KIND, bool HAS_T>
 __global__ void __launch_bounds__(kQThreads, 2)
     quant_tile_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_q,
-                      const __grid_constant__ CUtensorMap tm_qt, const __grid_constant__ CUtensorMap tm_y,
-                      int64_t rows, int64_t cols, uint8_t *__restrict__ scale_u8, uint8_t *__restrict__ scale_t_u8,
-                      float *scale_f, float *scale_t_f, const uint32_t *__restrict__ amax_bits, ProdArgs prod,
-                      int tiles_n, int ntiles) {
-    static_assert(PROD == kProdNone || KIND == kQuantBlockAct, "producers feed the activation quantiser");
+                      const __grid_constant__ CUtensorMap tm_qt, int64_t rows, int64_t cols,
+                      uint8_t *__restrict__ scale_u8, uint8_t *__restrict__ scale_t_u8, float *scale_f,
+                      float *scale_t_f, const uint32_t *__restrict__ amax_bits, int tiles_n, int ntiles) {
+    static_assert(KIND == kQuantBlockWeight || KIND == kQuantTensor, "activations use quant_act_kernel");
     extern __shared__ uint8_t smem_raw[];
     QuantSmem &sm = *reinterpret_cast<QuantSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                    ~static_cast<uintptr_t>(1023));
@@ -468,33 +431,20 @@ __global__ void __launch_bounds__(kQThreads, 2)
     };
     int tile = blockIdx.x;
     if (tid == 0 && tile < ntiles) issue_load(tile, 0);
-    uint4 un[8];  // kProdSwiGlu: this thread's block of u for the current tile
-    if constexpr (PROD == kProdSwiGlu) {
-        if (tile < ntiles) load_up_block(un, prod, tile, tiles_n, br, bc);
-    }
     for (int it = 0; tile < ntiles; ++it, tile += gridDim.x) {
         const int buf = it & 1;
         const int64_t r0 = static_cast<int64_t>(tile / tiles_n) * kQT;
         const int64_t c0 = static_cast<int64_t>(tile % tiles_n) * kQT;
         if (tid == 0) {
             const int next = tile + gridDim.x;
-            // with a y output, the buffer's last reader was the y store of
-            // tile it-1: all but the newest bulk group (its code stores) done
-            if (PROD != kProdNone && prod.write_y) bulk_wait_group_read<1>();
-            if (next < ntiles) issue_load(next, buf ^ 1);  // its buffer was last read before (S2) of it-1
+            if (next < ntiles) issue_load(next, buf ^ 1);  // its buffer was last read before (S3) of it-1
             // The previous tile's TMA stores must have read the staging tiles
-            // before they are rewritten.  Per-tensor mode writes them right
-            // after (S1); the blockwise modes first spend phase A (and B) on
-            // the scales, so they wait just before the last barrier ahead of
-            // phase C and the stores' reads overlap that work.
+            // before they are rewritten: per-tensor mode writes them right
+            // after (S1); the weight kind waits just before (S2).
             if constexpr (KIND == kQuantTensor) bulk_wait_group_read0();
         }
         // Every thread waits on the tile's barrier itself, which makes the
-        // TMA-written tile visible to it.  The blockwise kinds need no CTA
-        // barrier here: the shared buffers they write before (S2) were last
-        // read before (S4) of the previous tile.  Per-tensor mode writes the
-        // staging tiles right away, so it waits (S1) for thread 0 to have
-        // seen the previous stores read them.
+        // TMA-written tile visible to it.
         mbar_wait_bounded(&sm.full[buf], static_cast<uint32_t>(it >> 1) & 1u, kQuantWaitNs);
         if constexpr (KIND == kQuantTensor) __syncthreads();  // (S1) staging free
 
@@ -503,131 +453,34 @@ __global__ void __launch_bounds__(kQThreads, 2)
         uint4 v[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) v[i] = *reinterpret_cast<const uint4 *>(in + (8 * br + i) * kQT + 8 * bc);
-        if constexpr (PROD == kProdRmsNorm) {
-            // y = bf16((h * rstd) * gamma), formed in place (each thread its
-            // own block; the y store waits for (S2)).
-            rmsnorm_block(v, prod, r0 + 8 * br, c0 + 8 * bc, rows, cols);
-#pragma unroll
-            for (int i = 0; i < 8; ++i) *reinterpret_cast<uint4 *>(sm.in[buf] + (8 * br + i) * kQT + 8 * bc) = v[i];
-            if (prod.write_y) fence_proxy_async_smem();
-        } else if constexpr (PROD == kProdSwiGlu) {
-            // y = bf16(silu(g) * u), formed in place like the RMSNorm output
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                v[i] = swiglu_chunk(v[i], un[i]);
-                *reinterpret_cast<uint4 *>(sm.in[buf] + (8 * br + i) * kQT + 8 * bc) = v[i];
-            }
-            if (prod.write_y) fence_proxy_async_smem();
-            const int next = tile + gridDim.x;
-            if (next < ntiles) load_up_block(un, prod, next, tiles_n, br, bc);
-        }
 
-        // ---- A: partial maxima
-        if constexpr (KIND == kQuantBlockAct) {
-#pragma unroll
-            for (int p = 0; p < 4; ++p) {  // row pair (2p, 2p+1) -> one word
-                const uint32_t m0 = max_abs4(v[2 * p]), m1 = max_abs4(v[2 * p + 1]);
-                const uint32_t a0 = max(m0 & 0xFFFFu, m0 >> 16), a1 = max(m1 & 0xFFFFu, m1 >> 16);
-                sm.row_part[4 * br + p][bc] = a0 | (a1 << 16);
-            }
-            uint4 cm;  // column pair k: max over the 8 rows, 16 bits per column
-            cm.x = cm.y = cm.z = cm.w = 0u;
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                cm.x = __vmaxu2(cm.x, v[i].x & 0x7FFF7FFFu);
-                cm.y = __vmaxu2(cm.y, v[i].y & 0x7FFF7FFFu);
-                cm.z = __vmaxu2(cm.z, v[i].z & 0x7FFF7FFFu);
-                cm.w = __vmaxu2(cm.w, v[i].w & 0x7FFF7FFFu);
-            }
-            *reinterpret_cast<uint4 *>(&sm.col_part[br][4 * bc]) = cm;
-        } else if constexpr (KIND == kQuantBlockWeight) {
+        // ---- the tile's scale
+        float mul = t_mul;
+        uint32_t blk_g = 0;
+        if constexpr (KIND == kQuantBlockWeight) {
             uint32_t m = 0;
 #pragma unroll
             for (int i = 0; i < 8; ++i) m = __vmaxu2(m, max_abs4(v[i]));
             m = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
             if (lane == 0) sm.red[warp] = m;
             if (tid == 0) bulk_wait_group_read0();  // staging free (see above)
+            __syncthreads();                         // (S2) block maxima written, staging free
+            m = __reduce_max_sync(0xFFFFFFFFu, sm.red[lane & 7]);
+            blk_g = e8m0_exponent<FMT>(m);
+            mul = mul_of(blk_g);
         }
-        if constexpr (KIND != kQuantTensor) __syncthreads();  // (S2) partials written
-        if constexpr (PROD != kProdNone) {
-            if (prod.write_y && tid == 0) {  // every block's y is in shared memory
-                tma_store_2d(&tm_y, sm.in[buf], static_cast<int32_t>(c0), static_cast<int32_t>(r0));
-                bulk_commit_group();
-            }
-        }
+        const uint64_t m2 = f32x2(mul, mul);
+        const bool nan_all = isnan(mul);
 
-        // ---- B: finish the scales (thread t < 128: row t; t >= 128: column t - 128)
-        if constexpr (KIND == kQuantBlockAct) {
-            if (tid < kQT) {
-                const uint4 *rp = reinterpret_cast<const uint4 *>(sm.row_part[tid >> 1]);
-                const uint4 a = rp[0], b = rp[1], c = rp[2], d = rp[3];
-                uint32_t m = __vmaxu2(__vmaxu2(__vmaxu2(a.x, a.y), __vmaxu2(a.z, a.w)),
-                                      __vmaxu2(__vmaxu2(b.x, b.y), __vmaxu2(b.z, b.w)));
-                m = __vmaxu2(m, __vmaxu2(__vmaxu2(__vmaxu2(c.x, c.y), __vmaxu2(c.z, c.w)),
-                                         __vmaxu2(__vmaxu2(d.x, d.y), __vmaxu2(d.z, d.w))));
-                const uint32_t g = e8m0_exponent<FMT>((tid & 1) ? (m >> 16) : (m & 0xFFFFu));
-                sm.row_mul[tid] = mul_of(g);
-                sm.row_g[tid] = static_cast<uint8_t>(g);
-            } else if (HAS_T) {
-                const int c = tid - kQT;
-                uint32_t m = 0;
-#pragma unroll
-                for (int b = 0; b < 16; ++b) m = __vmaxu2(m, sm.col_part[b][c >> 1]);
-                const uint32_t g = e8m0_exponent<FMT>((c & 1) ? (m >> 16) : (m & 0xFFFFu));
-                sm.col_mul[c] = mul_of(g);
-                sm.col_g[c] = static_cast<uint8_t>(g);
-            }
-            if (tid == 0) {  // staging free (see above); a y store issued after (S2) may still run
-                if (PROD != kProdNone && prod.write_y)
-                    bulk_wait_group_read<1>();
-                else
-                    bulk_wait_group_read0();
-            }
-            __syncthreads();  // (S3) scales ready, staging free
-        }
-
-        float rmul[8], cmul[8];
-        uint32_t blk_g = 0;
-        if constexpr (KIND == kQuantBlockAct) {
-            const float4 r_lo = *reinterpret_cast<const float4 *>(&sm.row_mul[8 * br]);
-            const float4 r_hi = *reinterpret_cast<const float4 *>(&sm.row_mul[8 * br + 4]);
-            rmul[0] = r_lo.x; rmul[1] = r_lo.y; rmul[2] = r_lo.z; rmul[3] = r_lo.w;
-            rmul[4] = r_hi.x; rmul[5] = r_hi.y; rmul[6] = r_hi.z; rmul[7] = r_hi.w;
-        } else {
-            float mul = t_mul;
-            if constexpr (KIND == kQuantBlockWeight) {
-                uint32_t m = sm.red[lane & 7];
-                m = __reduce_max_sync(0xFFFFFFFFu, m);
-                blk_g = e8m0_exponent<FMT>(m);
-                mul = mul_of(blk_g);
-            }
-#pragma unroll
-            for (int i = 0; i < 8; ++i) rmul[i] = cmul[i] = mul;
-        }
-
-        // ---- C: rowwise codes (row i, 8 columns) and transposed codes
-        // (column j, 8 rows) from the same block.  The block is re-read from
-        // shared memory here rather than kept live across (S2)/(S3).
-        if constexpr (KIND != kQuantTensor) {
-#pragma unroll
-            for (int i = 0; i < 8; ++i) v[i] = *reinterpret_cast<const uint4 *>(in + (8 * br + i) * kQT + 8 * bc);
-        }
+        // ---- rowwise codes (row i, 8 columns) and transposed codes (column j, 8 rows)
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
-            const uint64_t m2 = f32x2(rmul[i], rmul[i]);
-            const bool nan_row = isnan(rmul[i]);
             uint2 o;
-            o.x = quant4<FMT>(bf16_lo(v[i].x), bf16_hi(v[i].x), bf16_lo(v[i].y), bf16_hi(v[i].y), m2, nan_row);
-            o.y = quant4<FMT>(bf16_lo(v[i].z), bf16_hi(v[i].z), bf16_lo(v[i].w), bf16_hi(v[i].w), m2, nan_row);
+            o.x = quant4<FMT>(bf16_lo(v[i].x), bf16_hi(v[i].x), bf16_lo(v[i].y), bf16_hi(v[i].y), m2, nan_all);
+            o.y = quant4<FMT>(bf16_lo(v[i].z), bf16_hi(v[i].z), bf16_lo(v[i].w), bf16_hi(v[i].w), m2, nan_all);
             *reinterpret_cast<uint2 *>(sm.q_stage + (8 * br + i) * kQT + 8 * bc) = o;
         }
         if constexpr (HAS_T) {
-            if constexpr (KIND == kQuantBlockAct) {  // column scales, loaded once the row codes are out
-                const float4 c_lo = *reinterpret_cast<const float4 *>(&sm.col_mul[8 * bc]);
-                const float4 c_hi = *reinterpret_cast<const float4 *>(&sm.col_mul[8 * bc + 4]);
-                cmul[0] = c_lo.x; cmul[1] = c_lo.y; cmul[2] = c_lo.z; cmul[3] = c_lo.w;
-                cmul[4] = c_hi.x; cmul[5] = c_hi.y; cmul[6] = c_hi.z; cmul[7] = c_hi.w;
-            }
             // Column j's 8 codes (rows 8br .. 8br+7) go to transposed row
             // 8bc + j, bytes 8br .. 8br+7.  Lanes of one half-warp share br,
             // so they would all hit the same swizzled chunk if they stored
@@ -637,16 +490,14 @@ __global__ void __launch_bounds__(kQThreads, 2)
             uint2 cc[8];
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
-                const uint64_t m2 = f32x2(cmul[j], cmul[j]);
-                const bool nan_col = isnan(cmul[j]);
                 float c[8];
 #pragma unroll
                 for (int i = 0; i < 8; ++i) {
                     const uint32_t w = (j >> 1) == 0 ? v[i].x : (j >> 1) == 1 ? v[i].y : (j >> 1) == 2 ? v[i].z : v[i].w;
                     c[i] = (j & 1) ? bf16_hi(w) : bf16_lo(w);
                 }
-                cc[j].x = quant4<FMT>(c[0], c[1], c[2], c[3], m2, nan_col);
-                cc[j].y = quant4<FMT>(c[4], c[5], c[6], c[7], m2, nan_col);
+                cc[j].x = quant4<FMT>(c[0], c[1], c[2], c[3], m2, nan_all);
+                cc[j].y = quant4<FMT>(c[4], c[5], c[6], c[7], m2, nan_all);
             }
             const int rot = bc & 7;
 #pragma unroll
@@ -666,28 +517,299 @@ __global__ void __launch_bounds__(kQThreads, 2)
         }
 
         fence_proxy_async_smem();
+        __syncthreads();  // (S3) staging complete
+        if (tid == 0) {
+            tma_store_2d(&tm_q, sm.q_stage, static_cast<int32_t>(c0), static_cast<int32_t>(r0));
+            if (HAS_T) tma_store_2d(&tm_qt, sm.qt_stage, static_cast<int32_t>(r0), static_cast<int32_t>(c0));
+            bulk_commit_group();
+        }
+        if constexpr (KIND == kQuantBlockWeight) {
+            // Scale vectors in the tensor-core layout: thread i < 128 writes
+            // row i of the rowwise operand (k-block c0/128), thread 128 + i
+            // writes row i of the transposed operand (k-block r0/128); the
+            // block's exponent repeats over its 128 rows.
+            const bool col = tid >= kQT;
+            if (!col || HAS_T) {
+                const int i = tid & (kQT - 1);
+                const int64_t op_rows0 = col ? c0 : r0;
+                const int64_t kb = (col ? r0 : c0) / kQT;
+                const int64_t kblocks = (col ? rows : cols) / kQT;
+                store_scale_vec(col ? scale_t_u8 : scale_u8, op_rows0 + i, kb, kblocks, static_cast<uint8_t>(blk_g));
+            }
+        }
+    }
+    if (tid == 0) bulk_wait_group0();
+}
+
+// ------------------------------------------- activation cast kernel (512)
+// The 1x128 activation / gradient quantiser (optionally fed by a producer)
+// with 512 threads per 128x128 tile: thread t owns the 8x4 block of rows
+// 8*br .. 8*br+7 and columns 4*bc .. 4*bc+3, br = warp (0..15), bc = lane.
+// A warp thus holds eight whole rows, so a row's group maximum is one
+// warp-wide redux per row and needs no shared memory; the column maxima go
+// through shared memory as before.  Compared with 256 threads on 8x8
+// blocks, twice the warps per SM hide the latency of each phase (the
+// kernel is latency bound at two 256-thread CTAs per SM), at about half the
+// registers per thread.  Rows and columns are whole tiles (the blockwise
+// entry points require multiples of 128).
+constexpr int kQAThreads = 512;
+
+struct QuantActSmem {
+    alignas(1024) uint8_t q_stage[kQT * kQT];    // rowwise codes, plain rows
+    alignas(1024) uint8_t qt_stage[kQT * kQT];   // transposed codes, 128B-swizzled rows
+    alignas(128) uint16_t in[2][kQT * kQT];      // bf16 tile, double buffered
+    alignas(16) uint32_t col_part[16][kQT / 2];  // [row block][column pair]: 16-bit column maxima, two per word
+    alignas(16) float col_mul[kQT];
+    alignas(16) uint8_t row_g[kQT];
+    alignas(16) uint8_t col_g[kQT];
+    uint64_t full[2];
+};
+
+// y = bf16((h * rstd) * gamma) for a 4-value chunk.
+PURO_DEV uint2 rmsnorm_chunk4(uint2 w, float rs, const float (&gm)[4], bool has_gamma) {
+    uint32_t ws[2] = {w.x, w.y};
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+        float lo = __fmul_rn(__uint_as_float(ws[j] << 16), rs), hi = __fmul_rn(__uint_as_float(ws[j] & 0xFFFF0000u), rs);
+        if (has_gamma) {
+            lo = __fmul_rn(lo, gm[2 * j]);
+            hi = __fmul_rn(hi, gm[2 * j + 1]);
+        }
+        __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+        ws[j] = *reinterpret_cast<uint32_t *>(&v);
+    }
+    return make_uint2(ws[0], ws[1]);
+}
+
+// y = bf16(silu(g) * u) for a 4-value chunk.
+PURO_DEV uint2 swiglu_chunk4(uint2 g, uint2 u) {
+    const uint32_t gw[2] = {g.x, g.y}, uw[2] = {u.x, u.y};
+    uint32_t out[2];
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+        const float lo = __fmul_rn(silu_f32(__uint_as_float(gw[j] << 16)), __uint_as_float(uw[j] << 16));
+        const float hi = __fmul_rn(silu_f32(__uint_as_float(gw[j] & 0xFFFF0000u)), __uint_as_float(uw[j] & 0xFFFF0000u));
+        __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+        out[j] = *reinterpret_cast<uint32_t *>(&v);
+    }
+    return make_uint2(out[0], out[1]);
+}
+
+template <int FMT, bool HAS_T, int PROD>
+__global__ void __launch_bounds__(kQAThreads, 2)
+    quant_act_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_q,
+                     const __grid_constant__ CUtensorMap tm_qt, const __grid_constant__ CUtensorMap tm_y,
+                     int64_t rows, int64_t cols, uint8_t *__restrict__ scale_u8, uint8_t *__restrict__ scale_t_u8,
+                     ProdArgs prod, int tiles_n, int ntiles) {
+    extern __shared__ uint8_t smem_raw[];
+    QuantActSmem &sm = *reinterpret_cast<QuantActSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                         ~static_cast<uintptr_t>(1023));
+    const int tid = threadIdx.x, lane = tid & 31;
+    const int br = tid >> 5;  // block row: tile rows 8br .. 8br+7 (the warp)
+    const int bc = lane;      // block column: tile columns 4bc .. 4bc+3
+    if (tid == 0) {
+        mbar_init(&sm.full[0], 1);
+        mbar_init(&sm.full[1], 1);
+        fence_mbarrier_init();
+        tma_prefetch_desc(&tm_x);
+        tma_prefetch_desc(&tm_q);
+        if (HAS_T) tma_prefetch_desc(&tm_qt);
+    }
+    __syncthreads();
+
+    auto issue_load = [&](int t, int b) {
+        mbar_arrive_expect_tx(&sm.full[b], kQT * kQT * 2);
+        tma_load_2d(sm.in[b], &tm_x, &sm.full[b], (t % tiles_n) * kQT, (t / tiles_n) * kQT);
+    };
+    int tile = blockIdx.x;
+    if (tid == 0 && tile < ntiles) issue_load(tile, 0);
+    uint2 un[8];  // kProdSwiGlu: this thread's block of u for the current tile
+    auto load_up = [&](int t) {
+        const int64_t row0 = static_cast<int64_t>(t / tiles_n) * kQT + 8 * br;
+        const int64_t col0 = static_cast<int64_t>(t % tiles_n) * kQT + 4 * bc;
+        const uint16_t *p = prod.up + row0 * prod.ld + col0;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) un[i] = __ldg(reinterpret_cast<const uint2 *>(p + i * prod.ld));
+    };
+    if constexpr (PROD == kProdSwiGlu) {
+        if (tile < ntiles) load_up(tile);
+    }
+    for (int it = 0; tile < ntiles; ++it, tile += gridDim.x) {
+        const int buf = it & 1;
+        const int64_t r0 = static_cast<int64_t>(tile / tiles_n) * kQT;
+        const int64_t c0 = static_cast<int64_t>(tile % tiles_n) * kQT;
+        if (tid == 0) {
+            const int next = tile + gridDim.x;
+            // with a y output, the buffer's last reader was the y store of
+            // tile it-1: all but the newest bulk group (its code stores) done
+            if (PROD != kProdNone && prod.write_y) bulk_wait_group_read<1>();
+            if (next < ntiles) issue_load(next, buf ^ 1);  // its buffer was last read before (S4) of it-1
+        }
+        // Every thread waits on the tile's barrier itself (which makes the
+        // TMA-written tile visible to it); the shared buffers written before
+        // (S2) were last read before (S4) of the previous tile.
+        mbar_wait_bounded(&sm.full[buf], static_cast<uint32_t>(it >> 1) & 1u, kQuantWaitNs);
+
+        uint16_t *in = sm.in[buf];
+        uint2 v[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[i] = *reinterpret_cast<const uint2 *>(in + (8 * br + i) * kQT + 4 * bc);
+        if constexpr (PROD == kProdRmsNorm) {
+            float gm[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+            const bool has_gamma = prod.gamma != nullptr;
+            if (has_gamma) {
+                const uint2 g = __ldg(reinterpret_cast<const uint2 *>(prod.gamma + c0 + 4 * bc));
+                gm[0] = __uint_as_float(g.x << 16);
+                gm[1] = __uint_as_float(g.x & 0xFFFF0000u);
+                gm[2] = __uint_as_float(g.y << 16);
+                gm[3] = __uint_as_float(g.y & 0xFFFF0000u);
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                v[i] = rmsnorm_chunk4(v[i], __ldg(prod.rstd + r0 + 8 * br + i), gm, has_gamma);
+                *reinterpret_cast<uint2 *>(in + (8 * br + i) * kQT + 4 * bc) = v[i];
+            }
+            if (prod.write_y) fence_proxy_async_smem();
+        } else if constexpr (PROD == kProdSwiGlu) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                v[i] = swiglu_chunk4(v[i], un[i]);
+                *reinterpret_cast<uint2 *>(in + (8 * br + i) * kQT + 4 * bc) = v[i];
+            }
+            if (prod.write_y) fence_proxy_async_smem();
+            const int next = tile + gridDim.x;
+            if (next < ntiles) load_up(next);
+        }
+
+        // ---- A: row groups (a warp holds its eight rows whole) and column partials
+        float rmul[8];
+        {
+            uint32_t rmax[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const uint32_t m = __vmaxu2(v[i].x & 0x7FFF7FFFu, v[i].y & 0x7FFF7FFFu);
+                rmax[i] = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
+            }
+            // lane i < 8 derives row 8br+i's scale; every lane then takes the
+            // eight multipliers from those lanes
+            uint32_t mine = rmax[0];
+#pragma unroll
+            for (int i = 1; i < 8; ++i) mine = (lane == i) ? rmax[i] : mine;
+            const uint32_t g = e8m0_exponent<FMT>(mine);
+            const float mul = mul_of(g);
+            if (lane < 8) sm.row_g[8 * br + lane] = static_cast<uint8_t>(g);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) rmul[i] = __shfl_sync(0xFFFFFFFFu, mul, i);
+        }
+        if constexpr (HAS_T) {
+            uint2 cm = make_uint2(0u, 0u);  // columns (4bc, 4bc+1), (4bc+2, 4bc+3): max over the 8 rows
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                cm.x = __vmaxu2(cm.x, v[i].x & 0x7FFF7FFFu);
+                cm.y = __vmaxu2(cm.y, v[i].y & 0x7FFF7FFFu);
+            }
+            *reinterpret_cast<uint2 *>(&sm.col_part[br][2 * bc]) = cm;
+        }
+        __syncthreads();  // (S2) partials and row scales written
+        if constexpr (PROD != kProdNone) {
+            if (prod.write_y && tid == 0) {  // every block's y is in shared memory
+                tma_store_2d(&tm_y, sm.in[buf], static_cast<int32_t>(c0), static_cast<int32_t>(r0));
+                bulk_commit_group();
+            }
+        }
+
+        // ---- B: column scales, two threads per column (eight row blocks each)
+        if constexpr (HAS_T) {
+            if (tid < 2 * kQT) {
+                const int c = tid >> 1, h = tid & 1;
+                uint32_t m = 0;
+#pragma unroll
+                for (int b = 0; b < 8; ++b) m = __vmaxu2(m, sm.col_part[8 * h + b][c >> 1]);
+                m = __vmaxu2(m, __shfl_xor_sync(0xFFFFFFFFu, m, 1));
+                if (h == 0) {
+                    const uint32_t g = e8m0_exponent<FMT>((c & 1) ? (m >> 16) : (m & 0xFFFFu));
+                    sm.col_mul[c] = mul_of(g);
+                    sm.col_g[c] = static_cast<uint8_t>(g);
+                }
+            }
+        }
+        if (tid == 0) {  // staging free; a y store issued after (S2) may still run
+            if (PROD != kProdNone && prod.write_y)
+                bulk_wait_group_read<1>();
+            else
+                bulk_wait_group_read0();
+        }
+        __syncthreads();  // (S3) column scales ready, staging free
+
+        // ---- C: rowwise codes (row i, 4 columns) and transposed codes
+        // (column j, 8 rows) from the block, re-read from shared memory.
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[i] = *reinterpret_cast<const uint2 *>(in + (8 * br + i) * kQT + 4 * bc);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const uint64_t m2 = f32x2(rmul[i], rmul[i]);
+            const uint32_t o = quant4<FMT>(bf16_lo(v[i].x), bf16_hi(v[i].x), bf16_lo(v[i].y), bf16_hi(v[i].y), m2,
+                                           isnan(rmul[i]));
+            *reinterpret_cast<uint32_t *>(sm.q_stage + (8 * br + i) * kQT + 4 * bc) = o;  // a warp: one 128-byte row
+        }
+        if constexpr (HAS_T) {
+            const float4 cmv = *reinterpret_cast<const float4 *>(&sm.col_mul[4 * bc]);
+            const float cmul[4] = {cmv.x, cmv.y, cmv.z, cmv.w};
+            uint2 cc[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const uint64_t m2 = f32x2(cmul[j], cmul[j]);
+                const bool nan_col = isnan(cmul[j]);
+                float c[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const uint32_t w = (j >> 1) ? v[i].y : v[i].x;
+                    c[i] = (j & 1) ? bf16_hi(w) : bf16_lo(w);
+                }
+                cc[j].x = quant4<FMT>(c[0], c[1], c[2], c[3], m2, nan_col);
+                cc[j].y = quant4<FMT>(c[4], c[5], c[6], c[7], m2, nan_col);
+            }
+            // Column j's 8 codes (rows 8br .. 8br+7) go to transposed row
+            // 4bc + j, bytes 8br .. 8br+7, whose 16-byte chunk is
+            // (br / 2) ^ ((4bc + j) % 8) under the 128-byte swizzle.  All 32
+            // lanes of a warp share br, so storing the same j together would
+            // put them in two chunks; lane bc stores column (s + bc / 2) % 4 at
+            // step s, which spreads them over all eight (a rotation of cc).
+            const int rot = (bc >> 1) & 3;
+#pragma unroll
+            for (int b = 1; b < 4; b <<= 1) {  // cc[s] <- cc[(s + rot) % 4], one rotate-by-b stage per bit
+                const bool on = (rot & b) != 0;
+                uint2 t[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) t[k] = on ? cc[(k + b) & 3] : cc[k];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) cc[k] = t[k];
+            }
+#pragma unroll
+            for (int st = 0; st < 4; ++st) {
+                const int r = 4 * bc + ((st + rot) & 3);  // transposed row (tile column)
+                *reinterpret_cast<uint2 *>(sm.qt_stage + r * kQT + 16 * ((br >> 1) ^ (r & 7)) + 8 * (br & 1)) = cc[st];
+            }
+        }
+
+        fence_proxy_async_smem();
         __syncthreads();  // (S4) staging complete
         if (tid == 0) {
             tma_store_2d(&tm_q, sm.q_stage, static_cast<int32_t>(c0), static_cast<int32_t>(r0));
             if (HAS_T) tma_store_2d(&tm_qt, sm.qt_stage, static_cast<int32_t>(r0), static_cast<int32_t>(c0));
             bulk_commit_group();
         }
-        if constexpr (KIND != kQuantTensor) {
-            // Scale vectors in the tensor-core layout: thread i < 128 writes
-            // row i of the rowwise operand (k-block c0/128), thread 128 + i
-            // writes row i of the transposed operand (k-block r0/128).
+        // Scale vectors: thread i < 128 writes row i of the rowwise operand
+        // (k-block c0/128), thread 128 + i row i of the transposed operand
+        // (k-block r0/128).
+        if (tid < 2 * kQT) {
             const bool col = tid >= kQT;
             if (!col || HAS_T) {
                 const int i = tid & (kQT - 1);
-                const int64_t op_rows0 = col ? c0 : r0;       // first operand row of this tile
-                const int64_t kb = (col ? r0 : c0) / kQT;     // k-block of this tile
+                const int64_t op_rows0 = col ? c0 : r0;
+                const int64_t kb = (col ? r0 : c0) / kQT;
                 const int64_t kblocks = (col ? rows : cols) / kQT;
-                uint8_t g;
-                if constexpr (KIND == kQuantBlockAct)
-                    g = col ? sm.col_g[i] : sm.row_g[i];
-                else
-                    g = static_cast<uint8_t>(blk_g);
-                store_scale_vec(col ? scale_t_u8 : scale_u8, op_rows0 + i, kb, kblocks, g);
+                store_scale_vec(col ? scale_t_u8 : scale_u8, op_rows0 + i, kb, kblocks, col ? sm.col_g[i] : sm.row_g[i]);
             }
         }
     }
@@ -715,20 +837,37 @@ template <int FMT, int KIND, bool HAS_T, int PROD = kProdNone>
 static cudaError_t launch_quant_t(const QuantArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_q,
                                   const CUtensorMap &tm_qt, cudaStream_t s, const CUtensorMap *tm_y = nullptr,
                                   ProdArgs prod = ProdArgs{}) {
-    auto kern = quant_tile_kernel<FMT, KIND, HAS_T, PROD>;
-    const size_t smem = sizeof(QuantSmem) + 1024;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
-    if (e != cudaSuccess) return e;
-    const int tiles_m = static_cast<int>((a.rows + kQT - 1) / kQT);
-    const int tiles_n = static_cast<int>((a.cols + kQT - 1) / kQT);
-    const int ntiles = tiles_m * tiles_n;
-    int dev = 0, sms = 148;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int grid = ntiles < 2 * sms ? ntiles : 2 * sms;  // persistent: two CTAs per SM
-    kern<<<grid, kQThreads, smem, s>>>(tm_x, tm_q, tm_qt, tm_y ? *tm_y : tm_x, a.rows, a.cols, a.scale_u8,
-                                       a.scale_t_u8, a.scale_f, a.scale_t_f, a.amax, prod, tiles_n, ntiles);
-    return cudaGetLastError();
+    if constexpr (KIND == kQuantBlockAct) {  // the 512-thread activation kernel (whole tiles)
+        auto kern = quant_act_kernel<FMT, HAS_T, PROD>;
+        const size_t smem = sizeof(QuantActSmem) + 1024;
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+        const int tiles_n = static_cast<int>(a.cols / kQT);
+        const int ntiles = static_cast<int>(a.rows / kQT) * tiles_n;
+        int dev = 0, sms = 148;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        const int grid = ntiles < 2 * sms ? ntiles : 2 * sms;  // persistent: two CTAs per SM
+        kern<<<grid, kQAThreads, smem, s>>>(tm_x, tm_q, tm_qt, tm_y ? *tm_y : tm_x, a.rows, a.cols, a.scale_u8,
+                                            a.scale_t_u8, prod, tiles_n, ntiles);
+        return cudaGetLastError();
+    } else {
+        static_assert(PROD == kProdNone, "producers feed the activation quantiser");
+        auto kern = quant_tile_kernel<FMT, KIND, HAS_T>;
+        const size_t smem = sizeof(QuantSmem) + 1024;
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+        const int tiles_m = static_cast<int>((a.rows + kQT - 1) / kQT);
+        const int tiles_n = static_cast<int>((a.cols + kQT - 1) / kQT);
+        const int ntiles = tiles_m * tiles_n;
+        int dev = 0, sms = 148;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        const int grid = ntiles < 2 * sms ? ntiles : 2 * sms;  // persistent: two CTAs per SM
+        kern<<<grid, kQThreads, smem, s>>>(tm_x, tm_q, tm_qt, a.rows, a.cols, a.scale_u8, a.scale_t_u8, a.scale_f,
+                                           a.scale_t_f, a.amax, tiles_n, ntiles);
+        return cudaGetLastError();
+    }
 }
 
 template <int FMT, int KIND>

@@ -6,6 +6,7 @@ enough that a full capture ends in seconds).  Not part of the library.
     python -m paper_2608_27370_gb300.microbench.kernels rmsnorm  # [32768, 1536] with a gain
     python -m paper_2608_27370_gb300.microbench.kernels muonh    # gate_up [17920, 1536] + down [1536, 8960]
     python -m paper_2608_27370_gb300.microbench.kernels gemm     # down Fprop, M = 8192, N = 1536, K = 8960
+    python -m paper_2608_27370_gb300.microbench.kernels quant    # gate_up output gradient [8192, 17920], both copies
 
 Each input is larger than L2.  Every call is made twice: the second is the
 one to capture (ncu -s skips the first).
@@ -56,8 +57,13 @@ def main(which: str) -> None:
         d = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
         for _ in range(2):
             P.puro_fp8_linear_fprop(a.rowwise, b.rowwise, d)
+    elif which == "quant":
+        dy = W.normal_bf16((8192, 17920), 1e-3, dev, 3)
+        q = P.quantize(dy)
+        for _ in range(2):
+            P.quantize(dy, out=q)
     else:
-        raise SystemExit(f"unknown kernel {which!r}: swiglu, rmsnorm, muonh or gemm")
+        raise SystemExit(f"unknown kernel {which!r}: swiglu, rmsnorm, muonh, gemm or quant")
     torch.cuda.synchronize()
     print("ok", which)
 
