@@ -92,7 +92,7 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-bf16", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
-    ap.add_argument("--no-paper-model", action="store_true", help="skip the C6 (paper model shape), E5M2-gradient, producer-fusion and MuonH lines")
+    ap.add_argument("--no-paper-model", action="store_true", help="skip the C6 (paper model shape), E5M2-gradient, per-tensor, producer-fusion and MuonH lines")
     return ap.parse_args()
 
 
@@ -573,6 +573,25 @@ def grad_format_measure(P, torch, stack, steps=3, warmup=2):
             "quantize_gbs": q["units"] / q["time_s"] / 1e9}
 
 
+def tensor_scaling_measure(P, W, torch, device, layers=4, steps=3, warmup=2):
+    """The C5 step with per-tensor current scaling (the contrast the FP8
+    section draws: one scale per tensor, from an amax pass) on `layers` of
+    its 28 layers: amax, per-tensor quantise (both copies), and the three
+    FP8 GEMMs with the scale_inv product applied in the epilogue."""
+    wl = W.WORKLOADS["C5"]
+    stack = LinearStack(P, W, torch, wl, device, "tensor", layers, wl.M)
+    step_s, per = timed_steps(torch, stack, steps, warmup)
+    g, q = per["gemm"], per["quantize"]
+    out = {"workload": f"C5 with per-tensor scaling, {layers} of its 28 layers, M={wl.M}",
+           "value": stack.flops_per_step() / step_s / 1e12, "unit": "TFLOP/s", "ms_per_step": step_s * 1e3,
+           "steps": steps, "warmup": warmup, "gemm_only_tflops": g["units"] / g["time_s"] / 1e12,
+           "quantize_gbs": q["units"] / q["time_s"] / 1e9,
+           "amax_gbs": per["amax"]["units"] / per["amax"]["time_s"] / 1e9 if "amax" in per else None}
+    del stack
+    torch.cuda.empty_cache()
+    return out
+
+
 def paper_model_measure(P, W, torch, device, scaling, steps=5, warmup=3):
     """The same step on the paper's own production model shape: C6, the
     28-layer Qwen3-1.7B linear stack at its training micro-batch (2 x 4096
@@ -882,6 +901,8 @@ def main():
         result["rmsnorm_quantize_fusion"] = rmsnorm_fusion_measure(P, W, torch, device)
         result["swiglu_quantize_fusion"] = swiglu_fusion_measure(P, W, torch, device)
         result["muonh_step"] = muonh_measure(P, W, torch, device, peaks)
+        if args.scaling == "block":
+            result["tensor_scaling"] = tensor_scaling_measure(P, W, torch, device)
     if rank == 0:
         print(json.dumps(result), flush=True)
     if world > 1:
