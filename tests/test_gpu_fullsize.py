@@ -82,3 +82,58 @@ def test_c5_layers(layer, idx):
 def test_c6_paper_model_layers(layer, idx):
     """The paper's own model shape (Qwen3-1.7B linears, M = 8192)."""
     _sampled("C6", layer, idx, 600 + 4 * layer + idx)
+
+
+def test_c5_rmsnorm_quantize_full_size():
+    """The fused RMSNorm -> quantise on the C5 qkv/gate_up input [32768, 1536]
+    (with a gain), sampled: rstd of sampled rows within its bound, y and the
+    codes bit-exact given the kernel's rstd on sampled rows and columns."""
+    import oracle as O
+    from _parity import bits, sample_index
+
+    M, K = 32768, 1536
+    h = (W.student_t3_f32((M, K), DEV, 5100) * 4.0).to(torch.bfloat16)
+    gamma = W.normal_f32((K,), 0.1, DEV, 5101).add_(1.0).to(torch.bfloat16)
+    rstd = torch.empty(M, dtype=torch.float32, device=DEV)
+    y = torch.empty((M, K), dtype=torch.bfloat16, device=DEV)
+    q = P.quantize(torch.empty((M, K), dtype=torch.bfloat16, device=DEV))
+    P.puro_fp8_quantize_rmsnorm(h, gamma, 1e-6, P.E4M3, rstd, y, q.rowwise.data, q.rowwise.scale, q.colwise.data,
+                                q.colwise.scale)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(5102)
+    rows = torch.from_numpy(sample_index(M, 256, rng)).to(DEV)
+    cols = torch.from_numpy(sample_index(K, 64, rng)).to(DEV)
+    ref = O.rmsnorm_rstd(bits(h[rows]), 1e-6)
+    rel = np.abs(rstd[rows].double().cpu().numpy() - ref) / ref
+    assert float(rel.max()) <= (K / 64 + 8) * 2.0 ** -24
+    y_ref = O.rmsnorm_apply_f32(bits(h[rows]), rstd[rows].cpu().numpy(), bits(gamma))
+    assert np.array_equal(bits(y[rows]), y_ref), "normalised y differs on sampled rows"
+    check_block_act_quant(y, q, P.E4M3, rows=rows, cols=cols)
+
+
+def test_c5_swiglu_quantize_full_size():
+    """The fused SwiGLU -> quantise on the C5 down input [32768, 8960] from the
+    gate/up output [32768, 17920], sampled: h within one bf16 ulp of the
+    oracle on sampled rows, the codes bit-exact given the kernel's h."""
+    import oracle as O
+    from _parity import bits, sample_index
+
+    M, F = 32768, 8960
+    gu = (W.student_t3_f32((M, 2 * F), DEV, 5200) * 3.0).to(torch.bfloat16)
+    h = torch.empty((M, F), dtype=torch.bfloat16, device=DEV)
+    q = P.quantize(torch.empty((M, F), dtype=torch.bfloat16, device=DEV))
+    P.puro_fp8_quantize_swiglu(gu[:, :F], gu[:, F:], P.E4M3, h, q.rowwise.data, q.rowwise.scale, q.colwise.data,
+                               q.colwise.scale)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(5201)
+    rows = torch.from_numpy(sample_index(M, 256, rng)).to(DEV)
+    cols = torch.from_numpy(sample_index(F, 64, rng)).to(DEV)
+    g_rows = gu[rows]
+    ref = O.swiglu(bits(g_rows[:, :F]), bits(g_rows[:, F:]))
+    got = bits(h[rows])
+    rv = torch.from_numpy(ref.view(np.int16)).view(torch.bfloat16).double().numpy()
+    gv = torch.from_numpy(got.view(np.int16)).view(torch.bfloat16).double().numpy()
+    ulp = np.exp2(np.floor(np.log2(np.maximum(np.abs(rv), 2.0 ** -126))) - 7)
+    assert float((np.abs(gv - rv) / ulp).max()) <= 1.0
+    assert np.count_nonzero(got != ref) / got.size <= 1e-3
+    check_block_act_quant(h, q, P.E4M3, rows=rows, cols=cols)
