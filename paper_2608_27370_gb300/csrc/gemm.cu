@@ -250,6 +250,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     __syncthreads();
     cluster_sync();  // both CTAs' barriers exist before any copy or arrival targets them
     tc_fence_after_sync();
+    pdl_wait();  // the set-up above overlaps the previous kernel's tail
+    pdl_launch_dependents();
     const uint32_t tmem = sm.tmem_base;
 
     if (warp == 0) {
@@ -577,6 +579,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 // (chunk s starts split_stride4 float4s after chunk s-1).
 __global__ void __launch_bounds__(256) splitk_reduce_kernel(const float4 *__restrict__ ws, int splits, int64_t n4,
                                                             int64_t split_stride4, uint2 *__restrict__ out) {
+    pdl_wait();
+    pdl_launch_dependents();
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
     for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
         float4 a = ws[i];
@@ -597,6 +601,8 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const float4 *__rest
 __global__ void __launch_bounds__(256) splitk_reduce_add_f32_kernel(const float4 *__restrict__ ws, int splits,
                                                                     int64_t n4, int64_t split_stride4,
                                                                     float4 *__restrict__ out) {
+    pdl_wait();
+    pdl_launch_dependents();
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
     for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
         float4 a = ws[i];
@@ -732,8 +738,8 @@ static cudaError_t launch_kind(const GemmArgs &g, const GemmMaps &m, int splits,
     if (e != cudaSuccess) return e;
     const int pairs_max = max_resident_pairs<KIND, OUT, BN>(g.num_sms, smem);
     const int pairs = p.num_units < pairs_max ? p.num_units : pairs_max;
-    kern<<<2 * pairs, kThreads, smem, s>>>(m.a, m.b, OUT == kGemmOutF32Partial ? m.ws : m.d, m.sfa, m.sfb, p);
-    return cudaGetLastError();
+    return launch_pdl(kern, dim3(2 * pairs), dim3(kThreads), smem, s, m.a, m.b,
+                      OUT == kGemmOutF32Partial ? m.ws : m.d, m.sfa, m.sfb, p);
 }
 
 template <int KIND>
@@ -751,13 +757,12 @@ static cudaError_t launch_split_or_not(const GemmArgs &g, const GemmMaps &m, cud
     int64_t want = (n4 + 255) / 256;
     const int64_t cap = static_cast<int64_t>(g.num_sms) * 8;
     const int grid = static_cast<int>(want < cap ? want : cap);
+    const float4 *ws = reinterpret_cast<const float4 *>(g.workspace);
     if (g.accumulate_f32)
-        splitk_reduce_add_f32_kernel<<<grid, 256, 0, s>>>(reinterpret_cast<const float4 *>(g.workspace), g.splits, n4,
-                                                          stride4, reinterpret_cast<float4 *>(g.out));
-    else
-        splitk_reduce_kernel<<<grid, 256, 0, s>>>(reinterpret_cast<const float4 *>(g.workspace), g.splits, n4, stride4,
-                                                  reinterpret_cast<uint2 *>(g.out));
-    return cudaGetLastError();
+        return launch_pdl(splitk_reduce_add_f32_kernel, dim3(grid), dim3(256), 0, s, ws, g.splits, n4, stride4,
+                          reinterpret_cast<float4 *>(g.out));
+    return launch_pdl(splitk_reduce_kernel, dim3(grid), dim3(256), 0, s, ws, g.splits, n4, stride4,
+                      reinterpret_cast<uint2 *>(g.out));
 }
 
 cudaError_t launch_gemm(const GemmArgs &g, const GemmMaps &m, cudaStream_t s) {

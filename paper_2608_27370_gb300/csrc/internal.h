@@ -11,6 +11,25 @@
 
 namespace puro {
 
+// Launch `kern` on `s` with programmatic stream serialisation (the kernel
+// calls pdl_wait() before touching global memory; see ptx.cuh).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr.val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<Args &&>(args)...);
+}
+
+
 // How a quantiser groups values (section "FP8 Mixed-Precision Training").
 enum QuantKind : int {
     kQuantBlockAct = 0,     // 1x128 groups along cols (q) and along rows (q_t)

@@ -27,6 +27,7 @@
 #include <cmath>
 
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace puro {
 namespace {
@@ -79,6 +80,8 @@ __device__ __forceinline__ int matrix_of(const MuonhGroup &g, int b) {
 
 // Per-CTA partial sums {S_ww, S_wu, S_uu} of one chunk.
 __global__ void __launch_bounds__(kMuonhThreads) muonh_reduce_kernel(const __grid_constant__ MuonhGroup g) {
+    pdl_wait();
+    pdl_launch_dependents();
     const int b = blockIdx.x;
     const int m = matrix_of(g, b);
     const int64_t c4 = g.chunk4[m];
@@ -129,6 +132,8 @@ __global__ void __launch_bounds__(kMuonhThreads) muonh_reduce_kernel(const __gri
 // sums[m][k] = the matrix's chunk partials of sum k, in index order (CTA m,
 // warp k: lane-strided fp64 sums, then the butterfly).
 __global__ void __launch_bounds__(96) muonh_finalize_kernel(const __grid_constant__ MuonhGroup g) {
+    pdl_wait();
+    pdl_launch_dependents();
     const int m = blockIdx.x, k = threadIdx.x >> 5, lane = threadIdx.x & 31;
     double s = 0.0;
     for (int b = g.block_start[m] + lane; b < g.block_start[m + 1]; b += 32) s += g.partials[k * g.total_blocks + b];
@@ -139,6 +144,8 @@ __global__ void __launch_bounds__(96) muonh_finalize_kernel(const __grid_constan
 // W <- s (W - c u) on one chunk, c and s from the matrix's sums (fp64, once
 // per CTA).
 __global__ void __launch_bounds__(kMuonhThreads) muonh_apply_kernel(const __grid_constant__ MuonhGroup g) {
+    pdl_wait();
+    pdl_launch_dependents();
     const int b = blockIdx.x;
     const int m = matrix_of(g, b);
     __shared__ float cs[2];
@@ -204,17 +211,12 @@ enum MuonhPass { kReduce = 1, kApply = 2 };
 cudaError_t run_group(const MuonhGroup &g, int passes, cudaStream_t s) {
     if (g.count == 0) return cudaSuccess;
     if (passes & kReduce) {
-        muonh_reduce_kernel<<<g.total_blocks, kMuonhThreads, 0, s>>>(g);
-        cudaError_t e = cudaGetLastError();
+        cudaError_t e = launch_pdl(muonh_reduce_kernel, dim3(g.total_blocks), dim3(kMuonhThreads), 0, s, g);
         if (e != cudaSuccess) return e;
-        muonh_finalize_kernel<<<g.count, 96, 0, s>>>(g);
-        e = cudaGetLastError();
+        e = launch_pdl(muonh_finalize_kernel, dim3(g.count), dim3(96), 0, s, g);
         if (e != cudaSuccess) return e;
     }
-    if (passes & kApply) {
-        muonh_apply_kernel<<<g.total_blocks, kMuonhThreads, 0, s>>>(g);
-        return cudaGetLastError();
-    }
+    if (passes & kApply) return launch_pdl(muonh_apply_kernel, dim3(g.total_blocks), dim3(kMuonhThreads), 0, s, g);
     return cudaSuccess;
 }
 

@@ -27,6 +27,16 @@ PURO_DEV uint64_t global_timer_ns() {
     return t;
 }
 
+// --------------------------------------------- programmatic dependent launch
+// Kernels are launched with programmatic stream serialisation: a kernel may
+// start (and run its prologue: barrier set-up, tensor-memory allocation,
+// descriptor prefetch) while the previous kernel on the stream finishes.
+// pdl_wait() blocks until the previous kernels have completed and their
+// memory is visible; every kernel calls it before its first global-memory
+// access, then pdl_launch_dependents() lets the next kernel start launching.
+PURO_DEV void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+PURO_DEV void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // ---------------------------------------------------------------- mbarrier
 PURO_DEV void mbar_init(uint64_t *bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");

@@ -29,6 +29,8 @@ namespace puro {
 __global__ void __launch_bounds__(256) amax_kernel(const uint4 *__restrict__ x, int64_t nvec,
                                                    const uint16_t *__restrict__ tail, int ntail,
                                                    uint32_t *__restrict__ out) {
+    pdl_wait();
+    pdl_launch_dependents();
     uint32_t m2 = 0;  // two packed 16-bit running maxima
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
     int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
@@ -74,8 +76,8 @@ cudaError_t launch_amax(const uint16_t *x, int64_t n, uint32_t *amax, cudaStream
     int64_t want = (nvec + 255) / 256;
     int64_t cap = static_cast<int64_t>(sms) * 8;
     int grid = static_cast<int>(want < cap ? (want > 0 ? want : 1) : cap);
-    amax_kernel<<<grid, 256, 0, s>>>(reinterpret_cast<const uint4 *>(x), nvec, x + nvec * 8, ntail, amax);
-    return cudaGetLastError();
+    return launch_pdl(amax_kernel, dim3(grid), dim3(256), 0, s, reinterpret_cast<const uint4 *>(x), nvec,
+                      x + nvec * 8, ntail, amax);
 }
 
 // ------------------------------------------------------ scale helpers
@@ -186,6 +188,8 @@ PURO_DEV void store_scale_vec(uint8_t *__restrict__ base, int64_t row, int64_t k
 // row's loads are in flight together.
 __global__ void __launch_bounds__(256) rmsnorm_rstd_kernel(const uint16_t *__restrict__ h, int64_t rows, int64_t cols,
                                                            float eps, float *__restrict__ rstd) {
+    pdl_wait();
+    pdl_launch_dependents();
     constexpr int kBatch = 8;
     const int lane = threadIdx.x & 31;
     const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
@@ -253,6 +257,8 @@ PURO_DEV void load_gamma8(const uint16_t *gamma, int64_t c, int64_t cols, float 
 __global__ void __launch_bounds__(256) rmsnorm_apply_kernel(const uint16_t *__restrict__ h, int64_t rows, int64_t cols,
                                                             const float *__restrict__ rstd,
                                                             const uint16_t *__restrict__ gamma, uint16_t *__restrict__ y) {
+    pdl_wait();
+    pdl_launch_dependents();
     const int64_t per_row = cols / 8;
     const int64_t chunks = rows * per_row;
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -276,8 +282,7 @@ cudaError_t launch_rmsnorm_rstd(const uint16_t *h, int64_t rows, int64_t cols, f
     const int sms = sm_count_here();
     const int64_t want = (rows + 7) / 8;
     const int grid = static_cast<int>(want < 8 * sms ? want : 8 * sms);
-    rmsnorm_rstd_kernel<<<grid > 0 ? grid : 1, 256, 0, s>>>(h, rows, cols, eps, rstd);
-    return cudaGetLastError();
+    return launch_pdl(rmsnorm_rstd_kernel, dim3(grid > 0 ? grid : 1), dim3(256), 0, s, h, rows, cols, eps, rstd);
 }
 
 cudaError_t launch_rmsnorm_apply(const uint16_t *h, int64_t rows, int64_t cols, const float *rstd,
@@ -285,8 +290,7 @@ cudaError_t launch_rmsnorm_apply(const uint16_t *h, int64_t rows, int64_t cols, 
     const int sms = sm_count_here();
     const int64_t want = (rows * (cols / 8) + 255) / 256;
     const int grid = static_cast<int>(want < 8 * sms ? want : 8 * sms);
-    rmsnorm_apply_kernel<<<grid > 0 ? grid : 1, 256, 0, s>>>(h, rows, cols, rstd, gamma, y);
-    return cudaGetLastError();
+    return launch_pdl(rmsnorm_apply_kernel, dim3(grid > 0 ? grid : 1), dim3(256), 0, s, h, rows, cols, rstd, gamma, y);
 }
 
 // ------------------------------------------------------ SwiGLU producer
@@ -339,6 +343,8 @@ PURO_DEV uint4 swiglu_chunk(uint4 g, uint4 u) {
 __global__ void __launch_bounds__(256) swiglu_apply_kernel(const uint16_t *__restrict__ gate,
                                                            const uint16_t *__restrict__ up, int64_t rows,
                                                            int64_t cols, int64_t ld, uint16_t *__restrict__ y) {
+    pdl_wait();
+    pdl_launch_dependents();
     const int64_t per_row = cols / 8;
     const int64_t chunks = rows * per_row;
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -355,8 +361,7 @@ cudaError_t launch_swiglu_apply(const uint16_t *gate, const uint16_t *up, int64_
     const int sms = sm_count_here();
     const int64_t want = (rows * (cols / 8) + 255) / 256;
     const int grid = static_cast<int>(want < 8 * sms ? want : 8 * sms);
-    swiglu_apply_kernel<<<grid > 0 ? grid : 1, 256, 0, s>>>(gate, up, rows, cols, ld, y);
-    return cudaGetLastError();
+    return launch_pdl(swiglu_apply_kernel, dim3(grid > 0 ? grid : 1), dim3(256), 0, s, gate, up, rows, cols, ld, y);
 }
 
 // ------------------------------------------------------ cast kernel
@@ -399,6 +404,8 @@ __global__ void __launch_bounds__(kQThreads, 2)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int br = 2 * warp + (lane >> 4);  // block row: tile rows 8br .. 8br+7
     const int bc = lane & 15;               // block column: tile columns 8bc .. 8bc+7
+    pdl_wait();
+    pdl_launch_dependents();
 
     // Per-tensor mode: the one scale, from the device amax.
     float t_mul = 1.0f;
@@ -616,6 +623,8 @@ __global__ void __launch_bounds__(kQAThreads, 2)
         if (HAS_T) tma_prefetch_desc(&tm_qt);
     }
     __syncthreads();
+    pdl_wait();
+    pdl_launch_dependents();
 
     auto issue_load = [&](int t, int b) {
         mbar_arrive_expect_tx(&sm.full[b], kQT * kQT * 2);
@@ -819,6 +828,8 @@ __global__ void __launch_bounds__(kQAThreads, 2)
 // Per-tensor scale only (empty tensors: amax = 0 gives scale_inv = 1).
 template <int FMT>
 __global__ void tensor_scale_only_kernel(const uint32_t *amax_bits, float *scale_f, float *scale_t_f) {
+    pdl_wait();
+    pdl_launch_dependents();
     const uint32_t a = *amax_bits & 0xFFFFu;
     const float si = (a >= 0x7F80u) ? __uint_as_float(0x7FC00000u) : __fdiv_rn(1.0f, tensor_scale<FMT>(a));
     *scale_f = si;
@@ -826,11 +837,8 @@ __global__ void tensor_scale_only_kernel(const uint32_t *amax_bits, float *scale
 }
 
 cudaError_t launch_tensor_scale_only(const QuantArgs &a, cudaStream_t s) {
-    if (a.fmt == 0)
-        tensor_scale_only_kernel<0><<<1, 1, 0, s>>>(a.amax, a.scale_f, a.scale_t_f);
-    else
-        tensor_scale_only_kernel<1><<<1, 1, 0, s>>>(a.amax, a.scale_f, a.scale_t_f);
-    return cudaGetLastError();
+    return launch_pdl(a.fmt == 0 ? tensor_scale_only_kernel<0> : tensor_scale_only_kernel<1>, dim3(1), dim3(1), 0, s,
+                      a.amax, a.scale_f, a.scale_t_f);
 }
 
 template <int FMT, int KIND, bool HAS_T, int PROD = kProdNone>
@@ -848,9 +856,8 @@ static cudaError_t launch_quant_t(const QuantArgs &a, const CUtensorMap &tm_x, c
         cudaGetDevice(&dev);
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
         const int grid = ntiles < 2 * sms ? ntiles : 2 * sms;  // persistent: two CTAs per SM
-        kern<<<grid, kQAThreads, smem, s>>>(tm_x, tm_q, tm_qt, tm_y ? *tm_y : tm_x, a.rows, a.cols, a.scale_u8,
-                                            a.scale_t_u8, prod, tiles_n, ntiles);
-        return cudaGetLastError();
+        return launch_pdl(kern, dim3(grid), dim3(kQAThreads), smem, s, tm_x, tm_q, tm_qt, tm_y ? *tm_y : tm_x, a.rows,
+                          a.cols, a.scale_u8, a.scale_t_u8, prod, tiles_n, ntiles);
     } else {
         static_assert(PROD == kProdNone, "producers feed the activation quantiser");
         auto kern = quant_tile_kernel<FMT, KIND, HAS_T>;
@@ -864,9 +871,8 @@ static cudaError_t launch_quant_t(const QuantArgs &a, const CUtensorMap &tm_x, c
         cudaGetDevice(&dev);
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
         const int grid = ntiles < 2 * sms ? ntiles : 2 * sms;  // persistent: two CTAs per SM
-        kern<<<grid, kQThreads, smem, s>>>(tm_x, tm_q, tm_qt, a.rows, a.cols, a.scale_u8, a.scale_t_u8, a.scale_f,
-                                           a.scale_t_f, a.amax, tiles_n, ntiles);
-        return cudaGetLastError();
+        return launch_pdl(kern, dim3(grid), dim3(kQThreads), smem, s, tm_x, tm_q, tm_qt, a.rows, a.cols, a.scale_u8,
+                          a.scale_t_u8, a.scale_f, a.scale_t_f, a.amax, tiles_n, ntiles);
     }
 }
 
