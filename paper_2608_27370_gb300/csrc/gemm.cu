@@ -511,7 +511,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 }
                 tc_fence_before_sync();
                 __syncwarp();
-                if (lane == 0) mbar_arrive_cluster(tempty0 + 8u * buf);
+                if (lane == 0) mbar_arrive_cluster_cta_scope(tempty0 + 8u * buf);
             } else {
                 // BF16 tile in two halves of 128 columns (BN = 224: 128 + 96).
                 // Shifted (block kind, BN = 256): the half in the columns the
@@ -537,7 +537,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     if (hh == kReleaseAt) {
                         tc_fence_before_sync();
                         __syncwarp();
-                        if (lane == 0) mbar_arrive_cluster(tempty0 + 8u * buf);  // accumulator free for the next tile
+                        if (lane == 0) mbar_arrive_cluster_cta_scope(tempty0 + 8u * buf);  // accumulator free for the next tile
                     }
 #pragma unroll
                     for (int c = 0; c < 4; ++c) {
@@ -650,18 +650,19 @@ int choose_splits(int64_t M, int64_t N, int64_t K, bool bf16) {
 
 // Tile width of an unsplit block-scaled GEMM.  Modelled pair time = waves x
 // per-tile cycles, with constants fitted to measured GB300 times of both
-// forms: about 163 cycles per pair MMA plus a 2500-cycle accumulator hand-off
-// per tile for the 256-wide form, 170 cycles per MMA plus 350 per tile for
-// the 224-wide one.  The narrower form has more tiles, so it pays off only
-// where the hand-off dominates (short reductions) and the extra tiles do not
-// add a wave; it is taken only for a modelled gain above 5.5%, the margin the
-// fit needed to match every measured shape.
+// forms over the C5 and C6 linear shapes: about 163 cycles per pair MMA plus
+// a 600-cycle accumulator hand-off per tile for the 256-wide form, 176 cycles
+// per MMA plus 350 per tile for the 224-wide one (its helpers' scale images
+// slow the issue).  The narrower form has more tiles, so it pays off only
+// where the 256-wide tiles leave a much worse last wave; it is taken only for
+// a modelled gain above 5.5%.  (With the hand-off at 600 cycles the 256-wide
+// form measured faster on every shape of both models.)
 int choose_tile_n(int64_t M, int64_t N, int64_t K) {
     const int64_t stages = (K + kBKBytes - 1) / kBKBytes;
     const int64_t m_tiles = (M + kPairM - 1) / kPairM;
     auto waves = [&](int64_t bn) { return (m_tiles * ((N + bn - 1) / bn) + kSplitRefPairs - 1) / kSplitRefPairs; };
-    const int64_t c256 = waves(256) * (stages * kAtoms * 4 * 163 + 2500);
-    const int64_t c224 = waves(224) * (stages * kAtoms * 4 * 170 + 350);
+    const int64_t c256 = waves(256) * (stages * kAtoms * 4 * 163 + 600);
+    const int64_t c224 = waves(224) * (stages * kAtoms * 4 * 176 + 350);
     return c224 * 1000 < c256 * 945 ? 224 : 256;
 }
 

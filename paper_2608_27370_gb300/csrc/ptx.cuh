@@ -183,6 +183,17 @@ PURO_DEV void mbar_arrive_cluster(uint32_t bar_cluster) {
     asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
 }
 
+// The same arrive with release semantics at CTA scope only (the default of
+// mbarrier.arrive).  For a signal that publishes no generic memory -- an
+// epilogue telling the MMA thread that its tcgen05.ld reads of an
+// accumulator are done, ordered by tcgen05.wait::ld and the tcgen05 fences
+// around the barrier -- this is enough, and it does not wait, as the
+// cluster-scope release does, for the thread's earlier memory operations
+// (measured: about 1,500 cycles per arrive behind the epilogue's stores).
+PURO_DEV void mbar_arrive_cluster_cta_scope(uint32_t bar_cluster) {
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+}
+
 // 2-D tiled load into this CTA's shared memory whose completion is counted
 // on an mbarrier that may live in the peer CTA of the pair.
 PURO_DEV void tma_load_2d_pair(void *dst, const CUtensorMap *map, uint32_t bar_cluster, int32_t x, int32_t y) {
