@@ -6,6 +6,7 @@ enough that a full capture ends in seconds).  Not part of the library.
     python -m paper_2608_27370_gb300.microbench.kernels rmsnorm  # [32768, 1536] with a gain
     python -m paper_2608_27370_gb300.microbench.kernels muonh    # gate_up [17920, 1536] + down [1536, 8960]
     python -m paper_2608_27370_gb300.microbench.kernels gemm     # down Fprop, M = 8192, N = 1536, K = 8960
+    python -m paper_2608_27370_gb300.microbench.kernels gemm_k1536  # gate_up Fprop, M = 8192, N = 17920, K = 1536
     python -m paper_2608_27370_gb300.microbench.kernels quant    # gate_up output gradient [8192, 17920], both copies
 
 Each input is larger than L2.  Every call is made twice: the second is the
@@ -50,8 +51,8 @@ def main(which: str) -> None:
         ws = torch.empty(P.puro_muonh_grouped_workspace_size(mats), dtype=torch.uint8, device=dev)
         for _ in range(2):
             P.puro_muonh_step_grouped(mats, 4.08e-4, sums, ws)
-    elif which == "gemm":
-        M, N, K = 8192, 1536, 8960
+    elif which in ("gemm", "gemm_k1536"):
+        M, N, K = (8192, 1536, 8960) if which == "gemm" else (8192, 17920, 1536)
         a = P.quantize(W.normal_bf16((M, K), 1.0, dev, 1), transpose=False)
         b = P.quantize(W.normal_bf16((N, K), 0.02, dev, 2), P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT, transpose=False)
         d = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
@@ -63,7 +64,7 @@ def main(which: str) -> None:
         for _ in range(2):
             P.quantize(dy, out=q)
     else:
-        raise SystemExit(f"unknown kernel {which!r}: swiglu, rmsnorm, muonh, gemm or quant")
+        raise SystemExit(f"unknown kernel {which!r}: swiglu, rmsnorm, muonh, gemm, gemm_k1536 or quant")
     torch.cuda.synchronize()
     print("ok", which)
 
