@@ -92,7 +92,7 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-bf16", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
-    ap.add_argument("--no-paper-model", action="store_true", help="skip the C6 (paper model shape), E5M2-gradient, per-tensor, producer-fusion and MuonH lines")
+    ap.add_argument("--no-paper-model", action="store_true", help="skip the C6 (paper model shape), E5M2-gradient, per-tensor, producer/epilogue-fusion and MuonH lines")
     return ap.parse_args()
 
 
@@ -490,6 +490,68 @@ def swiglu_fusion_measure(P, W, torch, device):
                     "fused_us": tf * 1e6, "unfused_us": tu * 1e6, "fused_over_unfused_time": tf / tu,
                     "fused_algorithmic_gbs": fused_bytes / tf / 1e9})
         del gus, h, q
+        torch.cuda.empty_cache()
+    return out
+
+
+def dgrad_quantize_fusion_measure(P, W, torch, device):
+    """The Dgrad that quantises its own output in the epilogue
+    (puro_fp8_linear_dgrad_quantize: both blockwise copies of dX, no BF16
+    dX) against the BF16 Dgrad followed by the activation quantiser, and
+    against the BF16 Dgrad alone, on the four Dgrad shapes of C5 (M =
+    32768).  E4M3 operands and outputs."""
+
+    def timeit(fn, reps=20):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        s = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        s.record()
+        for _ in range(reps):
+            fn()
+        e.record()
+        torch.cuda.synchronize()
+        return s.elapsed_time(e) * 1e-3 / reps
+
+    wl = W.WORKLOADS["C5"]
+    M = wl.M
+    out = []
+    for j, (name, N, K) in enumerate(wl.linears):
+        # rotate over output gradients totalling more than twice L2
+        nbuf = max(2, -(-300_000_000 // (M * N)))
+        dyqs = []
+        for i in range(nbuf):
+            dy = W.normal_bf16((M, N), 1e-3, device, 8100 + 16 * j + i)
+            dyqs.append(P.quantize(dy, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT, transpose=False))
+            del dy
+        wt = P.quantize(W.normal_bf16((N, K), 0.02, device, 8200 + j), P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT).colwise
+        dx = torch.empty((M, K), dtype=torch.bfloat16, device=device)
+        q = P.quantize(dx)
+        it = [0]
+
+        def nxt():
+            it[0] = (it[0] + 1) % nbuf
+            return dyqs[it[0]].rowwise
+
+        def fused():
+            P.puro_fp8_linear_dgrad_quantize(nxt(), wt, P.E4M3, None, q.rowwise.data, q.rowwise.scale,
+                                             q.colwise.data, q.colwise.scale)
+
+        def unfused():
+            P.puro_fp8_linear_dgrad(nxt(), wt, dx)
+            P.quantize(dx, out=q)
+
+        def dgrad_only():
+            P.puro_fp8_linear_dgrad(nxt(), wt, dx)
+
+        tf, tu, td = timeit(fused), timeit(unfused), timeit(dgrad_only)
+        flop = 2.0 * M * N * K
+        out.append({"linear": f"C5 {name} Dgrad: dY [{M}, {N}] x W -> dX [{M}, {K}]",
+                    "fused_us": tf * 1e6, "unfused_us": tu * 1e6, "dgrad_bf16_us": td * 1e6,
+                    "fused_over_unfused_time": tf / tu, "fused_tflops": flop / tf / 1e12,
+                    "dgrad_bf16_tflops": flop / td / 1e12})
+        del dyqs, wt, dx, q
         torch.cuda.empty_cache()
     return out
 
@@ -892,6 +954,7 @@ def main():
         result["paper_model_shape"] = paper_model_measure(P, W, torch, device, args.scaling)
         result["rmsnorm_quantize_fusion"] = rmsnorm_fusion_measure(P, W, torch, device)
         result["swiglu_quantize_fusion"] = swiglu_fusion_measure(P, W, torch, device)
+        result["dgrad_quantize_fusion"] = dgrad_quantize_fusion_measure(P, W, torch, device)
         result["muonh_step"] = muonh_measure(P, W, torch, device, peaks)
         if args.scaling == "block":
             result["tensor_scaling"] = tensor_scaling_measure(P, W, torch, device)

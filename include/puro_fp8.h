@@ -244,6 +244,39 @@ puro_status_t puro_fp8_linear_wgrad(const puro_fp8_tensor_t *dy_t, const puro_fp
                                     int32_t *dev_status, void *stream);
 
 /*
+ * Dgrad with the next quantisation fused into its epilogue.
+ *
+ * The backward pass carries the output gradient of one linear, through the
+ * elementwise steps between layers, to the output gradient dY of the linear
+ * before it, and the FP8 pipeline quantises that dY twice: rowwise for the
+ * layer's Dgrad and transposed for its Wgrad (appendix "FP8 implementation
+ * pipeline"; section "FP8 Mixed-Precision Training": activation gradients
+ * in E4M3 with 1x128 groups along the reduction dimension).  Where the Dgrad
+ * output is that next dY, this entry point computes
+ *     dx = dy * w_t^T        (as puro_fp8_linear_dgrad; BLOCK scaling only)
+ * and quantises bf16(dx) in the GEMM's epilogue, writing exactly what
+ * puro_fp8_quantize(dx, M, K, fmt, PURO_SCALE_BLOCK, PURO_ROLE_ACT, ...)
+ * writes from the same BF16 values:
+ *   dxq [M, K] u8, dxq_scale: 1x128 groups along K (the scale layout of a
+ *     BLOCK operand [M, K], puro_fp8_scale_bytes(M, K) bytes);
+ *   dxq_t [K, M] u8, dxq_t_scale: groups of 128 rows of dx, stored
+ *     transposed (operand [K, M], puro_fp8_scale_bytes(K, M) bytes), or both
+ *     NULL for no transposed copy;
+ *   dx: bf16 [M, K], or NULL: then the BF16 product is not written;
+ *   fmt: PURO_E4M3 or PURO_E5M2, the format of both copies.
+ * dy, w_t: as in puro_fp8_linear_dgrad (both BLOCK; M, N, K multiples of
+ * 128).  The reduction is never split (no workspace).  All pointers 16-byte
+ * aligned.  dx, when written, equals puro_fp8_linear_dgrad's output for an
+ * unsplit reduction, bit for bit, and every code and scale is an exact
+ * function of those BF16 values.  One kernel on `stream`; K == 0 gives zero
+ * codes with exponent 127 (memsets).  dev_status as for the GEMMs.
+ */
+puro_status_t puro_fp8_linear_dgrad_quantize(const puro_fp8_tensor_t *dy, const puro_fp8_tensor_t *w_t,
+                                             int32_t fmt, void *dx, uint8_t *dxq, void *dxq_scale,
+                                             uint8_t *dxq_t, void *dxq_t_scale, int32_t *dev_status,
+                                             void *stream);
+
+/*
  * Wgrad accumulated into an FP32 main-grad:
  *     main_grad[n, k] += sum_m sA(n, m) sB(k, m) qA[n, m] qB[k, m]
  * (appendix "FP8 implementation pipeline": the weight gradient is

@@ -80,6 +80,7 @@ _SIGNATURES = {
     "puro_fp8_linear_fprop": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_dgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_wgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
+    "puro_fp8_linear_dgrad_quantize": (_I32, [_P, _P, _I32, _P, _P, _P, _P, _P, _P, _P]),
     "puro_fp8_linear_wgrad_main_grad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_wgrad_noalloc": (_I32, [_P, _P, _P, _P, _P]),
     "puro_fp8_workspace_size": (ctypes.c_size_t, [_I64, _I64, _I64]),
@@ -349,6 +350,22 @@ def puro_fp8_linear_dgrad(dy: FP8Operand, w_t: FP8Operand, dx: torch.Tensor, wor
                           stream=None) -> None:
     """dX [M,K] = dY [M,N] . W [N,K] (B operand = W^T [K,N])."""
     _gemm("puro_fp8_linear_dgrad", dy, w_t, dx, workspace, dev_status, stream)
+
+
+def puro_fp8_linear_dgrad_quantize(dy: FP8Operand, w_t: FP8Operand, fmt: int, dx: Optional[torch.Tensor],
+                                   dxq: torch.Tensor, dxq_scale: torch.Tensor, dxq_t: Optional[torch.Tensor] = None,
+                                   dxq_t_scale: Optional[torch.Tensor] = None, dev_status=None, stream=None) -> None:
+    """dX [M,K] = dY [M,N] . W [N,K], rounded to BF16 and quantised in the
+    GEMM's epilogue into the blockwise activation copies (dxq [M,K] with
+    1x128 groups; dxq_t [K,M] with 128-row groups, optional); dx (bf16) is
+    written only when given."""
+    ca, cb = dy.as_c(), w_t.as_c()
+    u8 = torch.uint8
+    st = load_library().puro_fp8_linear_dgrad_quantize(
+        ctypes.byref(ca), ctypes.byref(cb), fmt, _ptr(dx, torch.bfloat16, "dx"), _ptr(dxq, u8, "dxq"),
+        _ptr(dxq_scale, u8, "dxq_scale"), _ptr(dxq_t, u8, "dxq_t"), _ptr(dxq_t_scale, u8, "dxq_t_scale"),
+        _ptr(dev_status, torch.int32, "dev_status"), _stream(stream))
+    _check("puro_fp8_linear_dgrad_quantize", st)
 
 
 def puro_fp8_linear_wgrad(dy_t: FP8Operand, x_t: FP8Operand, dw: torch.Tensor, workspace=None, dev_status=None,

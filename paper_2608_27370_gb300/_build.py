@@ -18,7 +18,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libpuro_fp8.so")
 SOURCES = ["api.cu", "quantize.cu", "gemm.cu", "noalloc.cu", "muonh.cu"]
-HEADERS = ["ptx.cuh", "internal.h"]
+HEADERS = ["ptx.cuh", "internal.h", "quant_math.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
               "-Xcompiler", "-Wall", "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC]

@@ -194,6 +194,70 @@ puro_status_t bf16_gemm(const void *a, const void *b, void *d, int64_t M, int64_
     return cuda_status(launch_gemm(g, m, s));
 }
 
+// D[M,N] = A[M,K] * B[N,K]^T (block-scaled operands), rounded to BF16 and
+// quantised in the epilogue into the blockwise activation copies of D: Dq
+// [M, N] with 1x128 groups along N and, when q_t is given, Dq^T [N, M] with
+// groups of 128 rows; D itself in BF16 only when d is given.
+puro_status_t fp8_gemm_quant(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, int32_t fmt, void *d,
+                             uint8_t *q, void *q_scale, uint8_t *q_t, void *q_t_scale, int32_t *dev_status,
+                             void *stream) {
+    puro_status_t st = check_operand(a);
+    if (st != PURO_OK) return st;
+    st = check_operand(b);
+    if (st != PURO_OK) return st;
+    if (a->red != b->red || a->scaling != PURO_SCALE_BLOCK || b->scaling != PURO_SCALE_BLOCK)
+        return PURO_ERR_INVALID_ARG;
+    if (!valid_fmt(fmt)) return PURO_ERR_INVALID_ARG;
+    if (!q || !q_scale || !aligned16(q) || !aligned16(q_scale)) return PURO_ERR_INVALID_ARG;
+    if ((q_t == nullptr) != (q_t_scale == nullptr)) return PURO_ERR_INVALID_ARG;
+    if (q_t && (!aligned16(q_t) || !aligned16(q_t_scale))) return PURO_ERR_INVALID_ARG;
+    if (d && !aligned16(d)) return PURO_ERR_INVALID_ARG;
+    const int64_t M = a->rows, N = b->rows, K = a->red;  // multiples of 128 (check_operand)
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (M == 0 || N == 0) return PURO_OK;
+    if (K == 0) {  // a zero product: zero codes, scale exponent 127 (as the quantiser gives an all-zero tensor)
+        cudaError_t e = cudaMemsetAsync(q, 0, static_cast<size_t>(M * N), s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(q_scale, 127, static_cast<size_t>(M * ((N / 128 + 3) / 4) * 4), s);
+        if (e == cudaSuccess && q_t) e = cudaMemsetAsync(q_t, 0, static_cast<size_t>(M * N), s);
+        if (e == cudaSuccess && q_t)
+            e = cudaMemsetAsync(q_t_scale, 127, static_cast<size_t>(N * ((M / 128 + 3) / 4) * 4), s);
+        if (e == cudaSuccess && d) e = cudaMemsetAsync(d, 0, static_cast<size_t>(M * N) * 2, s);
+        return cuda_status(e);
+    }
+    GemmMaps m{};
+    if (!make_map(&m.a, CU_TENSOR_MAP_DATA_TYPE_UINT8, a->data, K, M, K, kGemmBKBytes, kGemmBM,
+                  CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, b->data, K, N, K, kGemmBKBytes, kGemmBN / 2,
+                  CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_scale_map(&m.sfa, a->scale, M, K) || !make_scale_map(&m.sfb, b->scale, N, K))
+        return PURO_ERR_CUDA;
+    m.d = m.a;  // the quantising epilogue stores from registers: no output map (the kernel prefetches tm_d)
+    m.ws = m.a;
+    GemmArgs g{};
+    g.kind = kGemmFP8Block;
+    g.a_fmt = a->fmt;
+    g.b_fmt = b->fmt;
+    g.M = M;
+    g.N = N;
+    g.K = K;
+    g.tile_n = 256;
+    g.sfb = static_cast<const uint8_t *>(b->scale);
+    g.status = dev_status;
+    g.wait_timeout_ns = g_wait_timeout_ns.load();
+    g.num_sms = sm_count();
+    if (g.num_sms <= 0) return PURO_ERR_CUDA;
+    g.out = d;
+    g.splits = 1;
+    g.quant_out = true;
+    g.q_fmt = fmt;
+    g.q = q;
+    g.q_scale = static_cast<uint8_t *>(q_scale);
+    g.qt = q_t;
+    g.qt_scale = static_cast<uint8_t *>(q_t_scale);
+    g.d_bf16 = d;
+    return cuda_status(launch_gemm(g, m, s));
+}
+
 }  // namespace
 
 puro_status_t fp8_gemm_entry(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, void *d, void *workspace,
@@ -394,6 +458,13 @@ PURO_API puro_status_t puro_fp8_linear_dgrad(const puro_fp8_tensor_t *dy, const 
                                              void *workspace, size_t workspace_bytes, int32_t *dev_status,
                                              void *stream) {
     return fp8_gemm(dy, w_t, dx, workspace, workspace_bytes, dev_status, stream);
+}
+
+PURO_API puro_status_t puro_fp8_linear_dgrad_quantize(const puro_fp8_tensor_t *dy, const puro_fp8_tensor_t *w_t,
+                                                      int32_t fmt, void *dx, uint8_t *dxq, void *dxq_scale,
+                                                      uint8_t *dxq_t, void *dxq_t_scale, int32_t *dev_status,
+                                                      void *stream) {
+    return fp8_gemm_quant(dy, w_t, fmt, dx, dxq, dxq_scale, dxq_t, dxq_t_scale, dev_status, stream);
 }
 
 PURO_API puro_status_t puro_fp8_linear_wgrad(const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t, void *dw,

@@ -52,8 +52,11 @@
 // barrier before tensor memory is freed.
 #include <cuda_bf16.h>
 
+#include <type_traits>
+
 #include "internal.h"
 #include "ptx.cuh"
+#include "quant_math.cuh"
 
 namespace puro {
 
@@ -76,7 +79,16 @@ constexpr int64_t kSplitRefPairs = 76;  // SM pairs the split heuristic plans fo
 static_assert(kAtomBytes == 128 && kStagesPerGroup * kBKBytes == 512, "whole k-blocks per stage, whole stages per group");
 static_assert(kAtoms == 2 && kStagesPerGroup == 2, "a stage holds k-blocks 2j, 2j+1 of a group of four");
 
-template <int BN>
+// Shared memory of the quantising epilogue (kGemmOutQuant): per group of
+// four epilogue warps (one 128-column half of the tile), the column maxima
+// each warp found over its 32 rows and the 128 column multipliers.
+struct QuantEpiSmem {
+    uint32_t colmax[2][4][64];        // [group][warp][column pair]: packed max |bf16| over the warp's rows
+    alignas(16) float colmul[2][128];  // [group][column]: 2^(127 - g), NaN for a non-finite column
+};
+struct NoQuantEpiSmem {};
+
+template <int BN, bool QOUT = false>
 struct GemmSmem {
     static constexpr int kBNHalf = BN / 2;                 // rows of B per CTA
     static constexpr bool kSfbByHelper = (BN != 256);      // B scale images built by warp 2
@@ -96,6 +108,7 @@ struct GemmSmem {
     uint64_t drain;
     uint32_t tmem_base;
     volatile int abort_flag;
+    std::conditional_t<QOUT, QuantEpiSmem, NoQuantEpiSmem> qe;
 };
 
 struct GemmParams {
@@ -112,6 +125,12 @@ struct GemmParams {
     const float *sib;
     int32_t *status;
     uint64_t wait_ns;
+    // kGemmOutQuant: the rowwise copy Dq [M, N] and its scale vectors, the
+    // transposed copy Dq^T [N, M] and its scale vectors (both null: none),
+    // the BF16 D (null: not stored), and the FP8 format of the copies
+    uint8_t *q, *q_scale, *qt, *qt_scale;
+    uint16_t *d_bf16;
+    int q_fmt;
 };
 
 // Instruction descriptors (tcgen05.mma), both operands K-major, M = 256
@@ -131,8 +150,8 @@ __host__ __device__ constexpr uint32_t idesc_mx(uint32_t atype, uint32_t btype, 
            (static_cast<uint32_t>(kPairM >> 4) << 24);
 }
 
-template <int BN>
-PURO_DEV void record_timeout(GemmSmem<BN> &sm, int32_t *status) {
+template <class Smem>
+PURO_DEV void record_timeout(Smem &sm, int32_t *status) {
     sm.abort_flag = 1;
     if (status) atomicExch(status, kStatusTimeout);
 }
@@ -175,6 +194,179 @@ PURO_DEV void pack_bf16x8(const uint32_t *src, float sab, uint32_t (&w)[4]) {
     }
 }
 
+// p ? a : b as one selp on registers.
+PURO_DEV uint32_t sel_u32(bool p, uint32_t a, uint32_t b) {
+    uint32_t r;
+    asm("{\n\t.reg .pred q;\n\tsetp.ne.u32 q, %3, 0;\n\tselp.b32 %0, %1, %2, q;\n\t}"
+        : "=r"(r)
+        : "r"(a), "r"(b), "r"(static_cast<uint32_t>(p)));
+    return r;
+}
+
+// Codes of two values of one row that belong to two columns with their own
+// multipliers m0, m1 (transposed copy); a non-finite column gives NaN codes
+// that keep each value's sign, as in quant4.
+template <int FMT>
+PURO_DEV uint32_t quant2_cols(float x0, float x1, float m0, float m1) {
+    uint32_t r = cvt_f32x2<FMT>(mul_f32x2(f32x2(x0, x1), f32x2(m0, m1)));
+    if (__builtin_expect(isnan(m0), 0)) r = (r & 0xFF00u) | ((__float_as_uint(x0) >> 24) & 0x80u) | 0x7Fu;
+    if (__builtin_expect(isnan(m1), 0)) r = (r & 0x00FFu) | ((((__float_as_uint(x1) >> 24) & 0x80u) | 0x7Fu) << 8);
+    return r;
+}
+
+// Quantising epilogue (kGemmOutQuant), run by warps 4..11 of both CTAs of
+// a pair.  Group g = (warp - 4) / 4 takes columns 128g .. 128g+127 of every
+// tile (so the two halves are quantised at the same time), warp q = warp % 4
+// (its tensor-memory lane quarter) the rows m0 + 32q .. m0 + 32q + 31, one
+// per lane.  Each thread rounds its row's 128 accumulators to BF16 (the
+// values the BF16 output has) and produces the codes and scales the
+// blockwise activation quantiser produces from them (section "FP8
+// Mixed-Precision Training": 1x128 groups along the row for the rowwise
+// copy; 128x1 groups along M -- exactly this CTA's 128 rows -- for the
+// transposed copy).  All outputs leave by plain global stores from
+// registers: a row's 128 codes as eight 16-byte stores; the transposed
+// codes after a 4x4 byte transpose within each quad of lanes, as 4-byte
+// stores that fill a 32-byte sector per column and warp.  The accumulator is
+// released once both halves are in registers (16 arrivals), so neither group
+// can fall a tile behind the MMAs.
+template <int FMT, class Smem>
+PURO_DEV void quant_epilogue(Smem &sm, const GemmParams &p, uint32_t tmem, int warp, int lane, int pair,
+                             int num_pairs, int rank) {
+    const int grp = (warp - 4) >> 2, q = warp & 3;
+    const uint32_t bar = 1u + static_cast<uint32_t>(grp);  // named barrier of the group's four warps
+    const uint32_t tempty0 = mapa_shared(smem_u32(&sm.tempty[0]), 0);  // the even CTA's
+    QuantEpiSmem &qe = sm.qe;
+    // quad byte transpose selectors (lane p of each quad of lanes)
+    const uint32_t sel1 = (lane & 1) ? 0x3715u : 0x6240u;
+    const uint32_t sel2 = (lane & 2) ? 0x3276u : 0x5410u;
+    int local = 0;
+    for (int u = pair; u < p.num_units; u += num_pairs, ++local) {
+        const WorkUnit wu = work_unit<256>(p, u);
+        const int m0 = wu.m0 + kBM * rank;
+        const int n0h = wu.n0 + 128 * grp;
+        bool ok = (sm.abort_flag == 0) && mbar_wait_bounded(&sm.tfull[0], static_cast<uint32_t>(local & 1), p.wait_ns);
+        // the group's warps meet at named barriers, so they leave together;
+        // each reaches this one after its own bounded wait
+        ok = named_bar_and(bar, 128, __all_sync(0xFFFFFFFFu, ok));
+        if (!ok) {
+            if (lane == 0) record_timeout(sm, p.status);
+            break;
+        }
+        tc_fence_after_sync();
+        // consecutive tiles' accumulators at columns 0 / 128 (shifted scheme)
+        const uint32_t t_row = tmem + (static_cast<uint32_t>(32 * q) << 16) +
+                               static_cast<uint32_t>((local & 1) * 128 + 128 * grp);
+        uint32_t v[64];  // the row in BF16, columns 2k / 2k+1 in the low / high half of v[k]
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            uint32_t r[32];
+            tmem_ld_32x32b_x32(t_row + 32 * c, r);
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
+                v[16 * c + i] = *reinterpret_cast<uint32_t *>(&b2);
+            }
+        }
+        tc_fence_before_sync();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster_cta_scope(tempty0);  // this warp's half is in registers
+        if (n0h >= p.N) continue;  // a half past the last column (N is a multiple of 128)
+        const bool rows_in = m0 < p.M;  // the CTA's 128 rows (uniform over the group)
+        const int64_t row = static_cast<int64_t>(m0 + 32 * q + lane);
+
+        if (p.d_bf16 && rows_in) {
+            uint4 *dst = reinterpret_cast<uint4 *>(p.d_bf16 + row * p.N + n0h);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) dst[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+        }
+
+        // ---- rowwise copy: the lane's row is one 1x128 group
+        {
+            uint32_t m2 = 0;
+#pragma unroll
+            for (int k = 0; k < 64; ++k) m2 = __vmaxu2(m2, v[k] & 0x7FFF7FFFu);
+            const uint32_t g = e8m0_exponent<FMT>(max(m2 & 0xFFFFu, m2 >> 16));
+            const float rmul = mul_of(g);
+            const uint64_t rm2 = f32x2(rmul, rmul);
+            const bool rnan = isnan(rmul);
+            if (rows_in) {
+                uint4 *dst = reinterpret_cast<uint4 *>(p.q + row * p.N + n0h);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {  // codes of columns 16i .. 16i+15
+                    uint32_t w[4];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const uint32_t a = v[8 * i + 2 * j], b = v[8 * i + 2 * j + 1];
+                        w[j] = quant4<FMT>(bf16_lo(a), bf16_hi(a), bf16_lo(b), bf16_hi(b), rm2, rnan);
+                    }
+                    dst[i] = make_uint4(w[0], w[1], w[2], w[3]);
+                }
+                store_scale_vec(p.q_scale, row, n0h / 128, p.N / 128, static_cast<uint8_t>(g));
+            }
+        }
+        if (p.qt == nullptr) continue;  // uniform
+
+        // ---- transposed copy: column j's group is its 128 rows in this CTA.
+        // Column maxima over the warp's 32 rows by a reduce-scatter butterfly
+        // on the packed |bf16| pairs, in two passes of 64 columns (32
+        // words): at the step with lane bit b the lane keeps the half of its
+        // words that bit selects and takes the max with the other half from
+        // lane ^ b; after five steps lane l holds word l of the pass
+        // (columns 64ps + 2l and 64ps + 2l + 1).
+#pragma unroll
+        for (int ps = 0; ps < 2; ++ps) {
+            uint32_t a[32];
+#pragma unroll
+            for (int k = 0; k < 32; ++k) a[k] = v[32 * ps + k] & 0x7FFF7FFFu;
+#pragma unroll
+            for (int st = 0; st < 5; ++st) {
+                const int half = 16 >> st;  // words kept after this step = lane bit of this step
+                const bool upper = (lane & half) != 0;
+#pragma unroll
+                for (int i = 0; i < half; ++i) {
+                    const uint32_t keep = sel_u32(upper, a[i + half], a[i]);
+                    const uint32_t send = sel_u32(upper, a[i], a[i + half]);
+                    a[i] = __vmaxu2(keep, __shfl_xor_sync(0xFFFFFFFFu, send, half));
+                }
+            }
+            qe.colmax[grp][q][32 * ps + lane] = a[0];
+        }
+        named_bar_sync(bar, 128);  // the group's column maxima written
+        {
+            const int t = 32 * q + lane;  // this thread's column
+            const uint32_t m2c = __vmaxu2(__vmaxu2(qe.colmax[grp][0][t >> 1], qe.colmax[grp][1][t >> 1]),
+                                          __vmaxu2(qe.colmax[grp][2][t >> 1], qe.colmax[grp][3][t >> 1]));
+            const uint32_t gc = e8m0_exponent<FMT>((t & 1) ? (m2c >> 16) : (m2c & 0xFFFFu));
+            qe.colmul[grp][t] = mul_of(gc);
+            if (rows_in) store_scale_vec(p.qt_scale, n0h + t, m0 / 128, p.M / 128, static_cast<uint8_t>(gc));
+        }
+        // column multipliers ready (and this group's colmax free again); any
+        // non-finite column in the half?
+        const bool any_nan = !named_bar_and(bar, 128, !isnan(qe.colmul[grp][32 * q + lane]));
+        uint8_t *qt_base = p.qt + static_cast<int64_t>(n0h + (lane & 3)) * p.M + m0 + 32 * q + 4 * (lane >> 2);
+#pragma unroll
+        for (int w = 0; w < 32; ++w) {  // columns 4w .. 4w+3
+            const float4 cm = *reinterpret_cast<const float4 *>(&qe.colmul[grp][4 * w]);
+            const uint32_t a = v[2 * w], b = v[2 * w + 1];
+            uint32_t lo, hi;
+            if (any_nan) {
+                lo = quant2_cols<FMT>(bf16_lo(a), bf16_hi(a), cm.x, cm.y);
+                hi = quant2_cols<FMT>(bf16_lo(b), bf16_hi(b), cm.z, cm.w);
+            } else {
+                lo = cvt_f32x2<FMT>(mul_f32x2(f32x2(bf16_lo(a), bf16_hi(a)), f32x2(cm.x, cm.y)));
+                hi = cvt_f32x2<FMT>(mul_f32x2(f32x2(bf16_lo(b), bf16_hi(b)), f32x2(cm.z, cm.w)));
+            }
+            // this row's codes of columns 4w .. 4w+3 -> (4x4 transpose in the
+            // quad) rows 4k .. 4k+3 of column 4w + (lane & 3)
+            uint32_t x = lo | (hi << 16);
+            x = __byte_perm(x, __shfl_xor_sync(0xFFFFFFFFu, x, 1), sel1);
+            x = __byte_perm(x, __shfl_xor_sync(0xFFFFFFFFu, x, 2), sel2);
+            if (rows_in) *reinterpret_cast<uint32_t *>(qt_base + static_cast<int64_t>(4 * w) * p.M) = x;
+        }
+    }
+}
+
 // OUT: kGemmOutBF16 writes D in BF16; kGemmOutF32Partial writes FP32
 // partial tiles of a split reduction to the workspace [splits * Mp, N],
 // Mp = num_m * 256 (rows split * Mp + m), so that a ragged last pair tile
@@ -185,13 +377,18 @@ PURO_DEV void pack_bf16x8(const uint32_t *src, float sab, uint32_t (&w)[4]) {
 // swizzle.
 // tm_sfa / tm_sfb (block kind only): the scale vectors of A / B viewed as
 // uint32 [chunks, 128] (one 512-byte chunk per row), box {128, 1}; tm_sfb is
-// read only with BN = 256.
+// read only with BN = 256.  kGemmOutQuant (block kind, BN = 256, 384
+// threads) quantises the BF16-rounded tile in the epilogue (quant_epilogue)
+// and does not use tm_d.
+template <int OUT>
+constexpr int gemm_threads() { return OUT == kGemmOutQuant ? kThreads + 128 : kThreads; }
+
 template <int KIND, int OUT, int BN>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(), 1)
     gemm_tn_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
                    const __grid_constant__ CUtensorMap tm_d, const __grid_constant__ CUtensorMap tm_sfa,
                    const __grid_constant__ CUtensorMap tm_sfb, const GemmParams p) {
-    using Smem = GemmSmem<BN>;
+    using Smem = GemmSmem<BN, OUT == kGemmOutQuant>;
     constexpr int kBNHalf = Smem::kBNHalf;
     constexpr bool kMX = (KIND == kGemmFP8Block);
     constexpr bool kHelper = kMX && Smem::kSfbByHelper;
@@ -205,8 +402,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     constexpr int kKSteps = kAtomBytes / 32;            // MMAs per atom (32 bytes of K each)
     constexpr uint32_t kStageBytes = (kBM + kBNHalf) * kBKBytes;  // one CTA's operand bytes per stage
     constexpr uint32_t kSfBytes = kHelper ? 512u : 512u + 1024u;  // one CTA's TMA scale bytes per group
-    constexpr bool OUT_F32 = (OUT != kGemmOutBF16);
-    static_assert(BN == 256 || (BN == 224 && kMX && !OUT_F32), "the 224-wide form is block-scaled, BF16 out");
+    constexpr bool OUT_F32 = (OUT == kGemmOutF32Partial || OUT == kGemmOutF32Add);
+    constexpr bool OUT_Q = (OUT == kGemmOutQuant);
+    static_assert(BN == 256 || (BN == 224 && kMX && OUT == kGemmOutBF16), "the 224-wide form is block-scaled, BF16 out");
+    static_assert(!OUT_Q || (kMX && BN == 256), "the quantising epilogue is block-scaled and 256-wide");
     static_assert(!kMX || kSfBase + kSfSets * kSfColsPerSet <= kTmemCols, "TMEM budget");
     static_assert(kAccShift + BN <= (kMX ? kSfBase : kTmemCols), "accumulators clear of the scale columns");
 
@@ -225,7 +424,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&sm.tfull[b], 1);
-            mbar_init(&sm.tempty[b], 8);  // four epilogue warps in each CTA
+            mbar_init(&sm.tempty[b], OUT_Q ? 16 : 8);  // the epilogue warps of both CTAs
         }
         for (int s = 0; s < kSfbSlots; ++s) {
             mbar_init(&sm.sfb_full[s], 2);  // the helper warp of each CTA
@@ -241,6 +440,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             tma_prefetch_desc(&tm_sfa);
             if (!kHelper) tma_prefetch_desc(&tm_sfb);
         }
+
     }
     if (warp == 1) {
         tmem_alloc_pair(&sm.tmem_base, kTmemCols);
@@ -448,6 +648,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 if (lane == 0) mbar_arrive_cluster(sfb_full0 + 8u * slot);
             }
         }
+    } else if (OUT_Q && warp >= 4) {
+        // ------------------------------------------------ quantising epilogue (both CTAs)
+        if constexpr (OUT_Q) {
+            if (p.q_fmt == 0)
+                quant_epilogue<0>(sm, p, tmem, warp, lane, pair, num_pairs, static_cast<int>(rank));
+            else
+                quant_epilogue<1>(sm, p, tmem, warp, lane, pair, num_pairs, static_cast<int>(rank));
+        }
     } else if (warp >= 4) {
         // ------------------------------------------------ epilogue (both CTAs)
         const int q = warp & 3;  // TMEM lane quarter of this warp
@@ -463,7 +671,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             const int buf = local % kAccBufs;
             const uint32_t acc_phase = static_cast<uint32_t>(local / kAccBufs) & 1u;
             bool ok = (sm.abort_flag == 0) && mbar_wait_bounded(&sm.tfull[buf], acc_phase, p.wait_ns);
-            if (!__all_sync(0xFFFFFFFFu, ok)) {
+            ok = __all_sync(0xFFFFFFFFu, ok);
+            if (!ok) {
                 if (lane == 0) record_timeout(sm, p.status);
                 break;
             }
@@ -685,7 +894,7 @@ static int max_resident_pairs(int num_sms, size_t smem) {
     if (dev >= 0 && dev < 64 && cache[dev] > 0) return cache[dev];
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(num_sms / 2 * 2), 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.blockDim = dim3(gemm_threads<OUT>(), 1, 1);
     cfg.dynamicSmemBytes = smem;
     cudaLaunchAttribute attr;
     attr.id = cudaLaunchAttributeClusterDimension;
@@ -733,18 +942,27 @@ static cudaError_t launch_kind(const GemmArgs &g, const GemmMaps &m, int splits,
     p.status = g.status;
     p.wait_ns = g.wait_timeout_ns;
 
+    p.q = g.q;
+    p.q_scale = g.q_scale;
+    p.qt = g.qt;
+    p.qt_scale = g.qt_scale;
+    p.d_bf16 = static_cast<uint16_t *>(g.d_bf16);
+    p.q_fmt = g.q_fmt;
+
     auto kern = gemm_tn_kernel<KIND, OUT, BN>;
-    const size_t smem = sizeof(GemmSmem<BN>) + 1024;
+    const size_t smem = sizeof(GemmSmem<BN, OUT == kGemmOutQuant>) + 1024;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     const int pairs_max = max_resident_pairs<KIND, OUT, BN>(g.num_sms, smem);
     const int pairs = p.num_units < pairs_max ? p.num_units : pairs_max;
-    return launch_pdl(kern, dim3(2 * pairs), dim3(kThreads), smem, s, m.a, m.b,
+    return launch_pdl(kern, dim3(2 * pairs), dim3(gemm_threads<OUT>()), smem, s, m.a, m.b,
                       OUT == kGemmOutF32Partial ? m.ws : m.d, m.sfa, m.sfb, p);
 }
 
 template <int KIND>
 static cudaError_t launch_split_or_not(const GemmArgs &g, const GemmMaps &m, cudaStream_t s) {
+    if constexpr (KIND == kGemmFP8Block)
+        if (g.quant_out) return launch_kind<KIND, kGemmOutQuant, 256>(g, m, 1, s);
     if (g.splits <= 1) {
         if (g.accumulate_f32) return launch_kind<KIND, kGemmOutF32Add, 256>(g, m, 1, s);
         if constexpr (KIND == kGemmFP8Block)

@@ -111,6 +111,7 @@ enum GemmOut : int {
     kGemmOutBF16 = 0,        // D in BF16
     kGemmOutF32Partial = 1,  // FP32 partial tiles of a split reduction (workspace)
     kGemmOutF32Add = 2,      // D (FP32) += the product (main-grad accumulation)
+    kGemmOutQuant = 3,       // D rounded to BF16, then its blockwise FP8 copies (block kind, 256-wide, unsplit)
 };
 
 struct GemmArgs {
@@ -134,6 +135,14 @@ struct GemmArgs {
     // out is an FP32 main-grad [M, N] that receives out += A * B^T (block
     // or per-tensor kinds; 256-wide tiles)
     bool accumulate_f32;
+    // kGemmOutQuant (block kind): the epilogue quantises bf16(D) into the
+    // rowwise copy q [M, N] (scales q_scale) and, when qt is set, the
+    // transposed copy qt [N, M] (scales qt_scale), in format q_fmt; D itself
+    // is stored in BF16 only when d_bf16 is set.
+    bool quant_out;
+    int q_fmt;
+    uint8_t *q, *q_scale, *qt, *qt_scale;
+    void *d_bf16;
 };
 
 // Tensor maps of one GEMM launch.

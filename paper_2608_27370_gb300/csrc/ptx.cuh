@@ -37,6 +37,23 @@ PURO_DEV uint64_t global_timer_ns() {
 PURO_DEV void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 PURO_DEV void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
+// ------------------------------------------------------ named barriers
+// Barrier `id` (1..15) among `threads` threads (a multiple of 32); with the
+// AND of every participant's predicate.
+PURO_DEV void named_bar_sync(uint32_t id, uint32_t threads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+PURO_DEV bool named_bar_and(uint32_t id, uint32_t threads, bool pred) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\tbar.red.and.pred q, %2, %3, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"(pred ? 1u : 0u), "r"(id), "r"(threads)
+        : "memory");
+    return r != 0;
+}
+
 // ---------------------------------------------------------------- mbarrier
 PURO_DEV void mbar_init(uint64_t *bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");

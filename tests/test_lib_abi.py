@@ -120,6 +120,26 @@ def test_gemm_validation(lib):
     assert f(r(_op(0, 384)), r(w), A, None, 0, None, None) == P.PURO_OK
 
 
+def test_dgrad_quantize_validation(lib):
+    f = lib.puro_fp8_linear_dgrad_quantize
+    r = ctypes.byref
+    dy, wt = _op(256, 384), _op(512, 384, role=P.ROLE_WEIGHT)
+    E4 = P.E4M3
+    assert f(r(dy), r(wt), 2, None, A, A, A, A, None, None) == BAD             # bad output format
+    assert f(r(dy), r(wt), E4, None, None, A, None, None, None, None) == BAD   # no rowwise codes
+    assert f(r(dy), r(wt), E4, None, A, None, None, None, None, None) == BAD   # no rowwise scales
+    assert f(r(dy), r(wt), E4, None, A, A, A, None, None, None) == BAD         # transposed codes without scales
+    assert f(r(dy), r(wt), E4, None, A, A, None, A, None, None) == BAD         # scales without transposed codes
+    assert f(r(dy), r(wt), E4, None, A + 8, A, None, None, None, None) == BAD  # misaligned codes
+    assert f(r(dy), r(wt), E4, A + 2, A, A, None, None, None, None) == BAD     # misaligned dx
+    assert f(r(dy), r(_op(512, 256, role=P.ROLE_WEIGHT)), E4, None, A, A, None, None, None, None) == BAD
+    assert f(r(_op(256, 384, scaling=P.SCALE_TENSOR)), r(_op(512, 384, scaling=P.SCALE_TENSOR)), E4, None, A, A,
+             None, None, None, None) == BAD                                     # BLOCK scaling only
+    assert f(None, r(wt), E4, None, A, A, None, None, None, None) == BAD
+    # an empty output extent is a valid no-op
+    assert f(r(_op(0, 384)), r(wt), E4, None, A, A, A, A, None, None) == P.PURO_OK
+
+
 def test_bf16_gemm_validation(lib):
     assert lib.puro_bf16_linear_fprop(A, A, A, 12, 16, 16, None, None) == BAD   # M % 8
     assert lib.puro_bf16_linear_fprop(A, A + 2, A, 16, 16, 16, None, None) == BAD
