@@ -7,6 +7,7 @@ enough that a full capture ends in seconds).  Not part of the library.
     python -m paper_2608_27370_gb300.microbench.kernels muonh    # gate_up [17920, 1536] + down [1536, 8960]
     python -m paper_2608_27370_gb300.microbench.kernels gemm     # down Fprop, M = 8192, N = 1536, K = 8960
     python -m paper_2608_27370_gb300.microbench.kernels gemm_k1536  # gate_up Fprop, M = 8192, N = 17920, K = 1536
+    python -m paper_2608_27370_gb300.microbench.kernels dgrad_quant  # down Dgrad + both FP8 copies of dX, M = 8192
     python -m paper_2608_27370_gb300.microbench.kernels quant    # gate_up output gradient [8192, 17920], both copies
 
 Each input is larger than L2.  Every call is made twice: the second is the
@@ -58,13 +59,22 @@ def main(which: str) -> None:
         d = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
         for _ in range(2):
             P.puro_fp8_linear_fprop(a.rowwise, b.rowwise, d)
+    elif which == "dgrad_quant":
+        # down Dgrad at M = 8192: dY [8192, 1536] x W [1536, 8960] -> dX [8192, 8960] quantised in the epilogue
+        M, N, K = 8192, 1536, 8960
+        dyq = P.quantize(W.normal_bf16((M, N), 1e-3, dev, 4), transpose=False)
+        wt = P.quantize(W.normal_bf16((N, K), 0.02, dev, 5), P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT).colwise
+        q = P.quantize(torch.empty((M, K), dtype=torch.bfloat16, device=dev))
+        for _ in range(2):
+            P.puro_fp8_linear_dgrad_quantize(dyq.rowwise, wt, P.E4M3, None, q.rowwise.data, q.rowwise.scale,
+                                             q.colwise.data, q.colwise.scale)
     elif which == "quant":
         dy = W.normal_bf16((8192, 17920), 1e-3, dev, 3)
         q = P.quantize(dy)
         for _ in range(2):
             P.quantize(dy, out=q)
     else:
-        raise SystemExit(f"unknown kernel {which!r}: swiglu, rmsnorm, muonh, gemm, gemm_k1536 or quant")
+        raise SystemExit(f"unknown kernel {which!r}: swiglu, rmsnorm, muonh, gemm, gemm_k1536, dgrad_quant or quant")
     torch.cuda.synchronize()
     print("ok", which)
 
