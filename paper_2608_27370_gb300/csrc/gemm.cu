@@ -79,12 +79,15 @@ constexpr int64_t kSplitRefPairs = 76;  // SM pairs the split heuristic plans fo
 static_assert(kAtomBytes == 128 && kStagesPerGroup * kBKBytes == 512, "whole k-blocks per stage, whole stages per group");
 static_assert(kAtoms == 2 && kStagesPerGroup == 2, "a stage holds k-blocks 2j, 2j+1 of a group of four");
 
-// Shared memory of the quantising epilogue (kGemmOutQuant): per group of
-// four epilogue warps (one 128-column half of the tile), the column maxima
-// each warp found over its 32 rows and the 128 column multipliers.
+// Shared memory of the quantising epilogue (kGemmOutQuant), per column
+// quarter j of the tile (64 columns, four epilogue warps q = 0..3): the row
+// maxima each warp found over its 64 columns (its partner quarter j ^ 1
+// covers the rest of the rows' 1x128 groups), the column maxima over each
+// warp's 32 rows, and the 64 column multipliers.
 struct QuantEpiSmem {
-    uint32_t colmax[2][4][64];        // [group][warp][column pair]: packed max |bf16| over the warp's rows
-    alignas(16) float colmul[2][128];  // [group][column]: 2^(127 - g), NaN for a non-finite column
+    uint32_t rowmax[4][4][32];        // [quarter][warp][lane]: max |bf16| of the lane's row over the quarter
+    uint32_t colmax[4][4][32];        // [quarter][warp][column pair]: packed max |bf16| over the warp's rows
+    alignas(16) float colmul[4][64];  // [quarter][column]: 2^(127 - g), NaN for a non-finite column
 };
 struct NoQuantEpiSmem {};
 
@@ -214,26 +217,29 @@ PURO_DEV uint32_t quant2_cols(float x0, float x1, float m0, float m1) {
     return r;
 }
 
-// Quantising epilogue (kGemmOutQuant), run by warps 4..11 of both CTAs of
-// a pair.  Group g = (warp - 4) / 4 takes columns 128g .. 128g+127 of every
-// tile (so the two halves are quantised at the same time), warp q = warp % 4
-// (its tensor-memory lane quarter) the rows m0 + 32q .. m0 + 32q + 31, one
-// per lane.  Each thread rounds its row's 128 accumulators to BF16 (the
-// values the BF16 output has) and produces the codes and scales the
-// blockwise activation quantiser produces from them (section "FP8
-// Mixed-Precision Training": 1x128 groups along the row for the rowwise
-// copy; 128x1 groups along M -- exactly this CTA's 128 rows -- for the
-// transposed copy).  All outputs leave by plain global stores from
-// registers: a row's 128 codes as eight 16-byte stores; the transposed
-// codes after a 4x4 byte transpose within each quad of lanes, as 4-byte
-// stores that fill a 32-byte sector per column and warp.  The accumulator is
-// released once both halves are in registers (16 arrivals), so neither group
-// can fall a tile behind the MMAs.
+// Quantising epilogue (kGemmOutQuant), run by warps 4..19 of both CTAs of
+// a pair.  Warp 4 + 4j + q takes column quarter j (columns 64j .. 64j+63 of
+// every tile; half h = j / 2) and, as its tensor-memory lane quarter q, the
+// rows m0 + 32q .. m0 + 32q + 31, one per lane; four warps per SM
+// sub-partition keep the conversion chains overlapped.  Each thread rounds
+// its row's 64 accumulators to BF16 (the values the BF16 output has) and
+// produces the codes and scales the blockwise activation quantiser produces
+// from them (section "FP8 Mixed-Precision Training": 1x128 groups along the
+// row for the rowwise copy -- a row's group spans quarters 2h and 2h+1,
+// whose warps exchange row maxima at the half's named barrier; 128x1 groups
+// along M -- exactly this CTA's 128 rows, the quarter's four warps -- for
+// the transposed copy).  All outputs leave by plain global stores from
+// registers: a row's 64 codes as four 16-byte stores; the transposed codes
+// after a 4x4 byte transpose within each quad of lanes, as 4-byte stores
+// that fill a 32-byte sector per column and warp.  The accumulator is
+// released once every quarter is in registers (32 arrivals), so no warp can
+// fall a tile behind the MMAs.
 template <int FMT, class Smem>
 PURO_DEV void quant_epilogue(Smem &sm, const GemmParams &p, uint32_t tmem, int warp, int lane, int pair,
                              int num_pairs, int rank) {
-    const int grp = (warp - 4) >> 2, q = warp & 3;
-    const uint32_t bar = 1u + static_cast<uint32_t>(grp);  // named barrier of the group's four warps
+    const int j = (warp - 4) >> 2, q = warp & 3, h = j >> 1;
+    const uint32_t bar_half = 1u + static_cast<uint32_t>(h);  // the half's eight warps
+    const uint32_t bar_quarter = 3u + static_cast<uint32_t>(j);  // the quarter's four warps
     const uint32_t tempty0 = mapa_shared(smem_u32(&sm.tempty[0]), 0);  // the even CTA's
     QuantEpiSmem &qe = sm.qe;
     // quad byte transpose selectors (lane p of each quad of lanes)
@@ -243,11 +249,11 @@ PURO_DEV void quant_epilogue(Smem &sm, const GemmParams &p, uint32_t tmem, int w
     for (int u = pair; u < p.num_units; u += num_pairs, ++local) {
         const WorkUnit wu = work_unit<256>(p, u);
         const int m0 = wu.m0 + kBM * rank;
-        const int n0h = wu.n0 + 128 * grp;
+        const int nq = wu.n0 + 64 * j;  // first column of the quarter
         bool ok = (sm.abort_flag == 0) && mbar_wait_bounded(&sm.tfull[0], static_cast<uint32_t>(local & 1), p.wait_ns);
-        // the group's warps meet at named barriers, so they leave together;
+        // the half's warps meet at named barriers, so they leave together;
         // each reaches this one after its own bounded wait
-        ok = named_bar_and(bar, 128, __all_sync(0xFFFFFFFFu, ok));
+        ok = named_bar_and(bar_half, 256, __all_sync(0xFFFFFFFFu, ok));
         if (!ok) {
             if (lane == 0) record_timeout(sm, p.status);
             break;
@@ -255,10 +261,10 @@ PURO_DEV void quant_epilogue(Smem &sm, const GemmParams &p, uint32_t tmem, int w
         tc_fence_after_sync();
         // consecutive tiles' accumulators at columns 0 / 128 (shifted scheme)
         const uint32_t t_row = tmem + (static_cast<uint32_t>(32 * q) << 16) +
-                               static_cast<uint32_t>((local & 1) * 128 + 128 * grp);
-        uint32_t v[64];  // the row in BF16, columns 2k / 2k+1 in the low / high half of v[k]
+                               static_cast<uint32_t>((local & 1) * 128 + 64 * j);
+        uint32_t v[32];  // the row's quarter in BF16, columns 2k / 2k+1 in the low / high half of v[k]
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+        for (int c = 0; c < 2; ++c) {
             uint32_t r[32];
             tmem_ld_32x32b_x32(t_row + 32 * c, r);
             tmem_ld_wait();
@@ -270,55 +276,57 @@ PURO_DEV void quant_epilogue(Smem &sm, const GemmParams &p, uint32_t tmem, int w
         }
         tc_fence_before_sync();
         __syncwarp();
-        if (lane == 0) mbar_arrive_cluster_cta_scope(tempty0);  // this warp's half is in registers
-        if (n0h >= p.N) continue;  // a half past the last column (N is a multiple of 128)
-        const bool rows_in = m0 < p.M;  // the CTA's 128 rows (uniform over the group)
+        if (lane == 0) mbar_arrive_cluster_cta_scope(tempty0);  // this warp's quarter is in registers
+        if (wu.n0 + 128 * h >= p.N) continue;  // a half past the last column (uniform over the half)
+        const bool rows_in = m0 < p.M;  // the CTA's 128 rows
         const int64_t row = static_cast<int64_t>(m0 + 32 * q + lane);
 
         if (p.d_bf16 && rows_in) {
-            uint4 *dst = reinterpret_cast<uint4 *>(p.d_bf16 + row * p.N + n0h);
+            uint4 *dst = reinterpret_cast<uint4 *>(p.d_bf16 + row * p.N + nq);
 #pragma unroll
-            for (int i = 0; i < 16; ++i) dst[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+            for (int i = 0; i < 8; ++i) dst[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
         }
 
-        // ---- rowwise copy: the lane's row is one 1x128 group
+        // ---- rowwise copy: the row's 1x128 group is this quarter and its partner
         {
             uint32_t m2 = 0;
 #pragma unroll
-            for (int k = 0; k < 64; ++k) m2 = __vmaxu2(m2, v[k] & 0x7FFF7FFFu);
-            const uint32_t g = e8m0_exponent<FMT>(max(m2 & 0xFFFFu, m2 >> 16));
+            for (int k = 0; k < 32; ++k) m2 = __vmaxu2(m2, v[k] & 0x7FFF7FFFu);
+            const uint32_t mine = max(m2 & 0xFFFFu, m2 >> 16);
+            qe.rowmax[j][q][lane] = mine;
+            named_bar_sync(bar_half, 256);  // both quarters' row maxima written
+            const uint32_t g = e8m0_exponent<FMT>(max(mine, qe.rowmax[j ^ 1][q][lane]));
             const float rmul = mul_of(g);
             const uint64_t rm2 = f32x2(rmul, rmul);
             const bool rnan = isnan(rmul);
             if (rows_in) {
-                uint4 *dst = reinterpret_cast<uint4 *>(p.q + row * p.N + n0h);
+                uint4 *dst = reinterpret_cast<uint4 *>(p.q + row * p.N + nq);
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {  // codes of columns 16i .. 16i+15
+                for (int i = 0; i < 4; ++i) {  // codes of columns 16i .. 16i+15 of the quarter
                     uint32_t w[4];
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const uint32_t a = v[8 * i + 2 * j], b = v[8 * i + 2 * j + 1];
-                        w[j] = quant4<FMT>(bf16_lo(a), bf16_hi(a), bf16_lo(b), bf16_hi(b), rm2, rnan);
+                    for (int k = 0; k < 4; ++k) {
+                        const uint32_t a = v[8 * i + 2 * k], b = v[8 * i + 2 * k + 1];
+                        w[k] = quant4<FMT>(bf16_lo(a), bf16_hi(a), bf16_lo(b), bf16_hi(b), rm2, rnan);
                     }
                     dst[i] = make_uint4(w[0], w[1], w[2], w[3]);
                 }
-                store_scale_vec(p.q_scale, row, n0h / 128, p.N / 128, static_cast<uint8_t>(g));
+                if ((j & 1) == 0)  // one scale per row and group
+                    store_scale_vec(p.q_scale, row, (wu.n0 + 128 * h) / 128, p.N / 128, static_cast<uint8_t>(g));
             }
         }
         if (p.qt == nullptr) continue;  // uniform
 
-        // ---- transposed copy: column j's group is its 128 rows in this CTA.
+        // ---- transposed copy: column c's group is its 128 rows in this CTA.
         // Column maxima over the warp's 32 rows by a reduce-scatter butterfly
-        // on the packed |bf16| pairs, in two passes of 64 columns (32
-        // words): at the step with lane bit b the lane keeps the half of its
-        // words that bit selects and takes the max with the other half from
-        // lane ^ b; after five steps lane l holds word l of the pass
-        // (columns 64ps + 2l and 64ps + 2l + 1).
-#pragma unroll
-        for (int ps = 0; ps < 2; ++ps) {
+        // on the packed |bf16| pairs: at the step with lane bit b the lane
+        // keeps the half of its words that bit selects and takes the max with
+        // the other half from lane ^ b; after five steps lane l holds word l
+        // (columns 2l and 2l + 1 of the quarter).
+        {
             uint32_t a[32];
 #pragma unroll
-            for (int k = 0; k < 32; ++k) a[k] = v[32 * ps + k] & 0x7FFF7FFFu;
+            for (int k = 0; k < 32; ++k) a[k] = v[k] & 0x7FFF7FFFu;
 #pragma unroll
             for (int st = 0; st < 5; ++st) {
                 const int half = 16 >> st;  // words kept after this step = lane bit of this step
@@ -330,24 +338,28 @@ PURO_DEV void quant_epilogue(Smem &sm, const GemmParams &p, uint32_t tmem, int w
                     a[i] = __vmaxu2(keep, __shfl_xor_sync(0xFFFFFFFFu, send, half));
                 }
             }
-            qe.colmax[grp][q][32 * ps + lane] = a[0];
+            qe.colmax[j][q][lane] = a[0];
         }
-        named_bar_sync(bar, 128);  // the group's column maxima written
+        named_bar_sync(bar_quarter, 128);  // the quarter's column maxima written
+        bool col_ok = true;
         {
-            const int t = 32 * q + lane;  // this thread's column
-            const uint32_t m2c = __vmaxu2(__vmaxu2(qe.colmax[grp][0][t >> 1], qe.colmax[grp][1][t >> 1]),
-                                          __vmaxu2(qe.colmax[grp][2][t >> 1], qe.colmax[grp][3][t >> 1]));
-            const uint32_t gc = e8m0_exponent<FMT>((t & 1) ? (m2c >> 16) : (m2c & 0xFFFFu));
-            qe.colmul[grp][t] = mul_of(gc);
-            if (rows_in) store_scale_vec(p.qt_scale, n0h + t, m0 / 128, p.M / 128, static_cast<uint8_t>(gc));
+            const int t = 32 * q + lane;  // t < 64: this thread's column
+            if (t < 64) {
+                const uint32_t m2c = __vmaxu2(__vmaxu2(qe.colmax[j][0][t >> 1], qe.colmax[j][1][t >> 1]),
+                                              __vmaxu2(qe.colmax[j][2][t >> 1], qe.colmax[j][3][t >> 1]));
+                const uint32_t gc = e8m0_exponent<FMT>((t & 1) ? (m2c >> 16) : (m2c & 0xFFFFu));
+                const float cmul = mul_of(gc);
+                qe.colmul[j][t] = cmul;
+                col_ok = !isnan(cmul);
+                if (rows_in) store_scale_vec(p.qt_scale, nq + t, m0 / 128, p.M / 128, static_cast<uint8_t>(gc));
+            }
         }
-        // column multipliers ready (and this group's colmax free again); any
-        // non-finite column in the half?
-        const bool any_nan = !named_bar_and(bar, 128, !isnan(qe.colmul[grp][32 * q + lane]));
-        uint8_t *qt_base = p.qt + static_cast<int64_t>(n0h + (lane & 3)) * p.M + m0 + 32 * q + 4 * (lane >> 2);
+        // column multipliers ready; any non-finite column in the quarter?
+        const bool any_nan = !named_bar_and(bar_quarter, 128, col_ok);
+        uint8_t *qt_base = p.qt + static_cast<int64_t>(nq + (lane & 3)) * p.M + m0 + 32 * q + 4 * (lane >> 2);
 #pragma unroll
-        for (int w = 0; w < 32; ++w) {  // columns 4w .. 4w+3
-            const float4 cm = *reinterpret_cast<const float4 *>(&qe.colmul[grp][4 * w]);
+        for (int w = 0; w < 16; ++w) {  // columns 4w .. 4w+3 of the quarter
+            const float4 cm = *reinterpret_cast<const float4 *>(&qe.colmul[j][4 * w]);
             const uint32_t a = v[2 * w], b = v[2 * w + 1];
             uint32_t lo, hi;
             if (any_nan) {
@@ -377,11 +389,11 @@ PURO_DEV void quant_epilogue(Smem &sm, const GemmParams &p, uint32_t tmem, int w
 // swizzle.
 // tm_sfa / tm_sfb (block kind only): the scale vectors of A / B viewed as
 // uint32 [chunks, 128] (one 512-byte chunk per row), box {128, 1}; tm_sfb is
-// read only with BN = 256.  kGemmOutQuant (block kind, BN = 256, 384
+// read only with BN = 256.  kGemmOutQuant (block kind, BN = 256, 640
 // threads) quantises the BF16-rounded tile in the epilogue (quant_epilogue)
 // and does not use tm_d.
 template <int OUT>
-constexpr int gemm_threads() { return OUT == kGemmOutQuant ? kThreads + 128 : kThreads; }
+constexpr int gemm_threads() { return OUT == kGemmOutQuant ? kThreads + 384 : kThreads; }
 
 template <int KIND, int OUT, int BN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(), 1)
@@ -424,7 +436,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&sm.tfull[b], 1);
-            mbar_init(&sm.tempty[b], OUT_Q ? 16 : 8);  // the epilogue warps of both CTAs
+            mbar_init(&sm.tempty[b], OUT_Q ? 32 : 8);  // the epilogue warps of both CTAs
         }
         for (int s = 0; s < kSfbSlots; ++s) {
             mbar_init(&sm.sfb_full[s], 2);  // the helper warp of each CTA
@@ -648,9 +660,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
                 if (lane == 0) mbar_arrive_cluster(sfb_full0 + 8u * slot);
             }
         }
-    } else if (OUT_Q && warp >= 4) {
+    } else if constexpr (OUT_Q) {
         // ------------------------------------------------ quantising epilogue (both CTAs)
-        if constexpr (OUT_Q) {
+        if (warp >= 4) {
             if (p.q_fmt == 0)
                 quant_epilogue<0>(sm, p, tmem, warp, lane, pair, num_pairs, static_cast<int>(rank));
             else
