@@ -138,6 +138,40 @@ puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t cols,
                                 void *stream);
 
 /*
+ * Many weights quantised in one call.
+ *
+ * The weights are quantised once per optimizer step (section "FP8
+ * Mixed-Precision Training": 128x128 blocks, the transposed copy sharing
+ * the block scales), so a caller can quantise all of a model's weights at
+ * once.  Each entry is quantised exactly as
+ *     puro_fp8_quantize(w, rows, cols, fmt, PURO_SCALE_BLOCK,
+ *                       PURO_ROLE_WEIGHT, NULL, q, scale, q_t, scale_t)
+ * would, with the same codes and scales bit for bit, but the tiles of up to
+ * 64 weights share one launch (more weights: one launch per 64).
+ *   w: bf16 [rows, cols] row-major, 16-byte aligned; rows and cols
+ *     multiples of 128 (an entry with rows or cols 0 is skipped).
+ *   q, scale: the rowwise copy [rows, cols] and its scale vectors
+ *     (puro_fp8_scale_bytes(rows, cols) bytes).
+ *   q_t, scale_t: the transposed copy [cols, rows] and its scale vectors,
+ *     or both NULL; either every non-empty entry has a transposed copy or
+ *     none does.
+ * fmt: PURO_E4M3 or PURO_E5M2 for all entries.  The table is read on the
+ * host during the call (it may be freed on return); every entry is checked
+ * before anything is enqueued.
+ */
+typedef struct {
+    const void *w;
+    int64_t rows, cols;
+    uint8_t *q;
+    void *scale;
+    uint8_t *q_t;
+    void *scale_t;
+} puro_fp8_weight_t;
+
+puro_status_t puro_fp8_quantize_weights(const puro_fp8_weight_t *weights, int32_t count, int32_t fmt,
+                                        void *stream);
+
+/*
  * RMSNorm fused ahead of the blockwise activation quantiser.
  *
  * The model normalises the hidden states with RMSNorm before the attention

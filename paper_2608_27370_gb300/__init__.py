@@ -81,6 +81,7 @@ _SIGNATURES = {
     "puro_fp8_linear_dgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_wgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_dgrad_quantize": (_I32, [_P, _P, _I32, _P, _P, _P, _P, _P, _P, _P]),
+    "puro_fp8_quantize_weights": (_I32, [_P, _I32, _I32, _P]),
     "puro_fp8_linear_wgrad_main_grad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_wgrad_noalloc": (_I32, [_P, _P, _P, _P, _P]),
     "puro_fp8_workspace_size": (ctypes.c_size_t, [_I64, _I64, _I64]),
@@ -197,6 +198,38 @@ def _gate_up(gate: torch.Tensor, up: torch.Tensor):
     if rows > 1 and up.stride(0) != ld:
         raise ValueError("gate and up must share one row stride")
     return gate.data_ptr() or None, up.data_ptr() or None, rows, cols, ld
+
+
+class puro_fp8_weight_t(ctypes.Structure):
+    _fields_ = [("w", ctypes.c_void_p), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64),
+                ("q", ctypes.c_void_p), ("scale", ctypes.c_void_p), ("q_t", ctypes.c_void_p),
+                ("scale_t", ctypes.c_void_p)]
+
+
+def weight_table(entries):
+    """The host table of puro_fp8_quantize_weights for a fixed list of
+    (w bf16 [rows, cols], Quantized with rowwise [rows, cols] and optional
+    colwise [cols, rows] operands): build it once and pass it to every call
+    (the tensors must stay alive and in place)."""
+    table = (puro_fp8_weight_t * max(1, len(entries)))()
+    u8 = torch.uint8
+    for i, (w, q) in enumerate(entries):
+        col = q.colwise
+        table[i] = puro_fp8_weight_t(_ptr(w, torch.bfloat16, "w"), w.shape[0], w.shape[1],
+                                     _ptr(q.rowwise.data, u8, "q"), _ptr(q.rowwise.scale, u8, "scale"),
+                                     _ptr(col.data, u8, "q_t") if col is not None else None,
+                                     _ptr(col.scale, u8, "scale_t") if col is not None else None)
+    table.count = len(entries)
+    return table
+
+
+def puro_fp8_quantize_weights(entries, fmt: int = E4M3, stream=None) -> None:
+    """Quantise many weights in 128x128 blocks in one call: entries is a list
+    of (w, Quantized) pairs or a table from weight_table().  Same bytes as
+    quantize(w, fmt, SCALE_BLOCK, ROLE_WEIGHT, out=q) for each."""
+    table = entries if isinstance(entries, ctypes.Array) else weight_table(entries)
+    st = load_library().puro_fp8_quantize_weights(table, table.count, fmt, _stream(stream))
+    _check("puro_fp8_quantize_weights", st)
 
 
 def puro_fp8_quantize_swiglu(gate: torch.Tensor, up: torch.Tensor, fmt: int, y: Optional[torch.Tensor],

@@ -269,6 +269,66 @@ puro_status_t fp8_gemm_entry(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t
 
 using namespace puro;
 
+PURO_API puro_status_t puro_fp8_quantize_weights(const puro_fp8_weight_t *weights, int32_t count, int32_t fmt,
+                                                 void *stream) {
+    if (count < 0 || (count > 0 && !weights) || !valid_fmt(fmt)) return PURO_ERR_INVALID_ARG;
+    if (count == 0) return PURO_OK;
+    bool has_t = false;  // from the first non-empty entry; empty entries are skipped unchecked
+    for (int32_t i = 0; i < count; ++i)
+        if (weights[i].rows > 0 && weights[i].cols > 0) {
+            has_t = weights[i].q_t != nullptr;
+            break;
+        }
+    for (int32_t i = 0; i < count; ++i) {  // every argument checked before anything is enqueued
+        const puro_fp8_weight_t &w = weights[i];
+        if (w.rows < 0 || w.cols < 0 || w.rows % 128 || w.cols % 128) return PURO_ERR_INVALID_ARG;
+        if (w.rows > INT32_MAX || w.cols > INT32_MAX) return PURO_ERR_UNSUPPORTED;
+        if (w.rows == 0 || w.cols == 0) continue;
+        if ((w.q_t != nullptr) != has_t || (w.scale_t != nullptr) != has_t) return PURO_ERR_INVALID_ARG;
+        if (!w.w || !w.q || !w.scale || !aligned16(w.w) || !aligned16(w.q) || !aligned16(w.scale) ||
+            !aligned16(w.q_t) || !aligned16(w.scale_t))
+            return PURO_ERR_INVALID_ARG;
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    static thread_local WeightGroup g;  // 26 KB: kept off the stack
+    int32_t i = 0;
+    while (i < count) {
+        g.count = 0;
+        g.tile_start[0] = 0;
+        int64_t tiles = 0;
+        for (; i < count && g.count < kWeightGroupMax; ++i) {
+            const puro_fp8_weight_t &w = weights[i];
+            if (w.rows == 0 || w.cols == 0) continue;
+            const int64_t wt = (w.rows / 128) * (w.cols / 128);
+            if (tiles + wt > INT32_MAX) break;
+            const int k = g.count;
+            if (!make_map(&g.x[k], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, w.w, w.cols, w.rows, w.cols * 2, 128, 128,
+                          CU_TENSOR_MAP_SWIZZLE_NONE) ||
+                !make_map(&g.q[k], CU_TENSOR_MAP_DATA_TYPE_UINT8, w.q, w.cols, w.rows, w.cols, 128, 128,
+                          CU_TENSOR_MAP_SWIZZLE_NONE))
+                return PURO_ERR_CUDA;
+            if (has_t) {
+                if (!make_map(&g.qt[k], CU_TENSOR_MAP_DATA_TYPE_UINT8, w.q_t, w.rows, w.cols, w.rows, 128, 128,
+                              CU_TENSOR_MAP_SWIZZLE_128B))
+                    return PURO_ERR_CUDA;
+            } else {
+                g.qt[k] = g.q[k];
+            }
+            g.scale[k] = static_cast<uint8_t *>(w.scale);
+            g.scale_t[k] = static_cast<uint8_t *>(w.scale_t);
+            g.tiles_n[k] = static_cast<int>(w.cols / 128);
+            g.kb_rows[k] = static_cast<int>(w.rows / 128);
+            tiles += wt;
+            g.tile_start[k + 1] = static_cast<int>(tiles);
+            ++g.count;
+        }
+        if (g.count == 0 && i < count) return PURO_ERR_UNSUPPORTED;  // one weight beyond the tile index range
+        const puro_status_t st = cuda_status(launch_quantize_weights(g, fmt, has_t, s));
+        if (st != PURO_OK) return st;
+    }
+    return PURO_OK;
+}
+
 PURO_API puro_status_t puro_fp8_amax(const void *x, int64_t rows, int64_t cols, uint32_t *amax_bits, void *stream) {
     if (!amax_bits || rows < 0 || cols < 0) return PURO_ERR_INVALID_ARG;
     if ((reinterpret_cast<uintptr_t>(amax_bits) & 3u) != 0) return PURO_ERR_INVALID_ARG;

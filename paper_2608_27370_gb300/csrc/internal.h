@@ -52,6 +52,21 @@ struct QuantArgs {
 
 cudaError_t launch_amax(const uint16_t *x, int64_t n, uint32_t *amax, cudaStream_t s);
 
+// Many weights quantised in one launch (128x128 blocks, optional transposed
+// copies): each weight's three tensor maps (as puro_fp8_quantize builds them)
+// and scale-vector pointers travel in the kernel's parameter block, so one
+// launch takes at most kWeightGroupMax weights.
+constexpr int kWeightGroupMax = 64;
+struct WeightGroup {
+    CUtensorMap x[kWeightGroupMax], q[kWeightGroupMax], qt[kWeightGroupMax];
+    uint8_t *scale[kWeightGroupMax], *scale_t[kWeightGroupMax];
+    int tile_start[kWeightGroupMax + 1];  // first 128x128 tile of each weight; [count] = all tiles
+    int tiles_n[kWeightGroupMax];         // column tiles of each weight (cols / 128)
+    int kb_rows[kWeightGroupMax];         // rows / 128 (k-blocks of the transposed copy)
+    int count;
+};
+cudaError_t launch_quantize_weights(const WeightGroup &g, int fmt, bool has_t, cudaStream_t s);
+
 // Producers fused ahead of the activation quantiser.
 enum QuantProd : int {
     kProdNone = 0,

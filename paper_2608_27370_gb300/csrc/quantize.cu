@@ -287,6 +287,56 @@ struct QuantSmem {
 constexpr uint64_t kQuantWaitNs = 2000000000ull;  // a TMA load always lands long before this
 
 
+// Rowwise codes (row i, 8 columns) and transposed codes (column j, 8 rows)
+// of one thread's 8x8 block v (rows 8br .. 8br+7, columns 8bc .. 8bc+7 of a
+// 128x128 tile) into the staging tiles, for a tile with one scale
+// (multiplier m2, twice; nan_all for a non-finite one).
+template <int FMT, bool HAS_T>
+PURO_DEV void tile_codes_to_stage(QuantSmem &sm, const uint4 (&v)[8], int br, int bc, uint64_t m2, bool nan_all) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        uint2 o;
+        o.x = quant4<FMT>(bf16_lo(v[i].x), bf16_hi(v[i].x), bf16_lo(v[i].y), bf16_hi(v[i].y), m2, nan_all);
+        o.y = quant4<FMT>(bf16_lo(v[i].z), bf16_hi(v[i].z), bf16_lo(v[i].w), bf16_hi(v[i].w), m2, nan_all);
+        *reinterpret_cast<uint2 *>(sm.q_stage + (8 * br + i) * kQT + 8 * bc) = o;
+    }
+    if constexpr (HAS_T) {
+        // Column j's 8 codes (rows 8br .. 8br+7) go to transposed row
+        // 8bc + j, bytes 8br .. 8br+7.  Lanes of one half-warp share br,
+        // so they would all hit the same swizzled chunk if they stored
+        // the same j together; instead lane bc stores column (s + bc) % 8
+        // at step s, which spreads the 16 lanes over all 32 banks.  The
+        // per-lane order is a barrel rotation of the code array.
+        uint2 cc[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            float c[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const uint32_t w = (j >> 1) == 0 ? v[i].x : (j >> 1) == 1 ? v[i].y : (j >> 1) == 2 ? v[i].z : v[i].w;
+                c[i] = (j & 1) ? bf16_hi(w) : bf16_lo(w);
+            }
+            cc[j].x = quant4<FMT>(c[0], c[1], c[2], c[3], m2, nan_all);
+            cc[j].y = quant4<FMT>(c[4], c[5], c[6], c[7], m2, nan_all);
+        }
+        const int rot = bc & 7;
+#pragma unroll
+        for (int b = 1; b < 8; b <<= 1) {  // cc[s] <- cc[(s + rot) % 8], one rotate-by-b stage per bit
+            const bool on = (rot & b) != 0;
+            uint2 t[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) t[k] = on ? cc[(k + b) & 7] : cc[k];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) cc[k] = t[k];
+        }
+#pragma unroll
+        for (int st = 0; st < 8; ++st) {
+            const int r = 8 * bc + ((st + rot) & 7);  // transposed row (tile column)
+            *reinterpret_cast<uint2 *>(sm.qt_stage + r * kQT + 16 * ((br >> 1) ^ (r & 7)) + 8 * (br & 1)) = cc[st];
+        }
+    }
+}
+
 // Weight (128x128 blocks) and per-tensor cast kernel: one scale per tile
 // (the block's or the tensor's), so every thread owns one 8x8 block of the
 // 128x128 tile (rows 8*br .. 8*br+7, columns 8*bc .. 8*bc+7; a warp holds
@@ -382,49 +432,7 @@ __global__ void __launch_bounds__(kQThreads, 2)
         const uint64_t m2 = f32x2(mul, mul);
         const bool nan_all = isnan(mul);
 
-        // ---- rowwise codes (row i, 8 columns) and transposed codes (column j, 8 rows)
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            uint2 o;
-            o.x = quant4<FMT>(bf16_lo(v[i].x), bf16_hi(v[i].x), bf16_lo(v[i].y), bf16_hi(v[i].y), m2, nan_all);
-            o.y = quant4<FMT>(bf16_lo(v[i].z), bf16_hi(v[i].z), bf16_lo(v[i].w), bf16_hi(v[i].w), m2, nan_all);
-            *reinterpret_cast<uint2 *>(sm.q_stage + (8 * br + i) * kQT + 8 * bc) = o;
-        }
-        if constexpr (HAS_T) {
-            // Column j's 8 codes (rows 8br .. 8br+7) go to transposed row
-            // 8bc + j, bytes 8br .. 8br+7.  Lanes of one half-warp share br,
-            // so they would all hit the same swizzled chunk if they stored
-            // the same j together; instead lane bc stores column (s + bc) % 8
-            // at step s, which spreads the 16 lanes over all 32 banks.  The
-            // per-lane order is a barrel rotation of the code array.
-            uint2 cc[8];
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                float c[8];
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const uint32_t w = (j >> 1) == 0 ? v[i].x : (j >> 1) == 1 ? v[i].y : (j >> 1) == 2 ? v[i].z : v[i].w;
-                    c[i] = (j & 1) ? bf16_hi(w) : bf16_lo(w);
-                }
-                cc[j].x = quant4<FMT>(c[0], c[1], c[2], c[3], m2, nan_all);
-                cc[j].y = quant4<FMT>(c[4], c[5], c[6], c[7], m2, nan_all);
-            }
-            const int rot = bc & 7;
-#pragma unroll
-            for (int b = 1; b < 8; b <<= 1) {  // cc[s] <- cc[(s + rot) % 8], one rotate-by-b stage per bit
-                const bool on = (rot & b) != 0;
-                uint2 t[8];
-#pragma unroll
-                for (int k = 0; k < 8; ++k) t[k] = on ? cc[(k + b) & 7] : cc[k];
-#pragma unroll
-                for (int k = 0; k < 8; ++k) cc[k] = t[k];
-            }
-#pragma unroll
-            for (int st = 0; st < 8; ++st) {
-                const int r = 8 * bc + ((st + rot) & 7);  // transposed row (tile column)
-                *reinterpret_cast<uint2 *>(sm.qt_stage + r * kQT + 16 * ((br >> 1) ^ (r & 7)) + 8 * (br & 1)) = cc[st];
-            }
-        }
+        tile_codes_to_stage<FMT, HAS_T>(sm, v, br, bc, m2, nan_all);
 
         fence_proxy_async_smem();
         __syncthreads();  // (S3) staging complete
@@ -726,6 +734,107 @@ __global__ void __launch_bounds__(kQAThreads, 2)
         }
     }
     if (tid == 0) bulk_wait_group0();
+}
+
+// ------------------------------------------------------ grouped weight cast
+// The weights of a model are quantised once per optimizer step (section "FP8
+// Mixed-Precision Training": 128x128 blocks), so all of them can go through
+// one launch: the persistent CTAs take the 128x128 tiles of every weight in
+// one sequence, weight after weight, and treat each exactly as
+// quant_tile_kernel<FMT, kQuantBlockWeight, HAS_T> does.  Small weights then
+// share waves instead of each paying a launch, a ramp and a tail.
+template <int FMT, bool HAS_T>
+__global__ void __launch_bounds__(kQThreads, 2) quant_weight_group_kernel(const __grid_constant__ WeightGroup g) {
+    extern __shared__ uint8_t smem_raw[];
+    QuantSmem &sm = *reinterpret_cast<QuantSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                   ~static_cast<uintptr_t>(1023));
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int br = 2 * warp + (lane >> 4);  // block row: tile rows 8br .. 8br+7
+    const int bc = lane & 15;               // block column: tile columns 8bc .. 8bc+7
+    pdl_wait();
+    pdl_launch_dependents();
+    if (tid == 0) {
+        mbar_init(&sm.full[0], 1);
+        mbar_init(&sm.full[1], 1);
+        fence_mbarrier_init();
+    }
+    __syncthreads();
+
+    const int ntiles = g.tile_start[g.count];
+    // the weight of tile t, scanning forward from w (tiles only increase)
+    auto locate = [&](int t, int w) {
+        while (t >= g.tile_start[w + 1]) ++w;
+        return w;
+    };
+    auto issue_load = [&](int t, int w, int b) {
+        const int lt = t - g.tile_start[w];
+        mbar_arrive_expect_tx(&sm.full[b], kQT * kQT * 2);
+        tma_load_2d(sm.in[b], &g.x[w], &sm.full[b], (lt % g.tiles_n[w]) * kQT, (lt / g.tiles_n[w]) * kQT);
+    };
+    int tile = blockIdx.x;
+    int w = 0;
+    if (tile < ntiles) {
+        w = locate(tile, 0);
+        if (tid == 0) issue_load(tile, w, 0);
+    }
+    for (int it = 0; tile < ntiles; ++it, tile += gridDim.x) {
+        w = locate(tile, w);
+        const int buf = it & 1;
+        const int lt = tile - g.tile_start[w];
+        const int64_t r0 = static_cast<int64_t>(lt / g.tiles_n[w]) * kQT;
+        const int64_t c0 = static_cast<int64_t>(lt % g.tiles_n[w]) * kQT;
+        if (tid == 0) {
+            const int next = tile + gridDim.x;
+            if (next < ntiles) issue_load(next, locate(next, w), buf ^ 1);  // buffer last read before (S3) of it-1
+        }
+        mbar_wait_bounded(&sm.full[buf], static_cast<uint32_t>(it >> 1) & 1u, kQuantWaitNs);
+
+        const uint16_t *in = sm.in[buf];
+        uint4 v[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[i] = *reinterpret_cast<const uint4 *>(in + (8 * br + i) * kQT + 8 * bc);
+        uint32_t m = 0;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) m = __vmaxu2(m, max_abs4(v[i]));
+        m = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
+        if (lane == 0) sm.red[warp] = m;
+        if (tid == 0) bulk_wait_group_read0();  // the previous tile's stores have read the staging
+        __syncthreads();                         // (S2) block maxima written, staging free
+        m = __reduce_max_sync(0xFFFFFFFFu, sm.red[lane & 7]);
+        const uint32_t blk_g = e8m0_exponent<FMT>(m);
+        const float mul = mul_of(blk_g);
+        tile_codes_to_stage<FMT, HAS_T>(sm, v, br, bc, f32x2(mul, mul), isnan(mul));
+
+        fence_proxy_async_smem();
+        __syncthreads();  // (S3) staging complete
+        if (tid == 0) {
+            tma_store_2d(&g.q[w], sm.q_stage, static_cast<int32_t>(c0), static_cast<int32_t>(r0));
+            if (HAS_T) tma_store_2d(&g.qt[w], sm.qt_stage, static_cast<int32_t>(r0), static_cast<int32_t>(c0));
+            bulk_commit_group();
+        }
+        // scale vectors: thread i < 128 row i of the rowwise copy, 128 + i row
+        // i of the transposed copy (the block's exponent over its 128 rows)
+        const bool col = tid >= kQT;
+        if (!col || HAS_T) {
+            const int i = tid & (kQT - 1);
+            store_scale_vec(col ? g.scale_t[w] : g.scale[w], (col ? c0 : r0) + i, (col ? r0 : c0) / kQT,
+                            col ? g.kb_rows[w] : g.tiles_n[w], static_cast<uint8_t>(blk_g));
+        }
+    }
+    if (tid == 0) bulk_wait_group0();
+}
+
+cudaError_t launch_quantize_weights(const WeightGroup &g, int fmt, bool has_t, cudaStream_t s) {
+    const int ntiles = g.tile_start[g.count];
+    if (ntiles == 0) return cudaSuccess;
+    auto kern = fmt == 0 ? (has_t ? quant_weight_group_kernel<0, true> : quant_weight_group_kernel<0, false>)
+                         : (has_t ? quant_weight_group_kernel<1, true> : quant_weight_group_kernel<1, false>);
+    const size_t smem = sizeof(QuantSmem) + 1024;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    const int sms = sm_count_here();
+    const int grid = ntiles < 2 * sms ? ntiles : 2 * sms;  // persistent: two CTAs per SM
+    return launch_pdl(kern, dim3(grid), dim3(kQThreads), smem, s, g);
 }
 
 // Per-tensor scale only (empty tensors: amax = 0 gives scale_inv = 1).

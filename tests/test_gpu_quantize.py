@@ -177,3 +177,39 @@ def test_tensor_quantize_empty():
     q = P.quantize(x, P.E4M3, P.SCALE_TENSOR, P.ROLE_ACT, transpose=False)
     torch.cuda.synchronize()
     assert int(host(q.amax)[0]) == 0 and host(q.rowwise.scale)[0] == 1.0
+
+
+@pytest.mark.parametrize("fmt,with_t", [(P.E4M3, True), (P.E5M2, True), (P.E4M3, False)])
+def test_grouped_weights_equal_the_single_calls(fmt, with_t):
+    """puro_fp8_quantize_weights over more than one launch's worth of weights
+    (70 entries: the four C5 shapes, an empty entry, many small ones, one
+    with a non-finite block) writes the bytes puro_fp8_quantize writes for
+    each weight; two of them are also checked against the oracle."""
+    shapes = [(2048, 1536), (1536, 1536), (17920, 1536), (1536, 8960), (0, 128)] + [(128, 256), (384, 128)] * 32 + \
+        [(256, 384)]
+    entries, singles = [], []
+    for i, (r, c) in enumerate(shapes):
+        w = W.student_t3_f32((r, c), DEV, 4000 + i).mul_(0.02).to(torch.bfloat16) if r else \
+            torch.empty((0, c), dtype=torch.bfloat16, device=DEV)
+        if i == len(shapes) - 1:
+            w[130, 200] = float("inf")  # a non-finite block
+        q = P.quantize(torch.empty_like(w), fmt, P.SCALE_BLOCK, P.ROLE_WEIGHT, transpose=with_t) if r else \
+            P.Quantized(P.FP8Operand(torch.empty((0, c), dtype=torch.uint8, device=DEV),
+                                     torch.empty(16, dtype=torch.uint8, device=DEV)), None)
+        entries.append((w, q))
+        if r:
+            singles.append(P.quantize(w, fmt, P.SCALE_BLOCK, P.ROLE_WEIGHT, transpose=with_t))
+        else:
+            singles.append(None)
+    P.puro_fp8_quantize_weights(entries, fmt)
+    torch.cuda.synchronize()
+    for i, ((w, q), s) in enumerate(zip(entries, singles)):
+        if s is None:
+            continue
+        assert torch.equal(q.rowwise.data, s.rowwise.data), f"entry {i}: codes"
+        assert torch.equal(q.rowwise.scale, s.rowwise.scale), f"entry {i}: scales"
+        if with_t:
+            assert torch.equal(q.colwise.data, s.colwise.data), f"entry {i}: transposed codes"
+            assert torch.equal(q.colwise.scale, s.colwise.scale), f"entry {i}: transposed scales"
+    check_block_weight_quant(entries[1][0], entries[1][1], fmt)
+    check_block_weight_quant(entries[-1][0], entries[-1][1], fmt)

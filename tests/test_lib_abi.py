@@ -140,6 +140,32 @@ def test_dgrad_quantize_validation(lib):
     assert f(r(_op(0, 384)), r(wt), E4, None, A, A, A, A, None, None) == P.PURO_OK
 
 
+def test_grouped_weight_quantize_validation(lib):
+    f = lib.puro_fp8_quantize_weights
+    W_ = P.puro_fp8_weight_t
+
+    def table(*entries):
+        t = (W_ * len(entries))()
+        for i, e in enumerate(entries):
+            t[i] = e
+        return t
+
+    good = W_(A, 256, 384, A, A, A, A)
+    no_t = W_(A, 256, 384, A, A, None, None)
+    assert f(None, 1, P.E4M3, None) == BAD                                   # no table
+    assert f(table(good), -1, P.E4M3, None) == BAD                           # negative count
+    assert f(table(good), 1, 5, None) == BAD                                 # bad format
+    assert f(table(W_(A, 200, 384, A, A, A, A)), 1, P.E4M3, None) == BAD      # rows % 128
+    assert f(table(good, no_t), 2, P.E4M3, None) == BAD                      # mixed transposed copies
+    assert f(table(W_(A, 256, 384, A, A, A, None)), 1, P.E4M3, None) == BAD  # q_t without scale_t
+    assert f(table(W_(A + 2, 256, 384, A, A, A, A)), 1, P.E4M3, None) == BAD  # misaligned input
+    assert f(table(W_(A, 256, 384, None, A, A, A)), 1, P.E4M3, None) == BAD   # no codes buffer
+    assert f(table(good, W_(A, 256, 384, A, A + 8, A, A)), 2, P.E4M3, None) == BAD  # checked before any launch
+    # nothing to do: valid no-ops
+    assert f(None, 0, P.E4M3, None) == P.PURO_OK
+    assert f(table(W_(None, 0, 384, None, None, None, None)), 1, P.E4M3, None) == P.PURO_OK
+
+
 def test_bf16_gemm_validation(lib):
     assert lib.puro_bf16_linear_fprop(A, A, A, 12, 16, 16, None, None) == BAD   # M % 8
     assert lib.puro_bf16_linear_fprop(A, A + 2, A, 16, 16, 16, None, None) == BAD
