@@ -46,17 +46,22 @@ FP8_PER_BF16 = 2.0  # nominal dense ratio (4.5 / 2.25 PFLOP/s)
 # sources it was captured on (sha1 prefix over the listed files) and is
 # reported as null once they change or for another workload.
 CAPTURED_TRAFFIC = {
-    "gemm": {"files": ["gemm.cu", "ptx.cuh", "internal.h", "api.cu"], "sha1": "e4c92a06da79201e",
-             "bytes_per_call": 465341077, "algorithmic_bytes_per_call": 417016966},
-    "quantize": {"files": ["quantize.cu", "ptx.cuh", "internal.h", "api.cu"], "sha1": "bb01d3c7357a17c7",
-                 "bytes_per_call": 375247893, "algorithmic_bytes_per_call": 417016966},
+    "gemm": {"files": ["gemm.cu", "ptx.cuh", "internal.h", "api.cu", "quant_math.cuh"], "sha1": "b9724bc0ccef98c9",
+             "bytes_per_algorithmic_byte": 466826602 / 417016966},
+    "quantize": {"files": ["quantize.cu", "ptx.cuh", "internal.h", "api.cu", "quant_math.cuh"], "sha1": "5aee0c2c601df405",
+                 "bytes_per_algorithmic_byte": 504511914 / 556022622},
 }
 CAPTURED_TRAFFIC_WORKLOAD = ("C5", 32768, "block")
 CAPTURED_TRAFFIC_PROFILE = "profiles/dram_traffic_C5_layer_M32768.md"
 
 
-def captured_traffic(kind: str, workload) -> "int | None":
-    """Per-call DRAM bytes of `kind` if the capture applies, else None."""
+def captured_traffic(kind: str, workload, algorithmic_bytes_per_launch: float) -> "int | None":
+    """DRAM bytes per launch of `kind` if the capture applies, else None: the
+    captured layer's DRAM bytes per algorithmic byte times the algorithmic
+    bytes of the step's average launch (the GEMM launches of a layer are the
+    same in every layer; the quantiser's grouped weight launch covers 56
+    layers' weights in the step and four in the captured layer, so its
+    average launch differs and the ratio carries over)."""
     import hashlib
 
     if tuple(workload) != CAPTURED_TRAFFIC_WORKLOAD:
@@ -66,7 +71,9 @@ def captured_traffic(kind: str, workload) -> "int | None":
     for f in rec["files"]:
         with open(os.path.join(ROOT, "paper_2608_27370_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
-    return rec["bytes_per_call"] if h.hexdigest().startswith(rec["sha1"]) else None
+    if not h.hexdigest().startswith(rec["sha1"]):
+        return None
+    return int(round(rec["bytes_per_algorithmic_byte"] * algorithmic_bytes_per_launch))
 
 
 def load_peaks():
@@ -327,6 +334,25 @@ class LinearStack:
 
     def flops_per_step(self):
         return self.L * sum(6.0 * self.M * N * K for _, N, K in self.wl.linears)
+
+    def gemm_algorithmic_bytes_per_call(self):
+        """Average over a layer's twelve GEMM calls of the bytes they move by
+        definition: both FP8 operands and their scales read once, the BF16
+        output written once (every layer has the same shapes)."""
+        M, tot = self.M, 0
+        for _, N, K in self.wl.linears:
+            tot += M * K + N * K + 2 * M * N + M * K // 128 + N * K // 16384   # fprop
+            tot += M * N + K * N + 2 * M * K + M * N // 128 + K * N // 16384   # dgrad
+            tot += N * M + K * M + 2 * N * K + N * M // 128 + K * M // 128     # wgrad
+        return tot / (3 * len(self.wl.linears))
+
+    def quantize_kernel_launches_per_step(self):
+        """Quantiser kernel launches of one step: the grouped weight call is
+        one launch per 64 weights."""
+        acts = 2 * self.L * len(self.wl.linears)
+        if self.wtable is not None:
+            return acts + -(-self.wtable.count // 64)
+        return acts + self.L * len(self.wl.linears)
 
 
 def bf16_layer_speedup(P, torch, stack):
@@ -929,14 +955,15 @@ def main():
         "roofline": {"bound": "tensor", "kernel": "gemm_tn_kernel<FP8 block-scaled>", "achieved": gemm_tflops,
                      "peak": fp8_peak_sust, "unit": "TFLOP/s", "frac": gemm_tflops / fp8_peak_sust,
                      "peak_source": f"2 x bf16_tflops_sustained ({peak_src}); kernel timed inside a long step",
-                     "traffic": captured_traffic("gemm", traffic_wl),
+                     "traffic": captured_traffic("gemm", traffic_wl, stack.gemm_algorithmic_bytes_per_call()),
                      "traffic_note": "DRAM bytes per GEMM call (avg of one layer's 12), " + CAPTURED_TRAFFIC_PROFILE,
                      "timing": "CUDA events around each launch of the last timed step, on the launching stream"},
         "roofline_quantize": {"bound": "hbm", "kernel": "quant_act_kernel (X, dY) + quant_weight_group_kernel (W)", "achieved": quant_gbs,
                               "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": quant_gbs / peaks["hbm_gbs"],
                               "peak_source": f"hbm_gbs ({peak_src})",
-                              "traffic": captured_traffic("quantize", traffic_wl),
-                              "traffic_note": "DRAM bytes per quantise call (avg of one layer's 12), " +
+                              "traffic": captured_traffic("quantize", traffic_wl,
+                                                          q["units"] / stack.quantize_kernel_launches_per_step()),
+                              "traffic_note": "DRAM bytes per quantiser launch: the captured layer's DRAM bytes per algorithmic byte times the step's average launch, " +
                                               CAPTURED_TRAFFIC_PROFILE,
                               "timing": "CUDA events around each launch of the last timed step, on the launching stream"},
     }
