@@ -300,6 +300,11 @@ class LinearStack:
               q.colwise.data, q.colwise.scale)
         self.launches_per_step += 1
 
+    def _backward_launches(self, N, K):
+        # one grouped launch when neither GEMM splits its reduction, else their own launches
+        dg, wg = self._gemm_launches(self.M, K, N), self._gemm_launches(N, K, self.M)
+        return 1 if dg == 1 and wg == 1 and self.scaling == self.P.SCALE_BLOCK else dg + wg
+
     def _gemm_launches(self, rows_out, cols_out, red):
         # one GEMM kernel, plus the reduction kernel when the split schedule is taken
         ws = self.P.puro_fp8_workspace_size(rows_out, cols_out, red)
@@ -326,25 +331,28 @@ class LinearStack:
                 _, N, K = self.wl.linears[j]
                 li = self.inputs[l][j]
                 self._quant(li.dy, P.ROLE_ACT, self.dyq[j], self.grad_fmt)
-                T.run("gemm", 2.0 * self.M * N * K, P.puro_fp8_linear_dgrad, self.dyq[j].rowwise,
-                      self.wq[l][j].colwise, self.dx[j], self.workspace)
-                T.run("gemm", 2.0 * self.M * N * K, P.puro_fp8_linear_wgrad, self.dyq[j].colwise, self.xqt[l][j],
-                      self.dw[j], self.workspace)
-                self.launches_per_step += self._gemm_launches(self.M, K, N) + self._gemm_launches(N, K, self.M)
+                # Dgrad and Wgrad of the linear: one grouped launch when both run unsplit
+                T.run("gemm", 4.0 * self.M * N * K, P.puro_fp8_linear_backward, self.dyq[j].rowwise,
+                      self.wq[l][j].colwise, self.dx[j], self.dyq[j].colwise, self.xqt[l][j], self.dw[j],
+                      self.workspace)
+                self.launches_per_step += self._backward_launches(N, K)
 
     def flops_per_step(self):
         return self.L * sum(6.0 * self.M * N * K for _, N, K in self.wl.linears)
 
     def gemm_algorithmic_bytes_per_call(self):
-        """Average over a layer's twelve GEMM calls of the bytes they move by
-        definition: both FP8 operands and their scales read once, the BF16
-        output written once (every layer has the same shapes)."""
-        M, tot = self.M, 0
+        """Algorithmic bytes per GEMM kernel launch of the step (a grouped
+        backward launch of a linear's Dgrad and Wgrad counts once; a split
+        reduction's summing kernel is part of its GEMM): both FP8 operands and
+        their scales read once and the BF16 output written once, per GEMM
+        (every layer has the same shapes)."""
+        M, tot, calls = self.M, 0, 0
         for _, N, K in self.wl.linears:
             tot += M * K + N * K + 2 * M * N + M * K // 128 + N * K // 16384   # fprop
             tot += M * N + K * N + 2 * M * K + M * N // 128 + K * N // 16384   # dgrad
             tot += N * M + K * M + 2 * N * K + N * M // 128 + K * M // 128     # wgrad
-        return tot / (3 * len(self.wl.linears))
+            calls += 1 + (1 if self._backward_launches(N, K) == 1 else 2)
+        return tot / calls
 
     def quantize_kernel_launches_per_step(self):
         """Quantiser kernel launches of one step: the grouped weight call is
@@ -956,7 +964,7 @@ def main():
                      "peak": fp8_peak_sust, "unit": "TFLOP/s", "frac": gemm_tflops / fp8_peak_sust,
                      "peak_source": f"2 x bf16_tflops_sustained ({peak_src}); kernel timed inside a long step",
                      "traffic": captured_traffic("gemm", traffic_wl, stack.gemm_algorithmic_bytes_per_call()),
-                     "traffic_note": "DRAM bytes per GEMM call (avg of one layer's 12), " + CAPTURED_TRAFFIC_PROFILE,
+                     "traffic_note": "DRAM bytes per GEMM launch: the captured layer's DRAM bytes per algorithmic byte times the step's average launch, " + CAPTURED_TRAFFIC_PROFILE,
                      "timing": "CUDA events around each launch of the last timed step, on the launching stream"},
         "roofline_quantize": {"bound": "hbm", "kernel": "quant_act_kernel (X, dY) + quant_weight_group_kernel (W)", "achieved": quant_gbs,
                               "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": quant_gbs / peaks["hbm_gbs"],

@@ -278,6 +278,28 @@ puro_status_t puro_fp8_linear_wgrad(const puro_fp8_tensor_t *dy_t, const puro_fp
                                     int32_t *dev_status, void *stream);
 
 /*
+ * Dgrad and Wgrad of one linear in one call.
+ *
+ *   dx = dy * w_t^T     (as puro_fp8_linear_dgrad)
+ *   dw = dy_t * x_t^T   (as puro_fp8_linear_wgrad)
+ * The two are independent (both need only the quantised output gradient),
+ * so when both run as unsplit 256-wide block-scaled GEMMs they share one
+ * persistent launch: the tiles of the GEMM with the longer reduction first,
+ * then the other's, which fill the last round of tiles.  Each output is
+ * then bit-identical to the separate call's without a workspace.  Otherwise
+ * (per-tensor scaling, a split reduction, the 224-wide tile form, an empty
+ * extent) the two GEMMs are launched one after the other, exactly as the
+ * separate entry points would.  Arguments as for those entry points; one
+ * workspace serves both (its bytes: the larger of the two
+ * puro_fp8_workspace_size values).  Both are validated before anything is
+ * enqueued.
+ */
+puro_status_t puro_fp8_linear_backward(const puro_fp8_tensor_t *dy, const puro_fp8_tensor_t *w_t, void *dx,
+                                       const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t, void *dw,
+                                       void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                                       void *stream);
+
+/*
  * Dgrad with the next quantisation fused into its epilogue.
  *
  * The backward pass carries the output gradient of one linear, through the

@@ -81,6 +81,7 @@ _SIGNATURES = {
     "puro_fp8_linear_dgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_wgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_dgrad_quantize": (_I32, [_P, _P, _I32, _P, _P, _P, _P, _P, _P, _P]),
+    "puro_fp8_linear_backward": (_I32, [_P, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_quantize_weights": (_I32, [_P, _I32, _I32, _P]),
     "puro_fp8_linear_wgrad_main_grad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_wgrad_noalloc": (_I32, [_P, _P, _P, _P, _P]),
@@ -383,6 +384,19 @@ def puro_fp8_linear_dgrad(dy: FP8Operand, w_t: FP8Operand, dx: torch.Tensor, wor
                           stream=None) -> None:
     """dX [M,K] = dY [M,N] . W [N,K] (B operand = W^T [K,N])."""
     _gemm("puro_fp8_linear_dgrad", dy, w_t, dx, workspace, dev_status, stream)
+
+
+def puro_fp8_linear_backward(dy: FP8Operand, w_t: FP8Operand, dx: torch.Tensor, dy_t: FP8Operand,
+                             x_t: FP8Operand, dw: torch.Tensor, workspace=None, dev_status=None, stream=None) -> None:
+    """dX [M,K] = dY . W and dW [N,K] = dY^T . X in one call (one grouped
+    launch when both are unsplit block-scaled GEMMs)."""
+    c = [op.as_c() for op in (dy, w_t, dy_t, x_t)]
+    ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    st = load_library().puro_fp8_linear_backward(
+        ctypes.byref(c[0]), ctypes.byref(c[1]), _ptr(dx, torch.bfloat16, "dx"), ctypes.byref(c[2]),
+        ctypes.byref(c[3]), _ptr(dw, torch.bfloat16, "dw"), _ptr(workspace, None, "workspace"), ws_bytes,
+        _ptr(dev_status, torch.int32, "dev_status"), _stream(stream))
+    _check("puro_fp8_linear_backward", st)
 
 
 def puro_fp8_linear_dgrad_quantize(dy: FP8Operand, w_t: FP8Operand, fmt: int, dx: Optional[torch.Tensor],

@@ -90,21 +90,36 @@ puro_status_t check_operand(const puro_fp8_tensor_t *t) {
     return PURO_OK;
 }
 
-// D[M,N] = A[M,K] * B[N,K]^T over quantised operands.
-// accumulate_f32: d is an FP32 [M, N] main-grad that receives d += A * B^T.
-puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, void *d, void *workspace,
-                       size_t workspace_bytes, int32_t *dev_status, void *stream, bool accumulate_f32 = false) {
+// What a validated GEMM call needs enqueued.
+enum GemmAction { kGemmNothing, kGemmZeroFill, kGemmLaunch };
+
+// The argument checks of D = A * B^T (host only, no CUDA call).
+puro_status_t validate_fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, const void *d) {
     puro_status_t st = check_operand(a);
     if (st != PURO_OK) return st;
     st = check_operand(b);
     if (st != PURO_OK) return st;
     if (a->red != b->red || a->scaling != b->scaling) return PURO_ERR_INVALID_ARG;
     if (!d || !aligned16(d)) return PURO_ERR_INVALID_ARG;
+    return PURO_OK;
+}
+
+// Validates D = A * B^T and prepares its launch (nothing is enqueued here).
+puro_status_t prepare_fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, void *d, void *workspace,
+                               size_t workspace_bytes, int32_t *dev_status, bool accumulate_f32, GemmArgs *gout,
+                               GemmMaps *mout, GemmAction *action) {
+    const puro_status_t st = validate_fp8_gemm(a, b, d);
+    if (st != PURO_OK) return st;
     const int64_t M = a->rows, N = b->rows, K = a->red;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    *action = kGemmNothing;
+    gout->M = M;
+    gout->N = N;
+    gout->out = d;
     if (M == 0 || N == 0) return PURO_OK;
-    if (K == 0)  // an empty reduction: the product is zero
-        return accumulate_f32 ? PURO_OK : cuda_status(cudaMemsetAsync(d, 0, static_cast<size_t>(M * N) * 2, s));
+    if (K == 0) {  // an empty reduction: the product is zero (a main-grad is left as it is)
+        if (!accumulate_f32) *action = kGemmZeroFill;
+        return PURO_OK;
+    }
     const bool block = a->scaling == PURO_SCALE_BLOCK;
 
     // Split the reduction across CTA pairs when the output has too few tiles
@@ -158,7 +173,57 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
         g.splits = sp;
         g.workspace = workspace;
     }
-    return cuda_status(launch_gemm(g, m, s));
+    *gout = g;
+    *mout = m;
+    *action = kGemmLaunch;
+    return PURO_OK;
+}
+
+puro_status_t run_fp8_gemm(GemmAction action, const GemmArgs &g, const GemmMaps &m, cudaStream_t s) {
+    if (action == kGemmZeroFill) return cuda_status(cudaMemsetAsync(g.out, 0, static_cast<size_t>(g.M * g.N) * 2, s));
+    if (action == kGemmLaunch) return cuda_status(launch_gemm(g, m, s));
+    return PURO_OK;
+}
+
+// D[M,N] = A[M,K] * B[N,K]^T over quantised operands.
+// accumulate_f32: d is an FP32 [M, N] main-grad that receives d += A * B^T.
+puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, void *d, void *workspace,
+                       size_t workspace_bytes, int32_t *dev_status, void *stream, bool accumulate_f32 = false) {
+    GemmArgs g{};
+    GemmMaps m{};
+    GemmAction action;
+    const puro_status_t st =
+        prepare_fp8_gemm(a, b, d, workspace, workspace_bytes, dev_status, accumulate_f32, &g, &m, &action);
+    if (st != PURO_OK) return st;
+    return run_fp8_gemm(action, g, m, static_cast<cudaStream_t>(stream));
+}
+
+// Dgrad and Wgrad of one linear: one grouped launch when both are unsplit
+// 256-wide block-scaled GEMMs (the problem with the longer reduction first,
+// so the other's shorter tiles fill the last round), else two.
+puro_status_t fp8_backward(const puro_fp8_tensor_t *dy, const puro_fp8_tensor_t *w_t, void *dx,
+                           const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t, void *dw, void *workspace,
+                           size_t workspace_bytes, int32_t *dev_status, void *stream) {
+    puro_status_t st = validate_fp8_gemm(dy, w_t, dx);  // both calls' arguments first
+    if (st != PURO_OK) return st;
+    st = validate_fp8_gemm(dy_t, x_t, dw);
+    if (st != PURO_OK) return st;
+    GemmArgs gd{}, gw{};
+    GemmMaps md{}, mw{};
+    GemmAction ad, aw;
+    st = prepare_fp8_gemm(dy, w_t, dx, workspace, workspace_bytes, dev_status, false, &gd, &md, &ad);
+    if (st != PURO_OK) return st;
+    st = prepare_fp8_gemm(dy_t, x_t, dw, workspace, workspace_bytes, dev_status, false, &gw, &mw, &aw);
+    if (st != PURO_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const bool grouped = ad == kGemmLaunch && aw == kGemmLaunch && gd.kind == kGemmFP8Block &&
+                         gw.kind == kGemmFP8Block && gd.splits == 1 && gw.splits == 1 && gd.tile_n == 256 &&
+                         gw.tile_n == 256;
+    if (grouped)
+        return cuda_status(gw.K >= gd.K ? launch_gemm_grouped(gw, mw, gd, md, s) : launch_gemm_grouped(gd, md, gw, mw, s));
+    st = run_fp8_gemm(ad, gd, md, s);
+    if (st != PURO_OK) return st;
+    return run_fp8_gemm(aw, gw, mw, s);
 }
 
 puro_status_t bf16_gemm(const void *a, const void *b, void *d, int64_t M, int64_t N, int64_t K,
@@ -518,6 +583,13 @@ PURO_API puro_status_t puro_fp8_linear_dgrad(const puro_fp8_tensor_t *dy, const 
                                              void *workspace, size_t workspace_bytes, int32_t *dev_status,
                                              void *stream) {
     return fp8_gemm(dy, w_t, dx, workspace, workspace_bytes, dev_status, stream);
+}
+
+PURO_API puro_status_t puro_fp8_linear_backward(const puro_fp8_tensor_t *dy, const puro_fp8_tensor_t *w_t, void *dx,
+                                                const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t, void *dw,
+                                                void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                                                void *stream) {
+    return fp8_backward(dy, w_t, dx, dy_t, x_t, dw, workspace, workspace_bytes, dev_status, stream);
 }
 
 PURO_API puro_status_t puro_fp8_linear_dgrad_quantize(const puro_fp8_tensor_t *dy, const puro_fp8_tensor_t *w_t,

@@ -134,6 +134,13 @@ struct GemmParams {
     uint8_t *q, *q_scale, *qt, *qt_scale;
     uint16_t *d_bf16;
     int q_fmt;
+    // A second problem in the same launch (the grouped backward pass: Dgrad
+    // and Wgrad of one linear; block kind, BF16 output, 256-wide, unsplit):
+    // units units0 .. num_units-1 are its whole tiles, read and written
+    // through tm_a1 .. tm_sfb1.  units0 == num_units: one problem.
+    int units0;
+    int N1, num_m1, num_n1, num_kb1, m_fastest1, kgroups1;
+    uint32_t idesc1;
 };
 
 // Instruction descriptors (tcgen05.mma), both operands K-major, M = 256
@@ -165,11 +172,25 @@ PURO_DEV void record_timeout(Smem &sm, int32_t *status) {
 // share (and read once) the blocks of the larger one.
 struct WorkUnit {
     int m0, n0, kb0, kb1, split;  // m0: first row of the pair tile
+    int problem;                  // 0, or 1 for the second problem of a grouped launch
 };
 
 template <int BN>
 PURO_DEV WorkUnit work_unit(const GemmParams &p, int u) {
     WorkUnit w;
+    if (u >= p.units0) {  // the second problem: whole tiles
+        const int tile = u - p.units0;
+        const int mb = p.m_fastest1 ? tile % p.num_m1 : tile / p.num_n1;
+        const int nb = p.m_fastest1 ? tile / p.num_m1 : tile % p.num_n1;
+        w.m0 = mb * kPairM;
+        w.n0 = nb * BN;
+        w.split = 0;
+        w.kb0 = 0;
+        w.kb1 = p.num_kb1;
+        w.problem = 1;
+        return w;
+    }
+    w.problem = 0;
     w.split = u / p.num_tiles;
     const int tile = u - w.split * p.num_tiles;
     const int mb = p.m_fastest ? tile % p.num_m : tile / p.num_n;
@@ -399,7 +420,10 @@ template <int KIND, int OUT, int BN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(), 1)
     gemm_tn_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
                    const __grid_constant__ CUtensorMap tm_d, const __grid_constant__ CUtensorMap tm_sfa,
-                   const __grid_constant__ CUtensorMap tm_sfb, const GemmParams p) {
+                   const __grid_constant__ CUtensorMap tm_sfb, const __grid_constant__ CUtensorMap tm_a1,
+                   const __grid_constant__ CUtensorMap tm_b1, const __grid_constant__ CUtensorMap tm_d1,
+                   const __grid_constant__ CUtensorMap tm_sfa1, const __grid_constant__ CUtensorMap tm_sfb1,
+                   const GemmParams p) {
     using Smem = GemmSmem<BN, OUT == kGemmOutQuant>;
     constexpr int kBNHalf = Smem::kBNHalf;
     constexpr bool kMX = (KIND == kGemmFP8Block);
@@ -452,6 +476,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
             tma_prefetch_desc(&tm_sfa);
             if (!kHelper) tma_prefetch_desc(&tm_sfb);
         }
+        if (p.units0 < p.num_units) {  // grouped launch: the second problem's maps
+            tma_prefetch_desc(&tm_a1);
+            tma_prefetch_desc(&tm_b1);
+            tma_prefetch_desc(&tm_d1);
+            tma_prefetch_desc(&tm_sfa1);
+            tma_prefetch_desc(&tm_sfb1);
+        }
 
     }
     if (warp == 1) {
@@ -477,6 +508,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
                 const WorkUnit wu = work_unit<BN>(p, u);
                 const int a_row = wu.m0 + kBM * static_cast<int>(rank);
                 const int b_row = wu.n0 + kBNHalf * static_cast<int>(rank);
+                const CUtensorMap *ma = wu.problem ? &tm_a1 : &tm_a;
+                const CUtensorMap *mb = wu.problem ? &tm_b1 : &tm_b;
+                const CUtensorMap *msfa = wu.problem ? &tm_sfa1 : &tm_sfa;
+                const CUtensorMap *msfb = wu.problem ? &tm_sfb1 : &tm_sfb;
+                const int kgroups = wu.problem ? p.kgroups1 : p.kgroups;
                 for (int kb = wu.kb0; kb < wu.kb1; ++kb) {
                     if (sm.abort_flag || !mbar_wait_bounded(&sm.empty[stage], phase ^ 1u, p.wait_ns)) {
                         record_timeout(sm, p.status);
@@ -489,17 +525,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
                         mbar_arrive_expect_tx(&sm.full[stage], 2u * (kStageBytes + (sf_load ? kSfBytes : 0u)));
 #pragma unroll
                     for (int at = 0; at < kAtoms; ++at) {
-                        tma_load_2d_pair(sm.a[stage][at], &tm_a, full_bar, kb * kBK + at * kAtomK, a_row);
-                        tma_load_2d_pair(sm.b[stage][at], &tm_b, full_bar, kb * kBK + at * kAtomK, b_row);
+                        tma_load_2d_pair(sm.a[stage][at], ma, full_bar, kb * kBK + at * kAtomK, a_row);
+                        tma_load_2d_pair(sm.b[stage][at], mb, full_bar, kb * kBK + at * kAtomK, b_row);
                     }
                     if (sf_load) {
                         // chunks beyond the operand's rows read as zero (their rows are zero too)
                         const int kg = kb / kStagesPerGroup;
-                        tma_load_2d_pair(sm.sf_a[stage], &tm_sfa, full_bar, 0, (a_row / 128) * p.kgroups + kg);
+                        tma_load_2d_pair(sm.sf_a[stage], msfa, full_bar, 0, (a_row / 128) * kgroups + kg);
                         if constexpr (!kHelper) {
-                            tma_load_2d_pair(sm.sf_b[stage], &tm_sfb, full_bar, 0, (wu.n0 / 128) * p.kgroups + kg);
-                            tma_load_2d_pair(sm.sf_b[stage] + 512, &tm_sfb, full_bar, 0,
-                                             (wu.n0 / 128 + 1) * p.kgroups + kg);
+                            tma_load_2d_pair(sm.sf_b[stage], msfb, full_bar, 0, (wu.n0 / 128) * kgroups + kg);
+                            tma_load_2d_pair(sm.sf_b[stage] + 512, msfb, full_bar, 0,
+                                             (wu.n0 / 128 + 1) * kgroups + kg);
                         }
                     }
                     ++issued;
@@ -572,7 +608,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
                     }
 #pragma unroll
                     for (int at = 0; at < kAtoms; ++at) {
-                        uint32_t idesc = p.idesc;
+                        uint32_t idesc = wu.problem ? p.idesc1 : p.idesc;
                         if constexpr (kMX) {
                             const uint32_t sf_id = static_cast<uint32_t>((kb * kAtoms + at) & 3);  // k-block in its group
                             idesc |= (sf_id << 29) | (sf_id << 4);
@@ -691,6 +727,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
             tc_fence_after_sync();
             const uint32_t t_row =
                 tmem + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>((local & 1) * kAccShift);
+            const int n_out = wu.problem ? p.N1 : p.N;  // columns of this unit's output
+            const CUtensorMap *md = wu.problem ? &tm_d1 : &tm_d;
             if constexpr (OUT_F32) {
                 // FP32 tile: 8 chunks of 32 columns (128 bytes per row), stored
                 // as a split partial or added to D
@@ -704,7 +742,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
 #pragma unroll
                     for (int c = 0; c < 4; ++c) {
                         const int col = n0 + 128 * h + 32 * c;
-                        if (col >= p.N) break;
+                        if (col >= n_out) break;
                         if (lane == 0) bulk_wait_group_read0();
                         __syncwarp();
                         uint8_t *row = stage_buf + 128 * lane;
@@ -723,9 +761,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
                         __syncwarp();
                         if (lane == 0) {
                             if constexpr (OUT == kGemmOutF32Add)
-                                tma_reduce_add_2d(&tm_d, stage_buf, col, row0);
+                                tma_reduce_add_2d(md, stage_buf, col, row0);
                             else
-                                tma_store_2d(&tm_d, stage_buf, col, row0);
+                                tma_store_2d(md, stage_buf, col, row0);
                             bulk_commit_group();
                         }
                     }
@@ -763,7 +801,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
 #pragma unroll
                     for (int c = 0; c < 4; ++c) {
                         const int col = n0 + 128 * h + 32 * c;
-                        if (c >= nc || col >= p.N) break;
+                        if (c >= nc || col >= n_out) break;
                         uint8_t *half = stage_buf + 2048 * (pieces & 1u);
                         if (lane == 0) bulk_wait_group_read<1>();  // the store that last read this half is done
                         __syncwarp();
@@ -777,7 +815,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
                         fence_proxy_async_smem();
                         __syncwarp();
                         if (lane == 0) {
-                            tma_store_2d(&tm_d, half, col, m0 + 32 * q);
+                            tma_store_2d(md, half, col, m0 + 32 * q);
                             bulk_commit_group();
                         }
                         ++pieces;
@@ -925,7 +963,7 @@ static int max_resident_pairs(int num_sms, size_t smem) {
 }
 
 template <int KIND, int OUT, int BN>
-static cudaError_t launch_kind(const GemmArgs &g, const GemmMaps &m, int splits, cudaStream_t s) {
+static GemmParams make_params(const GemmArgs &g, int splits) {
     constexpr int kElemBytes = (KIND == kGemmBF16) ? 2 : 1;
     constexpr int kBK = kBKBytes / kElemBytes;
     GemmParams p{};
@@ -960,7 +998,15 @@ static cudaError_t launch_kind(const GemmArgs &g, const GemmMaps &m, int splits,
     p.qt_scale = g.qt_scale;
     p.d_bf16 = static_cast<uint16_t *>(g.d_bf16);
     p.q_fmt = g.q_fmt;
+    p.units0 = p.num_units;  // one problem unless a grouped launch adds a second
+    return p;
+}
 
+// Launch with the parameters p; m1: the second problem's maps of a grouped
+// launch (unused otherwise).
+template <int KIND, int OUT, int BN>
+static cudaError_t launch_params(const GemmParams &p, const GemmArgs &g, const GemmMaps &m, const GemmMaps &m1,
+                                 cudaStream_t s) {
     auto kern = gemm_tn_kernel<KIND, OUT, BN>;
     const size_t smem = sizeof(GemmSmem<BN, OUT == kGemmOutQuant>) + 1024;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
@@ -968,7 +1014,12 @@ static cudaError_t launch_kind(const GemmArgs &g, const GemmMaps &m, int splits,
     const int pairs_max = max_resident_pairs<KIND, OUT, BN>(g.num_sms, smem);
     const int pairs = p.num_units < pairs_max ? p.num_units : pairs_max;
     return launch_pdl(kern, dim3(2 * pairs), dim3(gemm_threads<OUT>()), smem, s, m.a, m.b,
-                      OUT == kGemmOutF32Partial ? m.ws : m.d, m.sfa, m.sfb, p);
+                      OUT == kGemmOutF32Partial ? m.ws : m.d, m.sfa, m.sfb, m1.a, m1.b, m1.d, m1.sfa, m1.sfb, p);
+}
+
+template <int KIND, int OUT, int BN>
+static cudaError_t launch_kind(const GemmArgs &g, const GemmMaps &m, int splits, cudaStream_t s) {
+    return launch_params<KIND, OUT, BN>(make_params<KIND, OUT, BN>(g, splits), g, m, m, s);
 }
 
 template <int KIND>
@@ -994,6 +1045,25 @@ static cudaError_t launch_split_or_not(const GemmArgs &g, const GemmMaps &m, cud
                           reinterpret_cast<float4 *>(g.out));
     return launch_pdl(splitk_reduce_kernel, dim3(grid), dim3(256), 0, s, ws, g.splits, n4, stride4,
                       reinterpret_cast<uint2 *>(g.out));
+}
+
+// Two block-scaled GEMMs (BF16 output, 256-wide, unsplit) in one persistent
+// launch: g0's tiles first, then g1's (the caller puts the problem with the
+// longer reductions first, so the shorter tiles fill the last round).
+cudaError_t launch_gemm_grouped(const GemmArgs &g0, const GemmMaps &m0, const GemmArgs &g1, const GemmMaps &m1,
+                                cudaStream_t s) {
+    GemmParams p = make_params<kGemmFP8Block, kGemmOutBF16, 256>(g0, 1);
+    const GemmParams q = make_params<kGemmFP8Block, kGemmOutBF16, 256>(g1, 1);
+    p.units0 = p.num_units;
+    p.N1 = q.N;
+    p.num_m1 = q.num_m;
+    p.num_n1 = q.num_n;
+    p.num_kb1 = q.num_kb;
+    p.m_fastest1 = q.m_fastest;
+    p.kgroups1 = q.kgroups;
+    p.idesc1 = q.idesc;
+    p.num_units += q.num_units;
+    return launch_params<kGemmFP8Block, kGemmOutBF16, 256>(p, g0, m0, m1, s);
 }
 
 cudaError_t launch_gemm(const GemmArgs &g, const GemmMaps &m, cudaStream_t s) {

@@ -176,6 +176,10 @@ struct GemmMaps {
 };
 
 cudaError_t launch_gemm(const GemmArgs &g, const GemmMaps &m, cudaStream_t s);
+// Two block-scaled GEMMs with BF16 output in one launch (the Dgrad and Wgrad
+// of one linear): 256-wide tiles, neither reduction split.
+cudaError_t launch_gemm_grouped(const GemmArgs &g0, const GemmMaps &m0, const GemmArgs &g1, const GemmMaps &m1,
+                                cudaStream_t s);
 
 // The FP8 GEMM entry behind puro_fp8_linear_{fprop,dgrad,wgrad}: validates,
 // encodes the tensor maps and launches (D = A * B^T).

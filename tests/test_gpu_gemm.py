@@ -202,3 +202,38 @@ def test_wgrad_main_grad_zero_reduction_leaves_it_unchanged():
                                                stream) == 0
     torch.cuda.synchronize()
     assert torch.equal(main, before)
+
+
+@pytest.mark.parametrize("M,N,K", [(8192, 4096, 2048),     # both unsplit: one grouped launch
+                                   (4096, 2304, 1536),     # ragged last rounds in both
+                                   (2048, 1536, 1536)])    # Wgrad small enough to split: two launches
+def test_grouped_backward_equals_separate_calls(M, N, K):
+    """puro_fp8_linear_backward gives the same dX and dW as the separate
+    Dgrad and Wgrad calls, bit for bit (without a workspace both run
+    unsplit, as the grouped launch does), and within tolerance of the
+    oracle."""
+    x, w, dy = _inputs(M, N, K, 6000 + M + N + K)
+    xq = P.quantize(x, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT)
+    wq = P.quantize(w, P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT)
+    dyq = P.quantize(dy, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT)
+    dx, dw = torch.empty((M, K), dtype=torch.bfloat16, device=DEV), torch.empty((N, K), dtype=torch.bfloat16, device=DEV)
+    dx1, dw1 = torch.empty_like(dx), torch.empty_like(dw)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    P.puro_fp8_linear_backward(dyq.rowwise, wq.colwise, dx, dyq.colwise, xq.colwise, dw, dev_status=status)
+    P.puro_fp8_linear_dgrad(dyq.rowwise, wq.colwise, dx1)
+    P.puro_fp8_linear_wgrad(dyq.colwise, xq.colwise, dw1)
+    torch.cuda.synchronize()
+    assert P.puro_fp8_get_status(status) == 0
+    assert torch.equal(dx.view(torch.int16), dx1.view(torch.int16)), "dX differs from the separate Dgrad"
+    assert torch.equal(dw.view(torch.int16), dw1.view(torch.int16)), "dW differs from the separate Wgrad"
+    if M * N * K <= 4096 * 2304 * 1536:
+        ref = oracle_linear(x, w, dy, P.SCALE_BLOCK)
+        assert_close(dx, ref["dx"], "grouped dgrad")
+        assert_close(dw, ref["dw"], "grouped wgrad")
+    # with a workspace (the Wgrad may split): still within tolerance of the separate calls' results
+    ws = torch.empty(max(16, P.puro_fp8_workspace_size(M, K, N), P.puro_fp8_workspace_size(N, K, M)),
+                     dtype=torch.uint8, device=DEV)
+    P.puro_fp8_linear_backward(dyq.rowwise, wq.colwise, dx, dyq.colwise, xq.colwise, dw, ws, status)
+    torch.cuda.synchronize()
+    assert torch.equal(dx.view(torch.int16), dx1.view(torch.int16))
+    assert P.puro_fp8_get_status(status) == 0

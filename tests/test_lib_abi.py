@@ -166,6 +166,21 @@ def test_grouped_weight_quantize_validation(lib):
     assert f(table(W_(None, 0, 384, None, None, None, None)), 1, P.E4M3, None) == P.PURO_OK
 
 
+def test_backward_validation(lib):
+    f = lib.puro_fp8_linear_backward
+    r = ctypes.byref
+    # dY [256, 384], W^T [512, 384] -> dX [256, 512]; dY^T [384, 256], X^T [512, 256] -> dW [384, 512]
+    dy, wt = _op(256, 384), _op(512, 384, role=P.ROLE_WEIGHT)
+    dyt, xt = _op(384, 256), _op(512, 256)
+    assert f(r(dy), r(wt), None, r(dyt), r(xt), A, None, 0, None, None) == BAD              # no dX
+    assert f(r(dy), r(wt), A, r(dyt), r(xt), A + 4, None, 0, None, None) == BAD             # misaligned dW
+    assert f(r(dy), r(wt), A, r(dyt), r(_op(512, 128)), A, None, 0, None, None) == BAD      # Wgrad reduction mismatch
+    assert f(r(dy), r(_op(512, 256, role=P.ROLE_WEIGHT)), A, r(dyt), r(xt), A, None, 0, None, None) == BAD
+    assert f(None, r(wt), A, r(dyt), r(xt), A, None, 0, None, None) == BAD
+    # both empty: a valid no-op
+    assert f(r(_op(0, 384)), r(wt), A, r(_op(0, 256)), r(xt), A, None, 0, None, None) == P.PURO_OK
+
+
 def test_bf16_gemm_validation(lib):
     assert lib.puro_bf16_linear_fprop(A, A, A, 12, 16, 16, None, None) == BAD   # M % 8
     assert lib.puro_bf16_linear_fprop(A, A + 2, A, 16, 16, 16, None, None) == BAD
