@@ -5,11 +5,13 @@ One step = one forward + backward pass of every linear layer of the
 workload through the library's C ABI, in the paper's recipe (section "FP8
 Mixed-Precision Training"; appendix "FP8 implementation pipeline"):
 
-  forward, layer 0 .. L-1, each linear: quantise W (128x128 blocks, with the
-      transposed copy), quantise X (1x128 groups, rowwise for Fprop and the
-      transposed copy kept for Wgrad), Fprop Y = X W^T
+  first every weight W (128x128 blocks, with the transposed copy), 64 weights
+      per launch
+  forward, layer 0 .. L-1, each linear: quantise X (1x128 groups, rowwise for
+      Fprop and the transposed copy kept for Wgrad), Fprop Y = X W^T
   backward, layer L-1 .. 0, each linear in reverse: quantise dY (rowwise and
-      transposed), Dgrad dX = dY W, Wgrad dW = dY^T X
+      transposed), Dgrad dX = dY W and Wgrad dW = dY^T X (one grouped launch
+      when neither splits its reduction)
 
 Default workload: the 28-layer Qwen2-1.5B linear stack at M = 32768 tokens
 (qkv, o_proj, gate_up, down per layer), distinct seeded inputs per layer,
@@ -38,18 +40,18 @@ METRIC = "FP8 linear fwd+bwd TFLOP/s and % of FP8 peak; quantise HBM GB/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 FP8_PER_BF16 = 2.0  # nominal dense ratio (4.5 / 2.25 PFLOP/s)
 
-# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per call, averaged
-# over the 12 GEMM calls (split reductions included) and the 12 quantise calls
-# of one layer, from a one-pass ncu capture of one full-size layer of the C5
-# workload (block scaling, M = 32768).  All 28 layers have the same shapes, so
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per algorithmic
+# byte over the 10 GEMM launches (split reductions included) and the 9
+# quantise launches of one layer, from a one-pass ncu capture of one
+# full-size layer of the C5 workload (block scaling, M = 32768).  All 28 layers have the same shapes, so
 # one layer's calls stand for the step.  Each figure holds only for the kernel
 # sources it was captured on (sha1 prefix over the listed files) and is
 # reported as null once they change or for another workload.
 CAPTURED_TRAFFIC = {
     "gemm": {"files": ["gemm.cu", "ptx.cuh", "internal.h", "api.cu", "quant_math.cuh"], "sha1": "1b6e9d73d37ce447",
-             "bytes_per_algorithmic_byte": 571404902 / 500420360},
-    "quantize": {"files": ["quantize.cu", "ptx.cuh", "internal.h", "api.cu", "quant_math.cuh"], "sha1": "dfaf943fd3ae1c5a",
-                 "bytes_per_algorithmic_byte": 504492145 / 556022622},
+             "bytes_per_algorithmic_byte": 567309235 / 500420360},
+    "quantize": {"files": ["quantize.cu", "ptx.cuh", "internal.h", "api.cu", "quant_math.cuh"], "sha1": "1e5a40c737e147da",
+                 "bytes_per_algorithmic_byte": 504395093 / 556022622},
 }
 CAPTURED_TRAFFIC_WORKLOAD = ("C5", 32768, "block")
 CAPTURED_TRAFFIC_PROFILE = "profiles/dram_traffic_C5_layer_M32768.md"
@@ -60,7 +62,7 @@ def captured_traffic(kind: str, workload, algorithmic_bytes_per_launch: float) -
     captured layer's DRAM bytes per algorithmic byte times the algorithmic
     bytes of the step's average launch (the GEMM launches of a layer are the
     same in every layer; the quantiser's grouped weight launch covers 56
-    layers' weights in the step and four in the captured layer, so its
+    weights (14 layers) in the step and four in the captured layer, so its
     average launch differs and the ratio carries over)."""
     import hashlib
 
@@ -310,13 +312,18 @@ class LinearStack:
         ws = self.P.puro_fp8_workspace_size(rows_out, cols_out, red)
         return 2 if 0 < ws <= self.workspace.numel() else 1
 
-    def step(self):
+    def step(self, hooks=None):
+        """One step.  `hooks` (the end-to-end measurement) is told when a
+        layer's forward or backward starts, picks each Wgrad's output buffer
+        and is handed each finished dW; the calls made are the same."""
         P, T = self.P, self.timer
         self.launches_per_step = 0
         if self.wtable is not None:
             T.run("quantize", self.wbytes, P.puro_fp8_quantize_weights, self.wtable, P.E4M3)
             self.launches_per_step += -(-self.wtable.count // 64)
         for l in range(self.L):
+            if hooks is not None:
+                hooks.before_forward(l)
             for j, (_, N, K) in enumerate(self.wl.linears):
                 li = self.inputs[l][j]
                 if self.wtable is None:
@@ -327,15 +334,20 @@ class LinearStack:
                       self.y[j], self.workspace)
                 self.launches_per_step += self._gemm_launches(self.M, N, K)
         for l in reversed(range(self.L)):
+            if hooks is not None:
+                hooks.before_backward(l)
             for j in reversed(range(len(self.wl.linears))):
                 _, N, K = self.wl.linears[j]
                 li = self.inputs[l][j]
+                dw = self.dw[j] if hooks is None else hooks.dw(l, j)
                 self._quant(li.dy, P.ROLE_ACT, self.dyq[j], self.grad_fmt)
                 # Dgrad and Wgrad of the linear: one grouped launch when both run unsplit
                 T.run("gemm", 4.0 * self.M * N * K, P.puro_fp8_linear_backward, self.dyq[j].rowwise,
-                      self.wq[l][j].colwise, self.dx[j], self.dyq[j].colwise, self.xqt[l][j], self.dw[j],
+                      self.wq[l][j].colwise, self.dx[j], self.dyq[j].colwise, self.xqt[l][j], dw,
                       self.workspace)
                 self.launches_per_step += self._backward_launches(N, K)
+                if hooks is not None:
+                    hooks.after_backward(l, j, dw)
 
     def flops_per_step(self):
         return self.L * sum(6.0 * self.M * N * K for _, N, K in self.wl.linears)
@@ -719,83 +731,69 @@ def paper_model_measure(P, W, torch, device, scaling, steps=5, warmup=3):
 
 
 def e2e_measure(P, torch, stack, steps):
-    """Same step with host-resident inputs, through the same C ABI calls:
-    every layer's X and dY are copied from pinned host memory into device
-    buffers and every layer's dW is read back to pinned host memory, all
-    inside the timed region.  Copies run on their own streams (H2D, D2H) and
-    overlap the computation; each layer's compute waits for its own inputs,
-    and dW alternates between two device buffer sets so a read-back never
-    races the next layer's Wgrad.  The pinned source holds layer 0's inputs
-    and serves every layer (host memory stays bounded)."""
+    """The same step (the same library calls, through `stack.step`) with
+    host-resident inputs: every layer's X and dY are copied from pinned host
+    memory into device buffers and every layer's dW is read back to pinned
+    host memory, all inside the timed region.  Copies run on their own
+    streams (H2D, D2H) and overlap the computation; each layer's compute
+    waits for its own inputs, and dW alternates between two device buffer
+    sets so a read-back never races a later Wgrad into the same buffer.  The
+    pinned source holds layer 0's inputs and serves every layer (host memory
+    stays bounded); the weights stay resident, as a model's do."""
     comp = torch.cuda.current_stream()
-    n_h2d = 1  # striping over more copy streams measured slower (145 vs 163 GB/s)
-    h2d_s = [torch.cuda.Stream() for _ in range(n_h2d)]
+    h2d_s = torch.cuda.Stream()  # one stream: more measured slower (145 vs 163 GB/s)
     d2h_s = torch.cuda.Stream()
     J = len(stack.wl.linears)
     hx = [li.x.cpu().pin_memory() for li in stack.inputs[0]]
     hdy = [li.dy.cpu().pin_memory() for li in stack.inputs[0]]
     dw_sets = [stack.dw, [torch.empty_like(d) for d in stack.dw]]
     hdw = [[torch.empty(d.shape, dtype=d.dtype).pin_memory() for d in stack.dw] for _ in range(2)]
-    x_ready = [[torch.cuda.Event() for _ in range(n_h2d)] for _ in range(stack.L)]
-    dy_ready = [[torch.cuda.Event() for _ in range(n_h2d)] for _ in range(stack.L)]
-    dw_ready = [torch.cuda.Event() for _ in range(J)]
+    x_ready = [torch.cuda.Event() for _ in range(stack.L)]
+    dy_ready = [torch.cuda.Event() for _ in range(stack.L)]
+    dw_done = [torch.cuda.Event() for _ in range(J)]
     dw_read = [[torch.cuda.Event() for _ in range(J)] for _ in range(2)]
     counts = {"h2d": 0, "d2h": 0}
 
-    def striped_copy(dst, src):
-        """dst (device) <- src (pinned host), split into n_h2d row chunks."""
-        rows = dst.shape[0]
-        step = (rows + n_h2d - 1) // n_h2d
-        for k, st in enumerate(h2d_s):
-            r0, r1 = k * step, min(rows, (k + 1) * step)
-            if r0 < r1:
-                with torch.cuda.stream(st):
-                    dst[r0:r1].copy_(src[r0:r1], non_blocking=True)
-        counts["h2d"] += src.numel() * src.element_size()
+    class Hooks:
+        def before_forward(self, l):
+            comp.wait_event(x_ready[l])
+
+        def before_backward(self, l):
+            comp.wait_event(dy_ready[l])
+
+        def dw(self, l, j):
+            comp.wait_event(dw_read[l % 2][j])  # this buffer's previous read-back is done
+            return dw_sets[l % 2][j]
+
+        def after_backward(self, l, j, dw):
+            dw_done[j].record(comp)
+            d2h_s.wait_event(dw_done[j])
+            with torch.cuda.stream(d2h_s):
+                hdw[l % 2][j].copy_(dw, non_blocking=True)
+            dw_read[l % 2][j].record(d2h_s)
+            counts["d2h"] += dw.numel() * dw.element_size()
+
+    hooks = Hooks()
 
     def one_step():
         counts["h2d"] = counts["d2h"] = 0
         begin = torch.cuda.Event()
         begin.record(comp)
-        for st in h2d_s:
-            st.wait_event(begin)  # nothing is copied before this step starts
-        for l in range(stack.L):
-            for j in range(J):
-                striped_copy(stack.inputs[l][j].x, hx[j])
-            for k, st in enumerate(h2d_s):
-                x_ready[l][k].record(st)
-        for l in reversed(range(stack.L)):
-            for j in range(J):
-                striped_copy(stack.inputs[l][j].dy, hdy[j])
-            for k, st in enumerate(h2d_s):
-                dy_ready[l][k].record(st)
-        for l in range(stack.L):
-            for ev in x_ready[l]:
-                comp.wait_event(ev)
-            for j, (_, N, K) in enumerate(stack.wl.linears):
-                li = stack.inputs[l][j]
-                stack._quant(li.w, P.ROLE_WEIGHT, stack.wq[l][j])
-                stack._quant(li.x, P.ROLE_ACT, P.Quantized(stack.xq[j], stack.xqt[l][j], stack.xamax[j]))
-                P.puro_fp8_linear_fprop(stack.xq[j], stack.wq[l][j].rowwise, stack.y[j], stack.workspace)
-        for l in reversed(range(stack.L)):
-            for ev in dy_ready[l]:
-                comp.wait_event(ev)
-            par = l % 2
-            for j in reversed(range(J)):
-                li = stack.inputs[l][j]
-                stack._quant(li.dy, P.ROLE_ACT, stack.dyq[j])
-                P.puro_fp8_linear_dgrad(stack.dyq[j].rowwise, stack.wq[l][j].colwise, stack.dx[j], stack.workspace)
-                comp.wait_event(dw_read[par][j])  # this buffer's previous read-back is done
-                P.puro_fp8_linear_wgrad(stack.dyq[j].colwise, stack.xqt[l][j], dw_sets[par][j], stack.workspace)
-                dw_ready[j].record(comp)
-                d2h_s.wait_event(dw_ready[j])
-                with torch.cuda.stream(d2h_s):
-                    hdw[par][j].copy_(dw_sets[par][j], non_blocking=True)
-                dw_read[par][j].record(d2h_s)
-                counts["d2h"] += dw_sets[par][j].numel() * dw_sets[par][j].element_size()
+        h2d_s.wait_event(begin)  # nothing is copied before this step starts
+        with torch.cuda.stream(h2d_s):
+            for l in range(stack.L):
+                for j in range(J):
+                    stack.inputs[l][j].x.copy_(hx[j], non_blocking=True)
+                    counts["h2d"] += hx[j].numel() * hx[j].element_size()
+                x_ready[l].record(h2d_s)
+            for l in reversed(range(stack.L)):
+                for j in range(J):
+                    stack.inputs[l][j].dy.copy_(hdy[j], non_blocking=True)
+                    counts["h2d"] += hdy[j].numel() * hdy[j].element_size()
+                dy_ready[l].record(h2d_s)
+        stack.step(hooks)
         comp.wait_stream(d2h_s)
-        for st in h2d_s:
-            comp.wait_stream(st)
+        comp.wait_stream(h2d_s)
 
     stack.timer.enabled = False
     one_step()
@@ -813,7 +811,8 @@ def e2e_measure(P, torch, stack, steps):
             "h2d_bytes_per_step": counts["h2d"], "d2h_bytes_per_step": counts["d2h"],
             "h2d_gbs_effective": h2d_gbs,
             "note": "X and dY of every layer copied from pinned host memory (layer 0's bytes serve every layer) "
-                    "on a copy stream overlapping compute; every layer's dW read back on another"}
+                    "on a copy stream overlapping compute; every layer's dW read back on another; the "
+                    "host-to-device link measured about 200-211 GB/s with nothing else running"}
 
 
 def cpu_baseline(torch, stack, seconds_hint=True):

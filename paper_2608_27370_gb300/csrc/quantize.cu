@@ -24,43 +24,63 @@
 
 namespace puro {
 
+static int sm_count_here() {
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    return sms;
+}
+
 // --------------------------------------------------------------- amax
 // Integer max of (bits & 0x7FFF) over bf16 values: exact for finite values,
-// +inf sorts above them and NaN above +inf.
-__global__ void __launch_bounds__(256) amax_kernel(const uint4 *__restrict__ x, int64_t nvec,
-                                                   const uint16_t *__restrict__ tail, int ntail,
-                                                   uint32_t *__restrict__ out) {
+// +inf sorts above them and NaN above +inf.  A read-only stream: every
+// thread keeps eight 16-byte loads in flight (the remainder, fewer than
+// eight per thread, also in one batch), and the grid is the number of blocks
+// that are resident at once (four per SM at 64 registers), so the
+// grid-stride loop runs in one wave with about 20 MB in flight.
+constexpr int kAmaxThreads = 256;
+constexpr int kAmaxBlocksPerSm = 4;
+constexpr int kAmaxUnroll = 8;
+
+PURO_DEV uint32_t max_abs8(uint32_t m2, const uint4 &v) {
+    return __vmaxu2(m2, __vmaxu2(__vmaxu2(v.x & 0x7FFF7FFFu, v.y & 0x7FFF7FFFu),
+                                 __vmaxu2(v.z & 0x7FFF7FFFu, v.w & 0x7FFF7FFFu)));
+}
+
+__global__ void __launch_bounds__(kAmaxThreads, kAmaxBlocksPerSm)
+    amax_kernel(const uint4 *__restrict__ x, int64_t nvec, const uint16_t *__restrict__ tail, int ntail,
+                uint32_t *__restrict__ out) {
     pdl_wait();
     pdl_launch_dependents();
     uint32_t m2 = 0;  // two packed 16-bit running maxima
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
     int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-    for (; i + 3 * stride < nvec; i += 4 * stride) {
-        uint4 v0 = __ldg(x + i), v1 = __ldg(x + i + stride), v2 = __ldg(x + i + 2 * stride),
-              v3 = __ldg(x + i + 3 * stride);
-        m2 = __vmaxu2(m2, __vmaxu2(__vmaxu2(v0.x & 0x7FFF7FFFu, v0.y & 0x7FFF7FFFu),
-                                   __vmaxu2(v0.z & 0x7FFF7FFFu, v0.w & 0x7FFF7FFFu)));
-        m2 = __vmaxu2(m2, __vmaxu2(__vmaxu2(v1.x & 0x7FFF7FFFu, v1.y & 0x7FFF7FFFu),
-                                   __vmaxu2(v1.z & 0x7FFF7FFFu, v1.w & 0x7FFF7FFFu)));
-        m2 = __vmaxu2(m2, __vmaxu2(__vmaxu2(v2.x & 0x7FFF7FFFu, v2.y & 0x7FFF7FFFu),
-                                   __vmaxu2(v2.z & 0x7FFF7FFFu, v2.w & 0x7FFF7FFFu)));
-        m2 = __vmaxu2(m2, __vmaxu2(__vmaxu2(v3.x & 0x7FFF7FFFu, v3.y & 0x7FFF7FFFu),
-                                   __vmaxu2(v3.z & 0x7FFF7FFFu, v3.w & 0x7FFF7FFFu)));
+    for (; i + (kAmaxUnroll - 1) * stride < nvec; i += kAmaxUnroll * stride) {
+        uint4 v[kAmaxUnroll];
+#pragma unroll
+        for (int k = 0; k < kAmaxUnroll; ++k) v[k] = __ldg(x + i + k * stride);
+#pragma unroll
+        for (int k = 0; k < kAmaxUnroll; ++k) m2 = max_abs8(m2, v[k]);
     }
-    for (; i < nvec; i += stride) {
-        uint4 v = __ldg(x + i);
-        m2 = __vmaxu2(m2, __vmaxu2(__vmaxu2(v.x & 0x7FFF7FFFu, v.y & 0x7FFF7FFFu),
-                                   __vmaxu2(v.z & 0x7FFF7FFFu, v.w & 0x7FFF7FFFu)));
+    {  // fewer than kAmaxUnroll vectors remain per thread: load them together
+        uint4 v[kAmaxUnroll - 1];
+#pragma unroll
+        for (int k = 0; k < kAmaxUnroll - 1; ++k) {
+            const int64_t j = i + k * stride;
+            v[k] = j < nvec ? __ldg(x + j) : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int k = 0; k < kAmaxUnroll - 1; ++k) m2 = max_abs8(m2, v[k]);
     }
     if (blockIdx.x == 0 && threadIdx.x < ntail) m2 = __vmaxu2(m2, tail[threadIdx.x] & 0x7FFFu);
     uint32_t m = max(m2 & 0xFFFFu, m2 >> 16);
     m = __reduce_max_sync(0xFFFFFFFFu, m);
-    __shared__ uint32_t warp_max[8];
+    __shared__ uint32_t warp_max[kAmaxThreads / 32];
     const int warp = threadIdx.x >> 5;
     if ((threadIdx.x & 31) == 0) warp_max[warp] = m;
     __syncthreads();
     if (warp == 0) {
-        m = (threadIdx.x < 8) ? warp_max[threadIdx.x] : 0u;
+        m = (threadIdx.x < kAmaxThreads / 32) ? warp_max[threadIdx.x] : 0u;
         m = __reduce_max_sync(0xFFFFFFFFu, m);
         if (threadIdx.x == 0 && m != 0) atomicMax(out, m);
     }
@@ -71,13 +91,11 @@ cudaError_t launch_amax(const uint16_t *x, int64_t n, uint32_t *amax, cudaStream
     if (e != cudaSuccess || n == 0) return e;
     const int64_t nvec = n / 8;
     const int ntail = static_cast<int>(n - nvec * 8);
-    int dev = 0, sms = 148;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    int64_t want = (nvec + 255) / 256;
-    int64_t cap = static_cast<int64_t>(sms) * 8;
-    int grid = static_cast<int>(want < cap ? (want > 0 ? want : 1) : cap);
-    return launch_pdl(amax_kernel, dim3(grid), dim3(256), 0, s, reinterpret_cast<const uint4 *>(x), nvec,
+    const int sms = sm_count_here();
+    const int64_t want = (nvec + kAmaxThreads - 1) / kAmaxThreads;
+    const int64_t cap = static_cast<int64_t>(sms) * kAmaxBlocksPerSm;
+    const int grid = static_cast<int>(want < cap ? (want > 0 ? want : 1) : cap);
+    return launch_pdl(amax_kernel, dim3(grid), dim3(kAmaxThreads), 0, s, reinterpret_cast<const uint4 *>(x), nvec,
                       x + nvec * 8, ntail, amax);
 }
 
@@ -174,13 +192,6 @@ __global__ void __launch_bounds__(256) rmsnorm_apply_kernel(const uint16_t *__re
         reinterpret_cast<uint4 *>(y)[i] =
             rmsnorm_chunk(__ldg(reinterpret_cast<const uint4 *>(h) + i), __ldg(rstd + r), gm, gamma != nullptr);
     }
-}
-
-static int sm_count_here() {
-    int dev = 0, sms = 148;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    return sms;
 }
 
 cudaError_t launch_rmsnorm_rstd(const uint16_t *h, int64_t rows, int64_t cols, float eps, float *rstd, cudaStream_t s) {

@@ -30,7 +30,9 @@ def _t3(shape, seed, scale=1.0):
 
 
 # ------------------------------------------------------------------ amax
-@pytest.mark.parametrize("n", [0, 1, 7, 8, 9, 1000, 4096 * 33 + 5, 3_000_001])
+# sizes past the eight-load unrolled loop of a full grid (152 SMs x 4 x 256
+# threads x 8 vectors of 8 = 9.96M values) as well as below it
+@pytest.mark.parametrize("n", [0, 1, 7, 8, 9, 1000, 4096 * 33 + 5, 3_000_001, 12_000_007, 41_943_043])
 def test_amax_bit_exact(n):
     x = _t3((n,), 100 + n, 3.0)
     a = torch.full((1,), -1, dtype=torch.int32, device=DEV)
@@ -55,6 +57,19 @@ def test_amax_nonfinite_and_sign():
     P.puro_fp8_amax(x, a)
     torch.cuda.synchronize()
     assert int(host(a)[0]) == O.amax_bf16(bits(x)) > 0x7F80
+
+
+@pytest.mark.parametrize("pos", [0, 9_960_447, 19_999_999, 20_000_000, 20_000_004])
+def test_amax_finds_a_single_maximum_anywhere(pos):
+    # one value above all others at the first element, inside the unrolled
+    # loop's range, in the last whole vector, and in the ragged tail
+    n = 20_000_005
+    x = (torch.rand(n, device=DEV) * 2 - 1).to(torch.bfloat16)
+    x[pos] = -7.5
+    a = torch.zeros(1, dtype=torch.int32, device=DEV)
+    P.puro_fp8_amax(x, a)
+    torch.cuda.synchronize()
+    assert int(host(a)[0]) == 0x40F0  # |-7.5| in bf16
 
 
 # ------------------------------------------------- 1x128 groups (activations)
