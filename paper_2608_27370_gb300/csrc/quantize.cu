@@ -672,6 +672,22 @@ __global__ void __launch_bounds__(kQAThreads, 2)
         }
         __syncthreads();  // (S3) column scales ready, staging free
 
+        // Scale vectors: thread i < 128 writes row i of the rowwise operand
+        // (k-block c0/128), thread 128 + i row i of the transposed operand
+        // (k-block r0/128).  They read the exponents before (S4), so the next
+        // tile's row exponents (written before its (S2), after (S4) here)
+        // cannot overtake them.
+        if (tid < 2 * kQT) {
+            const bool col = tid >= kQT;
+            if (!col || HAS_T) {
+                const int i = tid & (kQT - 1);
+                const int64_t op_rows0 = col ? c0 : r0;
+                const int64_t kb = (col ? r0 : c0) / kQT;
+                const int64_t kblocks = (col ? rows : cols) / kQT;
+                store_scale_vec(col ? scale_t_u8 : scale_u8, op_rows0 + i, kb, kblocks, col ? sm.col_g[i] : sm.row_g[i]);
+            }
+        }
+
         // ---- C: rowwise codes (row i, 4 columns) and transposed codes
         // (column j, 8 rows) from the block, re-read from shared memory.
 #pragma unroll
@@ -729,19 +745,6 @@ __global__ void __launch_bounds__(kQAThreads, 2)
             tma_store_2d(&tm_q, sm.q_stage, static_cast<int32_t>(c0), static_cast<int32_t>(r0));
             if (HAS_T) tma_store_2d(&tm_qt, sm.qt_stage, static_cast<int32_t>(r0), static_cast<int32_t>(c0));
             bulk_commit_group();
-        }
-        // Scale vectors: thread i < 128 writes row i of the rowwise operand
-        // (k-block c0/128), thread 128 + i row i of the transposed operand
-        // (k-block r0/128).
-        if (tid < 2 * kQT) {
-            const bool col = tid >= kQT;
-            if (!col || HAS_T) {
-                const int i = tid & (kQT - 1);
-                const int64_t op_rows0 = col ? c0 : r0;
-                const int64_t kb = (col ? r0 : c0) / kQT;
-                const int64_t kblocks = (col ? rows : cols) / kQT;
-                store_scale_vec(col ? scale_t_u8 : scale_u8, op_rows0 + i, kb, kblocks, col ? sm.col_g[i] : sm.row_g[i]);
-            }
         }
     }
     if (tid == 0) bulk_wait_group0();
