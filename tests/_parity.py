@@ -31,21 +31,43 @@ def bf16_values(t: torch.Tensor) -> np.ndarray:
 # --------------------------------------------------------------------------
 # Running the path
 # --------------------------------------------------------------------------
-def run_linear(x, w, dy, scaling=P.SCALE_BLOCK, fmt_x=P.E4M3, fmt_w=P.E4M3, fmt_g=P.E4M3):
-    """Quantise X, W, dY (rowwise + transposed copies) and run the three GEMMs."""
+def run_linear(x, w, dy, scaling=P.SCALE_BLOCK, fmt_x=P.E4M3, fmt_w=P.E4M3, fmt_g=P.E4M3, step_calls=False):
+    """Quantise X, W, dY (rowwise + transposed copies) and run the three GEMMs.
+
+    With ``step_calls`` the calls are the training step's: a blockwise weight
+    goes through the grouped weight quantiser (puro_fp8_quantize_weights),
+    and Dgrad and Wgrad through puro_fp8_linear_backward with a workspace
+    large enough for any split, so a small-output Wgrad splits its reduction
+    and two unsplit block-scaled GEMMs share one launch.  Otherwise each
+    operand has its own quantise call and each GEMM its own unsplit call."""
     M, K = x.shape
     N = w.shape[0]
     dev = x.device
     xq = P.quantize(x, fmt_x, scaling, P.ROLE_ACT)
-    wq = P.quantize(w, fmt_w, scaling, P.ROLE_WEIGHT)
+    if step_calls and scaling == P.SCALE_BLOCK:
+        u8 = torch.uint8
+        wq = P.Quantized(
+            P.FP8Operand(torch.empty((N, K), dtype=u8, device=dev), P.empty_scales(N, K, scaling, P.ROLE_WEIGHT, dev),
+                         fmt_w, scaling, P.ROLE_WEIGHT),
+            P.FP8Operand(torch.empty((K, N), dtype=u8, device=dev), P.empty_scales(K, N, scaling, P.ROLE_WEIGHT, dev),
+                         fmt_w, scaling, P.ROLE_WEIGHT))
+        P.puro_fp8_quantize_weights([(w, wq)], fmt_w)
+    else:
+        wq = P.quantize(w, fmt_w, scaling, P.ROLE_WEIGHT)
     dyq = P.quantize(dy, fmt_g, scaling, P.ROLE_ACT)
     y = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
     dx = torch.empty((M, K), dtype=torch.bfloat16, device=dev)
     dw = torch.empty((N, K), dtype=torch.bfloat16, device=dev)
     status = torch.zeros(1, dtype=torch.int32, device=dev)
-    P.puro_fp8_linear_fprop(xq.rowwise, wq.rowwise, y, dev_status=status)
-    P.puro_fp8_linear_dgrad(dyq.rowwise, wq.colwise, dx, dev_status=status)
-    P.puro_fp8_linear_wgrad(dyq.colwise, xq.colwise, dw, dev_status=status)
+    if step_calls:
+        ws = torch.empty(max(16, P.puro_fp8_workspace_size(M, N, K), P.puro_fp8_workspace_size(M, K, N),
+                             P.puro_fp8_workspace_size(N, K, M)), dtype=torch.uint8, device=dev)
+        P.puro_fp8_linear_fprop(xq.rowwise, wq.rowwise, y, ws, dev_status=status)
+        P.puro_fp8_linear_backward(dyq.rowwise, wq.colwise, dx, dyq.colwise, xq.colwise, dw, ws, dev_status=status)
+    else:
+        P.puro_fp8_linear_fprop(xq.rowwise, wq.rowwise, y, dev_status=status)
+        P.puro_fp8_linear_dgrad(dyq.rowwise, wq.colwise, dx, dev_status=status)
+        P.puro_fp8_linear_wgrad(dyq.colwise, xq.colwise, dw, dev_status=status)
     torch.cuda.synchronize()
     assert P.puro_fp8_get_status(status) == 0
     return dict(xq=xq, wq=wq, dyq=dyq, y=y, dx=dx, dw=dw)

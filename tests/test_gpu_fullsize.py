@@ -1,5 +1,8 @@
 """GPU parity at the full sizes of the benchmark workloads, in the launch
-configuration the benchmark times.
+configuration the benchmark times: weights through the grouped weight
+quantiser, Dgrad and Wgrad through puro_fp8_linear_backward with a
+workspace (one grouped launch where both are unsplit, a split reduction for
+small-output Wgrads), as in the training step.
 
 C1 (one linear, M=256) is compared element by element in both scaling
 modes.  C2-C6 (C6: the paper's own Qwen3-1.7B-shaped model) use the
@@ -32,7 +35,7 @@ def _lib():
 def test_c1_full(scaling):
     wl = W.WORKLOADS["C1"]
     li = W.make_linear(wl, 0, 0, DEV)
-    out = run_linear(li.x, li.w, li.dy, scaling)
+    out = run_linear(li.x, li.w, li.dy, scaling, step_calls=True)
     if scaling == P.SCALE_TENSOR:
         check_tensor_quant(li.x, out["xq"], P.E4M3)
         check_tensor_quant(li.w, out["wq"], P.E4M3)
@@ -50,7 +53,7 @@ def test_c1_full(scaling):
 def _sampled(key, layer, idx, seed):
     wl = W.WORKLOADS[key]
     li = W.make_linear(wl, layer, idx, DEV)
-    out = run_linear(li.x, li.w, li.dy, P.SCALE_BLOCK)
+    out = run_linear(li.x, li.w, li.dy, P.SCALE_BLOCK, step_calls=True)
     check_linear_sampled(li.x, li.w, li.dy, out, np.random.default_rng(seed))
     del out, li
     torch.cuda.empty_cache()
