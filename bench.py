@@ -693,16 +693,21 @@ def grad_format_measure(P, torch, stack, steps=3, warmup=2):
             "quantize_gbs": q["units"] / q["time_s"] / 1e9}
 
 
-def tensor_scaling_measure(P, W, torch, device, layers=4, steps=3, warmup=2):
+def tensor_scaling_measure(P, W, torch, device, layers=4, steps=3, warmup=2, grad_fmt=None):
     """The C5 step with per-tensor current scaling (the contrast the FP8
     section draws: one scale per tensor, from an amax pass) on `layers` of
     its 28 layers: amax, per-tensor quantise (both copies), and the three
-    FP8 GEMMs with the scale_inv product applied in the epilogue."""
+    FP8 GEMMs with the scale_inv product applied in the epilogue.  With
+    grad_fmt = E5M2 the output gradients are cast to E5M2 (the hybrid
+    recipe: E4M3 forward, E5M2 backward)."""
     wl = W.WORKLOADS["C5"]
     stack = LinearStack(P, W, torch, wl, device, "tensor", layers, wl.M)
+    if grad_fmt is not None:
+        stack.set_grad_format(grad_fmt)
     step_s, per = timed_steps(torch, stack, steps, warmup)
     g, q = per["gemm"], per["quantize"]
-    out = {"workload": f"C5 with per-tensor scaling, {layers} of its 28 layers, M={wl.M}",
+    grads = "E5M2" if grad_fmt == P.E5M2 else "E4M3"
+    out = {"workload": f"C5 with per-tensor scaling, {grads} output gradients, {layers} of its 28 layers, M={wl.M}",
            "value": stack.flops_per_step() / step_s / 1e12, "unit": "TFLOP/s", "ms_per_step": step_s * 1e3,
            "steps": steps, "warmup": warmup, "gemm_only_tflops": g["units"] / g["time_s"] / 1e12,
            "quantize_gbs": q["units"] / q["time_s"] / 1e9,
@@ -1003,6 +1008,7 @@ def main():
         result["muonh_step"] = muonh_measure(P, W, torch, device, peaks)
         if args.scaling == "block":
             result["tensor_scaling"] = tensor_scaling_measure(P, W, torch, device)
+            result["tensor_scaling_e5m2_gradients"] = tensor_scaling_measure(P, W, torch, device, grad_fmt=P.E5M2)
     if rank == 0:
         print(json.dumps(result), flush=True)
     if world > 1:

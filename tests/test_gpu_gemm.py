@@ -72,6 +72,18 @@ def test_tensor_linear(M, N, K):
     assert_close(out["dw"], ref["dw"], "wgrad")
 
 
+@pytest.mark.parametrize("M,N,K", [(256, 1536, 1536), (272, 400, 208)])
+def test_tensor_linear_e5m2_gradients(M, N, K):
+    # the hybrid recipe the FP8 section contrasts with its own: per-tensor
+    # scales, X and W in E4M3, the output gradient in E5M2 (Dgrad and Wgrad
+    # multiply an E5M2 operand by an E4M3 one)
+    x, w, dy = _inputs(M, N, K, 2100 + M + N + K)
+    out = run_linear(x, w, dy, P.SCALE_TENSOR, P.E4M3, P.E4M3, P.E5M2, step_calls=True)
+    ref = oracle_linear(x, w, dy, P.SCALE_TENSOR, P.E4M3, P.E4M3, P.E5M2)
+    for k in ("y", "dx", "dw"):
+        assert_close(out[k], ref[k], k)
+
+
 @pytest.mark.parametrize("M,N,K", [(128, 256, 64), (264, 392, 200), (512, 1536, 1536)])
 def test_bf16_linear(M, N, K):
     x, w, dy = _inputs(M, N, K, 3000 + M)
