@@ -39,6 +39,7 @@ sys.path.insert(0, ROOT)
 METRIC = "FP8 linear fwd+bwd TFLOP/s and % of FP8 peak; quantise HBM GB/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 FP8_PER_BF16 = 2.0  # nominal dense ratio (4.5 / 2.25 PFLOP/s)
+FP8_FLOP_PER_CLK_SM = 16384  # dense FP8 tensor-pipe rate per SM (a 256x256x32 pair MMA per 128 cycles)
 
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per algorithmic
 # byte over the 10 GEMM launches (split reductions included) and the 9
@@ -54,7 +55,6 @@ CAPTURED_TRAFFIC = {
                  "bytes_per_algorithmic_byte": 504278897 / 556022622},
 }
 CAPTURED_TRAFFIC_WORKLOAD = ("C5", 32768, "block")
-CAPTURED_TRAFFIC_PROFILE = "profiles/dram_traffic_C5_layer_M32768.md"
 
 
 def captured_traffic(kind: str, workload, algorithmic_bytes_per_launch: float) -> "int | None":
@@ -190,10 +190,12 @@ class LaunchTimer:
 
     def __init__(self, torch):
         self.torch = torch
-        self.pending = []  # (category, units, start, end)
+        self.pending = []  # (category, label, units, start, end)
         self.enabled = False
+        self.label = None  # what the next run() call is (a shape), for the per-call breakdown
 
     def run(self, cat: str, units: float, fn, *args, **kw):
+        label, self.label = self.label, None
         if not self.enabled:
             return fn(*args, **kw)
         s = self.torch.cuda.Event(enable_timing=True)
@@ -201,17 +203,32 @@ class LaunchTimer:
         s.record()
         fn(*args, **kw)
         e.record()
-        self.pending.append((cat, units, s, e))
+        self.pending.append((cat, label or cat, units, s, e))
 
     def totals(self):
         out = {}
-        for cat, units, s, e in self.pending:
+        for cat, _, units, s, e in self.pending:
             t = s.elapsed_time(e) * 1e-3
             c = out.setdefault(cat, {"time_s": 0.0, "units": 0.0, "launches": 0})
             c["time_s"] += t
             c["units"] += units
             c["launches"] += 1
         return out
+
+    def by_label(self, cat: str, unit_scale: float):
+        """Per labelled call of category `cat`: launches, mean microseconds
+        and units per second (times unit_scale), slowest rate first."""
+        agg = {}
+        for c, label, units, s, e in self.pending:
+            if c != cat:
+                continue
+            a = agg.setdefault(label, [0, 0.0, 0.0])
+            a[0] += 1
+            a[1] += s.elapsed_time(e) * 1e-3
+            a[2] += units
+        rows = [{"call": k, "launches": n, "mean_us": t / n * 1e6, "rate": u / t * unit_scale}
+                for k, (n, t, u) in agg.items()]
+        return sorted(rows, key=lambda r: r["rate"])
 
 
 class LinearStack:
@@ -297,6 +314,7 @@ class LinearStack:
             T.run("amax", 2 * rows * cols, P.puro_fp8_amax, x, q.amax)
             self.launches_per_step += 1
         fmt = P.E4M3 if fmt is None else fmt
+        T.label = f"{'weight' if role == P.ROLE_WEIGHT else 'act'} [{rows}, {cols}]"
         T.run("quantize", self._qbytes(rows, cols, role), P.puro_fp8_quantize, x, fmt, self.scaling, role,
               q.amax if self.scaling == P.SCALE_TENSOR else None, q.rowwise.data, q.rowwise.scale,
               q.colwise.data, q.colwise.scale)
@@ -319,17 +337,19 @@ class LinearStack:
         P, T = self.P, self.timer
         self.launches_per_step = 0
         if self.wtable is not None:
+            T.label = f"all {self.wtable.count} weights, grouped"
             T.run("quantize", self.wbytes, P.puro_fp8_quantize_weights, self.wtable, P.E4M3)
             self.launches_per_step += -(-self.wtable.count // 64)
         for l in range(self.L):
             if hooks is not None:
                 hooks.before_forward(l)
-            for j, (_, N, K) in enumerate(self.wl.linears):
+            for j, (name, N, K) in enumerate(self.wl.linears):
                 li = self.inputs[l][j]
                 if self.wtable is None:
                     self._quant(li.w, P.ROLE_WEIGHT, self.wq[l][j])
                 xq = P.Quantized(self.xq[j], self.xqt[l][j], self.xamax[j])
                 self._quant(li.x, P.ROLE_ACT, xq)
+                T.label = f"fprop {name}"
                 T.run("gemm", 2.0 * self.M * N * K, P.puro_fp8_linear_fprop, self.xq[j], self.wq[l][j].rowwise,
                       self.y[j], self.workspace)
                 self.launches_per_step += self._gemm_launches(self.M, N, K)
@@ -337,11 +357,12 @@ class LinearStack:
             if hooks is not None:
                 hooks.before_backward(l)
             for j in reversed(range(len(self.wl.linears))):
-                _, N, K = self.wl.linears[j]
+                name, N, K = self.wl.linears[j]
                 li = self.inputs[l][j]
                 dw = self.dw[j] if hooks is None else hooks.dw(l, j)
                 self._quant(li.dy, P.ROLE_ACT, self.dyq[j], self.grad_fmt)
                 # Dgrad and Wgrad of the linear: one grouped launch when both run unsplit
+                T.label = f"dgrad+wgrad {name}"
                 T.run("gemm", 4.0 * self.M * N * K, P.puro_fp8_linear_backward, self.dyq[j].rowwise,
                       self.wq[l][j].colwise, self.dx[j], self.dyq[j].colwise, self.xqt[l][j], dw,
                       self.workspace)
@@ -815,9 +836,13 @@ def e2e_measure(P, torch, stack, steps):
     return {"value": stack.flops_per_step() / t / 1e12, "unit": "TFLOP/s", "ms_per_step": t * 1e3,
             "h2d_bytes_per_step": counts["h2d"], "d2h_bytes_per_step": counts["d2h"],
             "h2d_gbs_effective": h2d_gbs,
+            "steps": steps,
             "note": "X and dY of every layer copied from pinned host memory (layer 0's bytes serve every layer) "
-                    "on a copy stream overlapping compute; every layer's dW read back on another; the "
-                    "host-to-device link measured about 200-211 GB/s with nothing else running"}
+                    "on a copy stream overlapping compute; every layer's dW read back on another.  The step's "
+                    "results that leave the device are the weight gradients: Y and dX are activations and "
+                    "activation gradients that the rest of the model (not on this path) consumes on the device, "
+                    "so they are not read back.  The host-to-device link measured about 200-211 GB/s with "
+                    "nothing else running"}
 
 
 def cpu_baseline(torch, stack, seconds_hint=True):
@@ -968,21 +993,30 @@ def main():
                      "peak": fp8_peak_sust, "unit": "TFLOP/s", "frac": gemm_tflops / fp8_peak_sust,
                      "peak_source": f"2 x bf16_tflops_sustained ({peak_src}); kernel timed inside a long step",
                      "traffic": captured_traffic("gemm", traffic_wl, stack.gemm_algorithmic_bytes_per_call()),
-                     "traffic_note": "DRAM bytes per GEMM launch: the captured layer's DRAM bytes per algorithmic byte times the step's average launch, " + CAPTURED_TRAFFIC_PROFILE,
+                     "traffic_note": "DRAM bytes per GEMM launch: DRAM bytes per algorithmic byte from per-kernel ncu captures of one layer's GEMM calls, times the step's average launch",
                      "timing": "CUDA events around each launch of the last timed step, on the launching stream"},
         "roofline_quantize": {"bound": "hbm", "kernel": "quant_act_kernel (X, dY) + quant_weight_group_kernel (W)", "achieved": quant_gbs,
                               "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": quant_gbs / peaks["hbm_gbs"],
                               "peak_source": f"hbm_gbs ({peak_src})",
                               "traffic": captured_traffic("quantize", traffic_wl,
                                                           q["units"] / stack.quantize_kernel_launches_per_step()),
-                              "traffic_note": "DRAM bytes per quantiser launch: the captured layer's DRAM bytes per algorithmic byte times the step's average launch, " +
-                                              CAPTURED_TRAFFIC_PROFILE,
+                              "traffic_note": "DRAM bytes per quantiser launch: DRAM bytes per algorithmic byte from per-kernel ncu captures of one layer's quantiser calls, times the step's average launch",
                               "timing": "CUDA events around each launch of the last timed step, on the launching stream"},
     }
     if args.scaling == "tensor":
         result["roofline"]["kernel"] = "gemm_tn_kernel<FP8 per-tensor>"
+    result["gemm_by_call"] = stack.timer.by_label("gemm", 1e-12)        # rate: TFLOP/s
+    result["quantize_by_call"] = stack.timer.by_label("quantize", 1e-9)  # rate: GB/s (algorithmic)
     if clk:
         result["clocks"] = clk
+        # the tensor pipe's own ceiling at the clock the timed region ran at:
+        # a pair MMA (M 256, N 256, K 32 bytes of FP8) takes 128 cycles, so
+        # 16384 FP8 flop per clock per SM
+        sms = torch.cuda.get_device_properties(device).multi_processor_count
+        clock_peak = FP8_FLOP_PER_CLK_SM * sms * clk["sm_mhz"] * 1e6 / 1e12
+        result["roofline"]["clock_limited_tensor_peak"] = clock_peak
+        result["roofline"]["frac_vs_clock_limited_tensor_peak"] = gemm_tflops / clock_peak
+        result["step_frac_vs_clock_limited_tensor_peak"] = value / world / clock_peak
     if rank == 0 and world == 1 and not args.no_bf16 and args.scaling == "block":
         try:
             result["bf16_comparison"] = bf16_layer_speedup(P, torch, stack)
@@ -991,7 +1025,7 @@ def main():
     if rank == 0 and world == 1 and not args.no_paper_model and args.scaling == "block":
         result["e5m2_gradients"] = grad_format_measure(P, torch, stack)
     if not args.no_e2e:
-        result["e2e"] = e2e_measure(P, torch, stack, max(1, min(args.steps, 3)))
+        result["e2e"] = e2e_measure(P, torch, stack, 5)
         if world > 1:
             ms = max_over_ranks(result["e2e"]["ms_per_step"], world, device)
             result["e2e"]["ms_per_step"] = ms

@@ -8,12 +8,12 @@
  *     Y = X W^T, Dgrad dX = dY W, Wgrad dW = dY^T X -- from FP8 operands,
  *     accumulates in FP32 and writes a BF16 output;
  *   - operands are E4M3; inputs and weights are quantised from BF16
- *     immediately before the GEMM, with scales computed online per local
+ *     just ahead of the GEMM, with scales computed online per local
  *     group: 1x128 groups along the GEMM reduction dimension for activations
  *     and activation gradients, 128x128 blocks for weights;
  *   - each group scale is a power of two (E8M0 expressiveness);
  *   - the quantised input is kept for Wgrad.
- * A per-tensor ("one scale for an entire tensor", the contrast drawn in the
+ * A per-tensor (a single scale per tensor, the contrast drawn in the
  * same section) mode and the E5M2 format are provided as well.
  *
  * Conventions for every entry point
@@ -28,9 +28,11 @@
  *     is enqueued and return PURO_ERR_INVALID_ARG or PURO_ERR_UNSUPPORTED;
  *     a failed launch returns PURO_ERR_CUDA.  No entry point traps or
  *     asserts on the device.  Non-finite data is carried in-band (NaN codes,
- *     E8M0 0xFF, NaN scale_inv).  A GEMM whose pipeline wait exceeds its
- *     internal iteration bound exits cleanly and stores PURO_ERR_TIMEOUT in
- *     *dev_status when dev_status is non-NULL.
+ *     E8M0 0xFF, NaN scale_inv).  A GEMM or quantiser kernel whose wait on
+ *     the device exceeds its bound (puro_set_wait_timeout_ns) stops working
+ *     on its tiles, lets its own copies in flight land, exits cleanly and
+ *     stores PURO_ERR_TIMEOUT in *dev_status when dev_status is non-NULL;
+ *     the outputs of such a call are then incomplete.
  *   - Layout: every tensor is row-major and dense.  A quantised GEMM operand
  *     is stored [rows, red] with the reduction dimension `red` contiguous;
  *     all three GEMMs read both operands this way ("TN"), which is why the
@@ -107,7 +109,7 @@ puro_status_t puro_fp8_amax(const void *x, int64_t rows, int64_t cols,
 /*
  * quantize: BF16 -> FP8 with online scales (section "FP8 Mixed-Precision
  * Training"), optionally emitting the transposed copy that Wgrad consumes
- * (same section: "its quantized input is retained for Wgrad").
+ * (same section: the quantised input is kept for Wgrad).
  *   x        : device [rows, cols] bf16.
  *   fmt      : PURO_E4M3 or PURO_E5M2.
  *   scaling  : PURO_SCALE_BLOCK (the paper's recipe) or PURO_SCALE_TENSOR.
@@ -129,13 +131,15 @@ puro_status_t puro_fp8_amax(const void *x, int64_t rows, int64_t cols,
  * cols % 16 == 0, and rows % 16 == 0 when q_t is requested.  An empty
  * tensor (rows or cols 0) writes no codes, so x, q and q_t may be NULL;
  * in TENSOR mode it still writes scale_inv = 1 (amax of nothing is 0).
+ * dev_status: optional device int32, written only when a tile-load wait on
+ *   the device runs out (PURO_ERR_TIMEOUT); the caller zeroes it.
  */
 puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t cols,
                                 int32_t fmt, int32_t scaling, int32_t role,
                                 const uint32_t *amax_bits,
                                 uint8_t *q, void *scale,
                                 uint8_t *q_t, void *scale_t,
-                                void *stream);
+                                int32_t *dev_status, void *stream);
 
 /*
  * Many weights quantised in one call.
@@ -157,7 +161,7 @@ puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t cols,
  *     none does.
  * fmt: PURO_E4M3 or PURO_E5M2 for all entries.  The table is read on the
  * host during the call (it may be freed on return); every entry is checked
- * before anything is enqueued.
+ * before anything is enqueued.  dev_status: as in puro_fp8_quantize.
  */
 typedef struct {
     const void *w;
@@ -169,7 +173,7 @@ typedef struct {
 } puro_fp8_weight_t;
 
 puro_status_t puro_fp8_quantize_weights(const puro_fp8_weight_t *weights, int32_t count, int32_t fmt,
-                                        void *stream);
+                                        int32_t *dev_status, void *stream);
 
 /*
  * RMSNorm fused ahead of the blockwise activation quantiser.
@@ -187,7 +191,7 @@ puro_status_t puro_fp8_quantize_weights(const puro_fp8_weight_t *weights, int32_
  *   eps >= 0.
  *   rstd: fp32 [rows], written (kept for the RMSNorm backward).
  *   y: bf16 [rows, cols], or NULL: y itself is written only when asked.
- *   q, scale, q_t, scale_t: as in puro_fp8_quantize.
+ *   q, scale, q_t, scale_t, dev_status: as in puro_fp8_quantize.
  * rstd is an fp32 sum of squares in a fixed order, so it agrees with an
  * exact computation to within a few fp32 ulps; y and every code and scale
  * are then exactly determined by rstd.  Two kernels on `stream`; h is read
@@ -195,7 +199,7 @@ puro_status_t puro_fp8_quantize_weights(const puro_fp8_weight_t *weights, int32_
  */
 puro_status_t puro_fp8_quantize_rmsnorm(const void *h, int64_t rows, int64_t cols, const void *gamma, float eps,
                                         int32_t fmt, float *rstd, void *y, uint8_t *q, void *scale, uint8_t *q_t,
-                                        void *scale_t, void *stream);
+                                        void *scale_t, int32_t *dev_status, void *stream);
 
 /*
  * The same RMSNorm without the quantiser: rstd and y (bf16) as above, cols
@@ -222,7 +226,7 @@ puro_status_t puro_rmsnorm_bf16(const void *h, int64_t rows, int64_t cols, const
  *     passed as gate = out, up = out + cols, ld = 2*cols.  16-byte aligned.
  *   rows and cols multiples of 128.
  *   y: bf16 [rows, cols] contiguous, or NULL: written only when asked.
- *   q, scale, q_t, scale_t: as in puro_fp8_quantize.
+ *   q, scale, q_t, scale_t, dev_status: as in puro_fp8_quantize.
  * Every code and scale is an exact function of y.  y itself agrees with the
  * exactly rounded silu(gate) * up to within one bf16 ulp, and equals it for
  * all but about 1e-5 of typical inputs.  One kernel on `stream`; gate and up
@@ -230,7 +234,7 @@ puro_status_t puro_rmsnorm_bf16(const void *h, int64_t rows, int64_t cols, const
  */
 puro_status_t puro_fp8_quantize_swiglu(const void *gate, const void *up, int64_t rows, int64_t cols, int64_t ld,
                                        int32_t fmt, void *y, uint8_t *q, void *scale, uint8_t *q_t, void *scale_t,
-                                       void *stream);
+                                       int32_t *dev_status, void *stream);
 
 /*
  * The same SwiGLU without the quantiser: y (bf16, contiguous [rows, cols]) as
@@ -363,12 +367,17 @@ puro_status_t puro_fp8_linear_wgrad_main_grad(const puro_fp8_tensor_t *dy_t, con
  * (40 MiB) array inside the library's device image, held by every GPU that
  * loads the library until the process exits; no cudaMalloc, cudaFree or
  * allocating library call is made.
- *   - A shape whose split schedule needs more than PURO_NOALLOC_SCRATCH_BYTES
- *     (see puro_fp8_workspace_size) returns PURO_ERR_UNSUPPORTED before any
- *     work is enqueued.
+ *   - Arguments are checked exactly as puro_fp8_linear_wgrad checks them
+ *     (PURO_ERR_INVALID_ARG for a malformed call); then a shape whose split
+ *     schedule needs more than PURO_NOALLOC_SCRATCH_BYTES (see
+ *     puro_fp8_workspace_size) returns PURO_ERR_UNSUPPORTED.  Both before
+ *     any work is enqueued.
  *   - The first call on each device looks up the array's device address
- *     (cudaGetSymbolAddress) with that device current and caches it; make
- *     that first call before any stream capture begins.
+ *     (cudaGetSymbolAddress) with that device current and caches it for the
+ *     life of the process; make that first call before any stream capture
+ *     begins.  The cached address belongs to the device's current context:
+ *     after cudaDeviceReset (or any other teardown of that context) it is
+ *     stale, and this entry point must not be called again in the process.
  *   - All calls share the one array, which keeps the last call's contents.
  *     Nothing in it needs to start at zero: each call writes every scratch
  *     byte before reading it.  Calls whose executions overlap on the GPU

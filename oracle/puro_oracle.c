@@ -26,7 +26,7 @@
  *     Here every product is formed from the dequantised operands and summed
  *     in fp64, in plain k order.
  *   - Per-tensor current scaling (the contrast drawn in the same section:
- *     "one scale for an entire tensor"): scale = fp32(fmt_max / amax),
+ *     a single scale per tensor): scale = fp32(fmt_max / amax),
  *     codes = RNE_sat(fp32(x * scale)), scale_inv = fp32(1 / scale).
  *   - RMSNorm ahead of the quantiser (the model's normalisation before the
  *     attention and MLP projections, section "Model architecture and

@@ -66,10 +66,10 @@ _I64 = ctypes.c_int64
 _I32 = ctypes.c_int32
 _SIGNATURES = {
     "puro_fp8_amax": (_I32, [_P, _I64, _I64, _P, _P]),
-    "puro_fp8_quantize": (_I32, [_P, _I64, _I64, _I32, _I32, _I32, _P, _P, _P, _P, _P, _P]),
-    "puro_fp8_quantize_rmsnorm": (_I32, [_P, _I64, _I64, _P, ctypes.c_float, _I32, _P, _P, _P, _P, _P, _P, _P]),
+    "puro_fp8_quantize": (_I32, [_P, _I64, _I64, _I32, _I32, _I32, _P, _P, _P, _P, _P, _P, _P]),
+    "puro_fp8_quantize_rmsnorm": (_I32, [_P, _I64, _I64, _P, ctypes.c_float, _I32, _P, _P, _P, _P, _P, _P, _P, _P]),
     "puro_rmsnorm_bf16": (_I32, [_P, _I64, _I64, _P, ctypes.c_float, _P, _P, _P]),
-    "puro_fp8_quantize_swiglu": (_I32, [_P, _P, _I64, _I64, _I64, _I32, _P, _P, _P, _P, _P, _P]),
+    "puro_fp8_quantize_swiglu": (_I32, [_P, _P, _I64, _I64, _I64, _I32, _P, _P, _P, _P, _P, _P, _P]),
     "puro_muonh_workspace_size": (ctypes.c_size_t, [_I64]),
     "puro_muonh_reduce": (_I32, [_P, _P, _I64, _P, _P, ctypes.c_size_t, _P]),
     "puro_muonh_apply": (_I32, [_P, _P, _I64, _P, ctypes.c_double, ctypes.c_double, _P, _P]),
@@ -82,7 +82,7 @@ _SIGNATURES = {
     "puro_fp8_linear_wgrad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_dgrad_quantize": (_I32, [_P, _P, _I32, _P, _P, _P, _P, _P, _P, _P]),
     "puro_fp8_linear_backward": (_I32, [_P, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
-    "puro_fp8_quantize_weights": (_I32, [_P, _I32, _I32, _P]),
+    "puro_fp8_quantize_weights": (_I32, [_P, _I32, _I32, _P, _P]),
     "puro_fp8_linear_wgrad_main_grad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_wgrad_noalloc": (_I32, [_P, _P, _P, _P, _P]),
     "puro_fp8_workspace_size": (ctypes.c_size_t, [_I64, _I64, _I64]),
@@ -157,21 +157,23 @@ def puro_fp8_amax(x: torch.Tensor, amax_bits: torch.Tensor, stream=None) -> None
 
 def puro_fp8_quantize(x: torch.Tensor, fmt: int, scaling: int, role: int, amax_bits: Optional[torch.Tensor],
                       q: torch.Tensor, scale: torch.Tensor, q_t: Optional[torch.Tensor] = None,
-                      scale_t: Optional[torch.Tensor] = None, stream=None) -> None:
+                      scale_t: Optional[torch.Tensor] = None, dev_status: Optional[torch.Tensor] = None,
+                      stream=None) -> None:
     rows, cols = x.shape
     u8 = torch.uint8
     sdt = u8 if scaling == SCALE_BLOCK else torch.float32
     st = load_library().puro_fp8_quantize(
         _ptr(x, torch.bfloat16, "x"), rows, cols, fmt, scaling, role,
         _ptr(amax_bits, (torch.int32, torch.uint32), "amax_bits"), _ptr(q, u8, "q"), _ptr(scale, sdt, "scale"),
-        _ptr(q_t, u8, "q_t"), _ptr(scale_t, sdt, "scale_t"), _stream(stream))
+        _ptr(q_t, u8, "q_t"), _ptr(scale_t, sdt, "scale_t"), _ptr(dev_status, torch.int32, "dev_status"),
+        _stream(stream))
     _check("puro_fp8_quantize", st)
 
 
 def puro_fp8_quantize_rmsnorm(h: torch.Tensor, gamma: Optional[torch.Tensor], eps: float, fmt: int,
                               rstd: torch.Tensor, y: Optional[torch.Tensor], q: torch.Tensor, scale: torch.Tensor,
                               q_t: Optional[torch.Tensor] = None, scale_t: Optional[torch.Tensor] = None,
-                              stream=None) -> None:
+                              dev_status: Optional[torch.Tensor] = None, stream=None) -> None:
     """RMSNorm of the rows of h (bf16, optional bf16 gain) fused ahead of the
     blockwise activation quantiser: writes rstd (fp32 [rows]), optionally y
     (bf16), and the codes and scales as puro_fp8_quantize does."""
@@ -180,7 +182,8 @@ def puro_fp8_quantize_rmsnorm(h: torch.Tensor, gamma: Optional[torch.Tensor], ep
     st = load_library().puro_fp8_quantize_rmsnorm(
         _ptr(h, torch.bfloat16, "h"), rows, cols, _ptr(gamma, torch.bfloat16, "gamma"), float(eps), fmt,
         _ptr(rstd, torch.float32, "rstd"), _ptr(y, torch.bfloat16, "y"), _ptr(q, u8, "q"), _ptr(scale, u8, "scale"),
-        _ptr(q_t, u8, "q_t"), _ptr(scale_t, u8, "scale_t"), _stream(stream))
+        _ptr(q_t, u8, "q_t"), _ptr(scale_t, u8, "scale_t"), _ptr(dev_status, torch.int32, "dev_status"),
+        _stream(stream))
     _check("puro_fp8_quantize_rmsnorm", st)
 
 
@@ -224,18 +227,21 @@ def weight_table(entries):
     return table
 
 
-def puro_fp8_quantize_weights(entries, fmt: int = E4M3, stream=None) -> None:
+def puro_fp8_quantize_weights(entries, fmt: int = E4M3, dev_status: Optional[torch.Tensor] = None,
+                              stream=None) -> None:
     """Quantise many weights in 128x128 blocks in one call: entries is a list
     of (w, Quantized) pairs or a table from weight_table().  Same bytes as
     quantize(w, fmt, SCALE_BLOCK, ROLE_WEIGHT, out=q) for each."""
     table = entries if isinstance(entries, ctypes.Array) else weight_table(entries)
-    st = load_library().puro_fp8_quantize_weights(table, table.count, fmt, _stream(stream))
+    st = load_library().puro_fp8_quantize_weights(table, table.count, fmt,
+                                                  _ptr(dev_status, torch.int32, "dev_status"), _stream(stream))
     _check("puro_fp8_quantize_weights", st)
 
 
 def puro_fp8_quantize_swiglu(gate: torch.Tensor, up: torch.Tensor, fmt: int, y: Optional[torch.Tensor],
                              q: torch.Tensor, scale: torch.Tensor, q_t: Optional[torch.Tensor] = None,
-                             scale_t: Optional[torch.Tensor] = None, stream=None) -> None:
+                             scale_t: Optional[torch.Tensor] = None, dev_status: Optional[torch.Tensor] = None,
+                             stream=None) -> None:
     """SwiGLU (silu(gate) * up, bf16) fused ahead of the blockwise activation
     quantiser: writes the codes and scales as puro_fp8_quantize does, and y
     (bf16) only when given.  gate and up may be row-strided views."""
@@ -243,7 +249,8 @@ def puro_fp8_quantize_swiglu(gate: torch.Tensor, up: torch.Tensor, fmt: int, y: 
     u8 = torch.uint8
     st = load_library().puro_fp8_quantize_swiglu(
         g, u, rows, cols, ld, fmt, _ptr(y, torch.bfloat16, "y"), _ptr(q, u8, "q"), _ptr(scale, u8, "scale"),
-        _ptr(q_t, u8, "q_t"), _ptr(scale_t, u8, "scale_t"), _stream(stream))
+        _ptr(q_t, u8, "q_t"), _ptr(scale_t, u8, "scale_t"), _ptr(dev_status, torch.int32, "dev_status"),
+        _stream(stream))
     _check("puro_fp8_quantize_swiglu", st)
 
 
@@ -510,7 +517,8 @@ def puro_fp8_scale_bytes(rows: int, red: int) -> int:
 
 
 def quantize(x: torch.Tensor, fmt: int = E4M3, scaling: int = SCALE_BLOCK, role: int = ROLE_ACT,
-             transpose: bool = True, out: Optional[Quantized] = None, stream=None) -> Quantized:
+             transpose: bool = True, out: Optional[Quantized] = None, dev_status: Optional[torch.Tensor] = None,
+             stream=None) -> Quantized:
     """Quantise x [rows, cols] (bf16) into a rowwise operand [rows, cols] and,
     if ``transpose``, a columnwise operand [cols, rows]; per-tensor mode runs
     the amax kernel first."""
@@ -529,7 +537,7 @@ def quantize(x: torch.Tensor, fmt: int = E4M3, scaling: int = SCALE_BLOCK, role:
         puro_fp8_amax(x, out.amax, stream)
     puro_fp8_quantize(x, fmt, scaling, role, out.amax if scaling == SCALE_TENSOR else None, out.rowwise.data,
                       out.rowwise.scale, out.colwise.data if out.colwise else None,
-                      out.colwise.scale if out.colwise else None, stream)
+                      out.colwise.scale if out.colwise else None, dev_status=dev_status, stream=stream)
     return out
 
 

@@ -330,12 +330,16 @@ puro_status_t fp8_gemm_entry(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t
     return fp8_gemm(a, b, d, workspace, workspace_bytes, dev_status, stream);
 }
 
+puro_status_t fp8_gemm_validate(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, const void *d) {
+    return validate_fp8_gemm(a, b, d);
+}
+
 }  // namespace puro
 
 using namespace puro;
 
 PURO_API puro_status_t puro_fp8_quantize_weights(const puro_fp8_weight_t *weights, int32_t count, int32_t fmt,
-                                                 void *stream) {
+                                                 int32_t *dev_status, void *stream) {
     if (count < 0 || (count > 0 && !weights) || !valid_fmt(fmt)) return PURO_ERR_INVALID_ARG;
     if (count == 0) return PURO_OK;
     bool has_t = false;  // from the first non-empty entry; empty entries are skipped unchecked
@@ -356,6 +360,8 @@ PURO_API puro_status_t puro_fp8_quantize_weights(const puro_fp8_weight_t *weight
     }
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     static thread_local WeightGroup g;  // 26 KB: kept off the stack
+    g.status = dev_status;
+    g.wait_ns = g_wait_timeout_ns.load();
     int32_t i = 0;
     while (i < count) {
         g.count = 0;
@@ -404,7 +410,7 @@ PURO_API puro_status_t puro_fp8_amax(const void *x, int64_t rows, int64_t cols, 
 
 PURO_API puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t cols, int32_t fmt, int32_t scaling,
                                          int32_t role, const uint32_t *amax_bits, uint8_t *q, void *scale,
-                                         uint8_t *q_t, void *scale_t, void *stream) {
+                                         uint8_t *q_t, void *scale_t, int32_t *dev_status, void *stream) {
     if (!valid_fmt(fmt) || rows < 0 || cols < 0) return PURO_ERR_INVALID_ARG;
     if ((q_t == nullptr) != (scale_t == nullptr) && scaling == PURO_SCALE_BLOCK) return PURO_ERR_INVALID_ARG;
     const bool has_t = q_t != nullptr;
@@ -413,6 +419,8 @@ PURO_API puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t co
     a.rows = rows;
     a.cols = cols;
     a.has_t = has_t;
+    a.status = dev_status;
+    a.wait_ns = g_wait_timeout_ns.load();
     if (scaling == PURO_SCALE_BLOCK) {
         if (role != PURO_ROLE_ACT && role != PURO_ROLE_WEIGHT) return PURO_ERR_INVALID_ARG;
         if (amax_bits != nullptr) return PURO_ERR_INVALID_ARG;
@@ -465,7 +473,7 @@ PURO_API puro_status_t puro_fp8_quantize(const void *x, int64_t rows, int64_t co
 // activation quantiser; see the header.
 PURO_API puro_status_t puro_fp8_quantize_rmsnorm(const void *h, int64_t rows, int64_t cols, const void *gamma,
                                                  float eps, int32_t fmt, float *rstd, void *y, uint8_t *q, void *scale,
-                                                 uint8_t *q_t, void *scale_t, void *stream) {
+                                                 uint8_t *q_t, void *scale_t, int32_t *dev_status, void *stream) {
     if (!valid_fmt(fmt) || rows < 0 || cols < 0 || !(eps >= 0.0f)) return PURO_ERR_INVALID_ARG;
     if (rows % 128 || cols % 128) return PURO_ERR_INVALID_ARG;
     if ((q_t == nullptr) != (scale_t == nullptr)) return PURO_ERR_INVALID_ARG;
@@ -484,6 +492,8 @@ PURO_API puro_status_t puro_fp8_quantize_rmsnorm(const void *h, int64_t rows, in
     a.kind = kQuantBlockAct;
     a.scale_u8 = static_cast<uint8_t *>(scale);
     a.scale_t_u8 = static_cast<uint8_t *>(scale_t);
+    a.status = dev_status;
+    a.wait_ns = g_wait_timeout_ns.load();
     a.x = static_cast<const uint16_t *>(h);
     CUtensorMap tm_x, tm_q, tm_qt, tm_y;
     if (!make_map(&tm_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h, cols, rows, cols * 2, 128, 128,
@@ -507,7 +517,7 @@ PURO_API puro_status_t puro_fp8_quantize_rmsnorm(const void *h, int64_t rows, in
 // SwiGLU fused ahead of the activation quantiser.
 PURO_API puro_status_t puro_fp8_quantize_swiglu(const void *gate, const void *up, int64_t rows, int64_t cols,
                                                 int64_t ld, int32_t fmt, void *y, uint8_t *q, void *scale,
-                                                uint8_t *q_t, void *scale_t, void *stream) {
+                                                uint8_t *q_t, void *scale_t, int32_t *dev_status, void *stream) {
     if (!valid_fmt(fmt) || rows < 0 || cols < 0 || ld < cols || ld % 8) return PURO_ERR_INVALID_ARG;
     if (rows % 128 || cols % 128) return PURO_ERR_INVALID_ARG;
     if ((q_t == nullptr) != (scale_t == nullptr)) return PURO_ERR_INVALID_ARG;
@@ -526,6 +536,8 @@ PURO_API puro_status_t puro_fp8_quantize_swiglu(const void *gate, const void *up
     a.kind = kQuantBlockAct;
     a.scale_u8 = static_cast<uint8_t *>(scale);
     a.scale_t_u8 = static_cast<uint8_t *>(scale_t);
+    a.status = dev_status;
+    a.wait_ns = g_wait_timeout_ns.load();
     a.x = static_cast<const uint16_t *>(gate);
     CUtensorMap tm_x, tm_q, tm_qt, tm_y;
     if (!make_map(&tm_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, gate, cols, rows, ld * 2, 128, 128,

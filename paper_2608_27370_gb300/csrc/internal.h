@@ -48,6 +48,8 @@ struct QuantArgs {
     float *scale_f;           // tensor scale_inv for q
     float *scale_t_f;         // tensor scale_inv for q_t (may be null)
     bool has_t;
+    int32_t *status;          // optional device status word (PURO_ERR_TIMEOUT when a tile load is given up)
+    uint64_t wait_ns;         // bound on each tile-load wait
 };
 
 cudaError_t launch_amax(const uint16_t *x, int64_t n, uint32_t *amax, cudaStream_t s);
@@ -64,6 +66,8 @@ struct WeightGroup {
     int tiles_n[kWeightGroupMax];         // column tiles of each weight (cols / 128)
     int kb_rows[kWeightGroupMax];         // rows / 128 (k-blocks of the transposed copy)
     int count;
+    int32_t *status;                      // optional device status word
+    uint64_t wait_ns;                     // bound on each tile-load wait
 };
 cudaError_t launch_quantize_weights(const WeightGroup &g, int fmt, bool has_t, cudaStream_t s);
 
@@ -185,6 +189,9 @@ cudaError_t launch_gemm_grouped(const GemmArgs &g0, const GemmMaps &m0, const Ge
 // encodes the tensor maps and launches (D = A * B^T).
 puro_status_t fp8_gemm_entry(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, void *d, void *workspace,
                              size_t workspace_bytes, int32_t *dev_status, void *stream);
+
+// The host-side argument checks of fp8_gemm_entry alone (no CUDA call).
+puro_status_t fp8_gemm_validate(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, const void *d);
 
 // Split count the GEMM uses for a shape (1: no split), and the workspace it
 // then needs.  Host-only, shape-only (plans for 152 SMs).

@@ -28,7 +28,8 @@ void *g_scratch_ptr[kMaxDevices] = {};
 // Device address of g_wgrad_scratch on the current device.  In host code
 // the array's name is only a host-side stand-in for the symbol, so the real
 // device address is looked up once per device (with that device current)
-// and cached.
+// and cached for the life of the process: after cudaDeviceReset the cached
+// address is stale (the header says so).
 cudaError_t scratch_address(void **out) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -52,9 +53,11 @@ using namespace puro;
 
 extern "C" __attribute__((visibility("default"))) puro_status_t puro_fp8_linear_wgrad_noalloc(
     const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t, void *dw, int32_t *dev_status, void *stream) {
-    if (!dy_t || !x_t) return PURO_ERR_INVALID_ARG;
-    if (dy_t->rows < 0 || x_t->rows < 0 || dy_t->red < 0) return PURO_ERR_INVALID_ARG;
-    // The split schedule this shape would take must fit the fixed scratch.
+    // The regular Wgrad's argument checks first, so a malformed call is
+    // reported as such whatever its shape; then the split schedule this
+    // shape would take must fit the fixed scratch.
+    const puro_status_t st = fp8_gemm_validate(dy_t, x_t, dw);
+    if (st != PURO_OK) return st;
     const size_t need = splitk_workspace_bytes(dy_t->rows, x_t->rows, dy_t->red, false);
     if (need > PURO_NOALLOC_SCRATCH_BYTES) return PURO_ERR_UNSUPPORTED;
     void *scratch = nullptr;

@@ -295,7 +295,35 @@ struct QuantSmem {
     uint64_t full[2];                            // TMA tile loads into in[0], in[1]
 };
 
-constexpr uint64_t kQuantWaitNs = 2000000000ull;  // a TMA load always lands long before this
+constexpr uint64_t kQuantDrainNs = 2000000000ull;  // after an abort: bound on the loads still in flight
+constexpr uint64_t kPollBelowNs = 100000ull;       // shorter bounds are polled without suspending
+constexpr int32_t kQuantStatusTimeout = 4;         // PURO_ERR_TIMEOUT
+
+// Wait for a tile load, bounded by the library's wait bound
+// (puro_set_wait_timeout_ns).  A bound under 100 us is polled with the
+// non-blocking test, so that a short bound is kept even where one
+// suspending try_wait would sleep until the copy lands; a zero bound is a
+// single test (it does not depend on the timer's resolution).
+PURO_DEV bool tile_landed(uint64_t *bar, uint32_t parity, uint64_t wait_ns) {
+    if (wait_ns >= kPollBelowNs) return mbar_wait_bounded(bar, parity, wait_ns);
+    if (mbar_test_wait(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    while (global_timer_ns() - t0 < wait_ns)
+        if (mbar_test_wait(bar, parity)) return true;
+    return false;
+}
+
+// A CTA gave up on the load of its tile `it` (every thread leaves the tile
+// loop together, after a block-wide vote): record the time-out, then let
+// the loads it still has in flight (this tile's and, when issued, the next
+// one's) land before it exits, since they write into its shared memory.
+// The drain is bounded too.  One thread.
+PURO_DEV void quant_abort(uint64_t *full, int it, bool next_issued, int32_t *status) {
+    if (status) atomicExch(status, kQuantStatusTimeout);
+    const int buf = it & 1;
+    mbar_wait_bounded(&full[buf], static_cast<uint32_t>(it >> 1) & 1u, kQuantDrainNs);
+    if (next_issued) mbar_wait_bounded(&full[buf ^ 1], static_cast<uint32_t>((it + 1) >> 1) & 1u, kQuantDrainNs);
+}
 
 
 // Rowwise codes (row i, 8 columns) and transposed codes (column j, 8 rows)
@@ -360,7 +388,8 @@ __global__ void __launch_bounds__(kQThreads, 2)
     quant_tile_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_q,
                       const __grid_constant__ CUtensorMap tm_qt, int64_t rows, int64_t cols,
                       uint8_t *__restrict__ scale_u8, uint8_t *__restrict__ scale_t_u8, float *scale_f,
-                      float *scale_t_f, const uint32_t *__restrict__ amax_bits, int tiles_n, int ntiles) {
+                      float *scale_t_f, const uint32_t *__restrict__ amax_bits, int tiles_n, int ntiles,
+                      int32_t *status, uint64_t wait_ns) {
     static_assert(KIND == kQuantBlockWeight || KIND == kQuantTensor, "activations use quant_act_kernel");
     extern __shared__ uint8_t smem_raw[];
     QuantSmem &sm = *reinterpret_cast<QuantSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -415,9 +444,15 @@ __global__ void __launch_bounds__(kQThreads, 2)
             if constexpr (KIND == kQuantTensor) bulk_wait_group_read0();
         }
         // Every thread waits on the tile's barrier itself, which makes the
-        // TMA-written tile visible to it.
-        mbar_wait_bounded(&sm.full[buf], static_cast<uint32_t>(it >> 1) & 1u, kQuantWaitNs);
-        if constexpr (KIND == kQuantTensor) __syncthreads();  // (S1) staging free
+        // TMA-written tile visible to it.  A wait that runs out is voted on
+        // at the next barrier, where every thread leaves together.
+        const bool landed = tile_landed(&sm.full[buf], static_cast<uint32_t>(it >> 1) & 1u, wait_ns);
+        if constexpr (KIND == kQuantTensor) {
+            if (__syncthreads_or(!landed)) {  // (S1) staging free
+                if (tid == 0) quant_abort(sm.full, it, tile + static_cast<int>(gridDim.x) < ntiles, status);
+                break;
+            }
+        }
 
         // ---- the thread's 8x8 block: v[i] = row 8br+i, columns 8bc .. 8bc+7
         const uint16_t *in = sm.in[buf];
@@ -435,7 +470,10 @@ __global__ void __launch_bounds__(kQThreads, 2)
             m = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
             if (lane == 0) sm.red[warp] = m;
             if (tid == 0) bulk_wait_group_read0();  // staging free (see above)
-            __syncthreads();                         // (S2) block maxima written, staging free
+            if (__syncthreads_or(!landed)) {         // (S2) block maxima written, staging free
+                if (tid == 0) quant_abort(sm.full, it, tile + static_cast<int>(gridDim.x) < ntiles, status);
+                break;
+            }
             m = __reduce_max_sync(0xFFFFFFFFu, sm.red[lane & 7]);
             blk_g = e8m0_exponent<FMT>(m);
             mul = mul_of(blk_g);
@@ -529,7 +567,7 @@ __global__ void __launch_bounds__(kQAThreads, 2)
     quant_act_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_q,
                      const __grid_constant__ CUtensorMap tm_qt, const __grid_constant__ CUtensorMap tm_y,
                      int64_t rows, int64_t cols, uint8_t *__restrict__ scale_u8, uint8_t *__restrict__ scale_t_u8,
-                     ProdArgs prod, int tiles_n, int ntiles) {
+                     ProdArgs prod, int tiles_n, int ntiles, int32_t *status, uint64_t wait_ns) {
     extern __shared__ uint8_t smem_raw[];
     QuantActSmem &sm = *reinterpret_cast<QuantActSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                          ~static_cast<uintptr_t>(1023));
@@ -578,8 +616,9 @@ __global__ void __launch_bounds__(kQAThreads, 2)
         }
         // Every thread waits on the tile's barrier itself (which makes the
         // TMA-written tile visible to it); the shared buffers written before
-        // (S2) were last read before (S4) of the previous tile.
-        mbar_wait_bounded(&sm.full[buf], static_cast<uint32_t>(it >> 1) & 1u, kQuantWaitNs);
+        // (S2) were last read before (S4) of the previous tile.  A wait that
+        // runs out is voted on at (S2): nothing global is written before it.
+        const bool landed = tile_landed(&sm.full[buf], static_cast<uint32_t>(it >> 1) & 1u, wait_ns);
 
         uint16_t *in = sm.in[buf];
         uint2 v[8];
@@ -641,7 +680,10 @@ __global__ void __launch_bounds__(kQAThreads, 2)
             }
             *reinterpret_cast<uint2 *>(&sm.col_part[br][2 * bc]) = cm;
         }
-        __syncthreads();  // (S2) partials and row scales written
+        if (__syncthreads_or(!landed)) {  // (S2) partials and row scales written
+            if (tid == 0) quant_abort(sm.full, it, tile + static_cast<int>(gridDim.x) < ntiles, status);
+            break;
+        }
         if constexpr (PROD != kProdNone) {
             if (prod.write_y && tid == 0) {  // every block's y is in shared memory
                 tma_store_2d(&tm_y, sm.in[buf], static_cast<int32_t>(c0), static_cast<int32_t>(r0));
@@ -801,7 +843,7 @@ __global__ void __launch_bounds__(kQThreads, 2) quant_weight_group_kernel(const 
             const int next = tile + gridDim.x;
             if (next < ntiles) issue_load(next, locate(next, w), buf ^ 1);  // buffer last read before (S3) of it-1
         }
-        mbar_wait_bounded(&sm.full[buf], static_cast<uint32_t>(it >> 1) & 1u, kQuantWaitNs);
+        const bool landed = tile_landed(&sm.full[buf], static_cast<uint32_t>(it >> 1) & 1u, g.wait_ns);
 
         const uint16_t *in = sm.in[buf];
         uint4 v[8];
@@ -813,7 +855,10 @@ __global__ void __launch_bounds__(kQThreads, 2) quant_weight_group_kernel(const 
         m = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
         if (lane == 0) sm.red[warp] = m;
         if (tid == 0) bulk_wait_group_read0();  // the previous tile's stores have read the staging
-        __syncthreads();                         // (S2) block maxima written, staging free
+        if (__syncthreads_or(!landed)) {         // (S2) block maxima written, staging free
+            if (tid == 0) quant_abort(sm.full, it, tile + static_cast<int>(gridDim.x) < ntiles, g.status);
+            break;
+        }
         m = __reduce_max_sync(0xFFFFFFFFu, sm.red[lane & 7]);
         const uint32_t blk_g = e8m0_exponent<FMT>(m);
         const float mul = mul_of(blk_g);
@@ -883,7 +928,7 @@ static cudaError_t launch_quant_t(const QuantArgs &a, const CUtensorMap &tm_x, c
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
         const int grid = ntiles < 2 * sms ? ntiles : 2 * sms;  // persistent: two CTAs per SM
         return launch_pdl(kern, dim3(grid), dim3(kQAThreads), smem, s, tm_x, tm_q, tm_qt, tm_y ? *tm_y : tm_x, a.rows,
-                          a.cols, a.scale_u8, a.scale_t_u8, prod, tiles_n, ntiles);
+                          a.cols, a.scale_u8, a.scale_t_u8, prod, tiles_n, ntiles, a.status, a.wait_ns);
     } else {
         static_assert(PROD == kProdNone, "producers feed the activation quantiser");
         auto kern = quant_tile_kernel<FMT, KIND, HAS_T>;
@@ -898,7 +943,7 @@ static cudaError_t launch_quant_t(const QuantArgs &a, const CUtensorMap &tm_x, c
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
         const int grid = ntiles < 2 * sms ? ntiles : 2 * sms;  // persistent: two CTAs per SM
         return launch_pdl(kern, dim3(grid), dim3(kQThreads), smem, s, tm_x, tm_q, tm_qt, a.rows, a.cols, a.scale_u8,
-                          a.scale_t_u8, a.scale_f, a.scale_t_f, a.amax, tiles_n, ntiles);
+                          a.scale_t_u8, a.scale_f, a.scale_t_f, a.amax, tiles_n, ntiles, a.status, a.wait_ns);
     }
 }
 

@@ -8,11 +8,57 @@ tensor-core scale vectors are plain index permutations.
 """
 from __future__ import annotations
 
+import os
+from concurrent.futures import ThreadPoolExecutor
+
 import numpy as np
 import torch
 
 import oracle as O
 import paper_2608_27370_gb300 as P
+
+
+# Host threads for the oracle at full size.  The oracle's ctypes calls
+# release the GIL, so bands of a tensor are quantised in parallel threads;
+# every quantisation group lies inside one band (bands are cut along the
+# other axis, or at multiples of 128), so the result is exactly the single
+# call's.
+NTHREADS = max(1, min(32, os.cpu_count() or 1))
+
+
+def _bands(n: int, align: int) -> list:
+    """Split range(n) into about NTHREADS bands whose starts are multiples of align."""
+    units = max(1, -(-n // align))
+    per = max(1, -(-units // NTHREADS))
+    return [(a * align, min(n, (a + per) * align)) for a in range(0, units, per)]
+
+
+def par_quantize_rows_1x128(xb: np.ndarray, fmt: int):
+    """O.quantize_rows_1x128 on bands of rows (each row's groups stay whole)."""
+    bands = _bands(xb.shape[0], 1)
+    with ThreadPoolExecutor(len(bands)) as ex:
+        parts = list(ex.map(lambda b: O.quantize_rows_1x128(xb[b[0]:b[1]], fmt), bands))
+    return np.concatenate([p[0] for p in parts]), np.concatenate([p[1] for p in parts])
+
+
+def par_quantize_cols_128x1(xb: np.ndarray, fmt: int):
+    """O.quantize_cols_128x1 on bands of columns (each column's groups stay whole)."""
+    bands = _bands(xb.shape[1], 1)
+    with ThreadPoolExecutor(len(bands)) as ex:
+        parts = list(ex.map(lambda b: O.quantize_cols_128x1(np.ascontiguousarray(xb[:, b[0]:b[1]]), fmt), bands))
+    return np.concatenate([p[0] for p in parts]), np.concatenate([p[1] for p in parts])
+
+
+def par_quantize_blocks_128x128(wb: np.ndarray, fmt: int):
+    """O.quantize_blocks_128x128 on bands of whole 128-row blocks."""
+    bands = _bands(wb.shape[0], 128)
+    with ThreadPoolExecutor(len(bands)) as ex:
+        parts = list(ex.map(lambda b: O.quantize_blocks_128x128(wb[b[0]:b[1]], fmt), bands))
+    return np.concatenate([p[0] for p in parts]), np.concatenate([p[1] for p in parts])
+
+
+def par_gemm_tn(a: np.ndarray, b: np.ndarray) -> np.ndarray:
+    return O.gemm_tn(a, b, NTHREADS)
 
 
 def bits(t: torch.Tensor) -> np.ndarray:
@@ -128,7 +174,7 @@ def check_block_act_quant(x: torch.Tensor, q: P.Quantized, fmt: int, rows=None, 
     """Bit-exact check of a 1x128 quantisation (rowwise + transposed copy).
     rows/cols: optional index subsets (full-size sampling)."""
     xb = bits(x if rows is None else x[rows])
-    q_ref, s_ref = O.quantize_rows_1x128(xb, fmt)
+    q_ref, s_ref = par_quantize_rows_1x128(xb, fmt)
     qr = q.rowwise.data if rows is None else q.rowwise.data[rows]
     assert_bytes(qr, q_ref, "rowwise codes")
     if rows is None:  # the whole buffer, padding bytes included
@@ -137,8 +183,8 @@ def check_block_act_quant(x: torch.Tensor, q: P.Quantized, fmt: int, rows=None, 
         assert np.array_equal(scales_of(q.rowwise)[host(rows)], s_ref), "rowwise scales (sampled rows)"
     if q.colwise is None:
         return
-    xc = bits(x if cols is None else x[:, cols])
-    qt_ref, st_ref = O.quantize_cols_128x1(xc, fmt)
+    xc = xb if (rows is None and cols is None) else bits(x if cols is None else x[:, cols])
+    qt_ref, st_ref = par_quantize_cols_128x1(xc, fmt)
     qc = q.colwise.data if cols is None else q.colwise.data[cols]
     assert_bytes(qc, qt_ref, "transposed codes")
     if cols is None:
@@ -148,7 +194,7 @@ def check_block_act_quant(x: torch.Tensor, q: P.Quantized, fmt: int, rows=None, 
 
 
 def check_block_weight_quant(w: torch.Tensor, q: P.Quantized, fmt: int):
-    q_ref, s_ref = O.quantize_blocks_128x128(bits(w), fmt)
+    q_ref, s_ref = par_quantize_blocks_128x128(bits(w), fmt)
     assert_bytes(q.rowwise.data, q_ref, "weight codes")
     assert_bytes(q.rowwise.scale, to_scale_vec(np.repeat(s_ref, 128, axis=0)), "weight scale vectors")
     if q.colwise is not None:
@@ -186,10 +232,17 @@ def sample_index(n: int, k_rand: int, rng: np.random.Generator) -> np.ndarray:
     return np.unique(idx)
 
 
-def check_linear_sampled(x, w, dy, out, rng, k_rand=64, fmt=P.E4M3, nthreads=16):
-    """Blockwise recipe at full size: quantised bytes on sampled rows/columns,
-    GEMM outputs on the cross product of sampled rows and columns (which
-    contains the four corner 128x128 tiles)."""
+def check_linear_sampled(x, w, dy, out, rng, k_rand=96, fmt=P.E4M3, full_bytes=False):
+    """Blockwise recipe at full size.
+
+    Quantised bytes: with ``full_bytes`` every FP8 byte and scale of X, W and
+    dY (both copies) against the oracle; otherwise W in full and X, dY on
+    sampled rows and columns (the first and last 128 and k_rand random ones).
+    GEMM outputs: the cross product of sampled rows and columns of each
+    output -- the first 128, the last 128 and k_rand random indices of each
+    dimension -- which holds the four complete corner 128x128 tiles and
+    k_rand^2 seeded random (m, n) entries (9216 at the default 96), against
+    the oracle's fp64 products of the same operands."""
     M, K = x.shape
     N = w.shape[0]
     Ms = sample_index(M, k_rand, rng)
@@ -197,9 +250,13 @@ def check_linear_sampled(x, w, dy, out, rng, k_rand=64, fmt=P.E4M3, nthreads=16)
     Ks = sample_index(K, k_rand, rng)
     Ms_t, Ns_t, Ks_t = (torch.from_numpy(a).to(x.device) for a in (Ms, Ns, Ks))
 
-    # quantised operands: X rows Ms / columns Ks, dY rows Ms / columns Ns, all of W
-    check_block_act_quant(x, out["xq"], fmt, rows=Ms_t, cols=Ks_t)
-    check_block_act_quant(dy, out["dyq"], fmt, rows=Ms_t, cols=Ns_t)
+    # quantised operands
+    if full_bytes:
+        check_block_act_quant(x, out["xq"], fmt)
+        check_block_act_quant(dy, out["dyq"], fmt)
+    else:
+        check_block_act_quant(x, out["xq"], fmt, rows=Ms_t, cols=Ks_t)
+        check_block_act_quant(dy, out["dyq"], fmt, rows=Ms_t, cols=Ns_t)
     check_block_weight_quant(w, out["wq"], fmt)
 
     # oracle operands for the sampled products
@@ -207,16 +264,41 @@ def check_linear_sampled(x, w, dy, out, rng, k_rand=64, fmt=P.E4M3, nthreads=16)
     X_rows = O.dequant_rows_1x128(xr_q, xr_s, fmt)
     dyr_q, dyr_s = O.quantize_rows_1x128(bits(dy[Ms_t]), fmt)         # dY rows (groups along N)
     dY_rows = O.dequant_rows_1x128(dyr_q, dyr_s, fmt)
-    wq, ws = O.quantize_blocks_128x128(bits(w), fmt)                  # W blocks
+    wq, ws = par_quantize_blocks_128x128(bits(w), fmt)                # W blocks
     W = O.dequant_blocks_128x128(wq, ws, fmt)
-    xc_q, xc_s = O.quantize_cols_128x1(bits(x[:, Ks_t]), fmt)         # X columns (groups along M)
+    xc_q, xc_s = par_quantize_cols_128x1(bits(x[:, Ks_t]), fmt)       # X columns (groups along M)
     Xt_rows = O.dequant_rows_1x128(xc_q, xc_s, fmt)
-    dyc_q, dyc_s = O.quantize_cols_128x1(bits(dy[:, Ns_t]), fmt)      # dY columns (groups along M)
+    dyc_q, dyc_s = par_quantize_cols_128x1(bits(dy[:, Ns_t]), fmt)    # dY columns (groups along M)
     dYt_rows = O.dequant_rows_1x128(dyc_q, dyc_s, fmt)
 
-    y_ref = O.gemm_tn(X_rows, W[Ns], nthreads)                         # Y[Ms, Ns]
-    dx_ref = O.gemm_tn(dY_rows, np.ascontiguousarray(W.T[Ks]), nthreads)  # dX[Ms, Ks]
-    dw_ref = O.gemm_tn(dYt_rows, Xt_rows, nthreads)                    # dW[Ns, Ks]
+    y_ref = par_gemm_tn(X_rows, W[Ns])                                 # Y[Ms, Ns]
+    dx_ref = par_gemm_tn(dY_rows, np.ascontiguousarray(W.T[Ks]))       # dX[Ms, Ks]
+    dw_ref = par_gemm_tn(dYt_rows, Xt_rows)                            # dW[Ns, Ks]
     assert_close(out["y"][Ms_t][:, Ns_t], y_ref, "fprop (sampled)")
     assert_close(out["dx"][Ms_t][:, Ks_t], dx_ref, "dgrad (sampled)")
     assert_close(out["dw"][Ns_t][:, Ks_t], dw_ref, "wgrad (sampled)")
+
+
+# --------------------------------------------------------------------------
+# Output coverage of a persistent GEMM: one sampled index in every 32
+# consecutive rows / columns, so the cross product meets every 32 x 32 piece
+# of every output tile (each epilogue warp's lane quarter and column chunk,
+# both CTAs of a pair, both accumulator buffers).
+# --------------------------------------------------------------------------
+def sample_every(n: int, rng: np.random.Generator, group: int = 32) -> np.ndarray:
+    """One random index in each run of `group` consecutive indices of range(n)
+    (the last run may be short), plus the first and last index."""
+    starts = np.arange(0, n, group)
+    picks = starts + rng.integers(0, np.minimum(group, n - starts))
+    return np.unique(np.concatenate([picks, [0, n - 1]]))
+
+
+def check_gemm_every_tile(out: torch.Tensor, a: np.ndarray, b: np.ndarray, rng: np.random.Generator, what: str):
+    """out [M, N] (bf16, device) against the fp64 product a[rows] . b[cols]^T
+    on the cross product of sample_every rows and columns; a [M, K] and b
+    [N, K] are the oracle's dequantised operands (fp64)."""
+    rows = sample_every(out.shape[0], rng)
+    cols = sample_every(out.shape[1], rng)
+    ref = par_gemm_tn(np.ascontiguousarray(a[rows]), np.ascontiguousarray(b[cols]))
+    r_t, c_t = (torch.from_numpy(v).to(out.device) for v in (rows, cols))
+    assert_close(out[r_t][:, c_t], ref, what)

@@ -6,10 +6,15 @@ small-output Wgrads), as in the training step.
 
 C1 (one linear, M=256) is compared element by element in both scaling
 modes.  C2-C6 (C6: the paper's own Qwen3-1.7B-shaped model) use the
-paper's blockwise recipe and are compared on sampled
-outputs the oracle computes one by one: every quantised byte and scale on
-sampled rows and columns, and every GEMM output on the cross product of
-sampled rows and columns (which contains the four corner 128x128 tiles).
+paper's blockwise recipe:
+  - quantised bytes: every FP8 byte and scale of X, W and dY (both copies)
+    on C2, C3, C4 and on layers 0, 13 and 27 of C5; W in full and X, dY on
+    the first/last 128 and 96 random rows and columns on the other 25 C5
+    layers and on C6;
+  - GEMM outputs (every layer of C5): the cross product of the first 128,
+    the last 128 and 96 random row and column indices of each output, i.e.
+    the four complete corner 128x128 tiles plus 9216 seeded random entries,
+    against the oracle's fp64 products.
 """
 import numpy as np
 import pytest
@@ -50,34 +55,39 @@ def test_c1_full(scaling):
     assert_close(out["dw"], ref["dw"], "wgrad")
 
 
-def _sampled(key, layer, idx, seed):
+def _sampled(key, layer, idx, seed, full_bytes=False):
     wl = W.WORKLOADS[key]
     li = W.make_linear(wl, layer, idx, DEV)
     out = run_linear(li.x, li.w, li.dy, P.SCALE_BLOCK, step_calls=True)
-    check_linear_sampled(li.x, li.w, li.dy, out, np.random.default_rng(seed))
+    check_linear_sampled(li.x, li.w, li.dy, out, np.random.default_rng(seed), full_bytes=full_bytes)
     del out, li
     torch.cuda.empty_cache()
 
 
 @pytest.mark.parametrize("idx", [0, 1])
 def test_c2_attention_projections(idx):
-    _sampled("C2", 0, idx, 20 + idx)
+    _sampled("C2", 0, idx, 20 + idx, full_bytes=True)
 
 
 @pytest.mark.parametrize("idx", [0, 1])
 def test_c3_mlp_with_outliers(idx):
-    _sampled("C3", 0, idx, 30 + idx)
+    _sampled("C3", 0, idx, 30 + idx, full_bytes=True)
 
 
 @pytest.mark.parametrize("idx", [0, 1, 2, 3])
 def test_c4_decoder_layer(idx):
-    _sampled("C4", 0, idx, 40 + idx)
+    _sampled("C4", 0, idx, 40 + idx, full_bytes=True)
 
 
-@pytest.mark.parametrize("layer", [0, 13, 27])
-@pytest.mark.parametrize("idx", [0, 1, 2, 3])
-def test_c5_layers(layer, idx):
-    _sampled("C5", layer, idx, 500 + 4 * layer + idx)
+C5_FULL_LAYERS = (0, 13, 27)
+
+
+@pytest.mark.parametrize("layer", range(28))
+def test_c5_layer(layer):
+    """All four linears of one C5 layer: every byte on layers 0, 13 and 27,
+    sampled rows and columns on the others; sampled GEMM outputs on all."""
+    for idx in range(4):
+        _sampled("C5", layer, idx, 500 + 4 * layer + idx, full_bytes=layer in C5_FULL_LAYERS)
 
 
 @pytest.mark.parametrize("layer", [0, 27])

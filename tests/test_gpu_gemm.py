@@ -14,7 +14,8 @@ import torch
 import oracle as O
 import paper_2608_27370_gb300 as P
 from paper_2608_27370_gb300 import workloads as W
-from _parity import assert_close, bits, host, oracle_linear, run_linear
+from _parity import (assert_close, bits, check_gemm_every_tile, host, oracle_linear, par_quantize_blocks_128x128,
+                     par_quantize_cols_128x1, par_quantize_rows_1x128, run_linear)
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda"
@@ -249,3 +250,108 @@ def test_grouped_backward_equals_separate_calls(M, N, K):
     torch.cuda.synchronize()
     assert torch.equal(dx.view(torch.int16), dx1.view(torch.int16))
     assert P.puro_fp8_get_status(status) == 0
+
+
+# --------------------------------------------------------------------------
+# Several tiles per CTA pair.  The persistent grid holds at most 76 pairs on
+# GB300 (152 SMs), so outputs of 256 or more 256-wide pair tiles make every
+# pair loop over 3-4 tiles: the persistent schedule, the alternation of the
+# accumulator buffers in tensor memory (two whole 256-column buffers for the
+# dense kinds, the shifted pair for the block-scaled kind) and the reuse of
+# the epilogue's staging.  Each output is checked on the cross product of one
+# sampled row and column in every 32 (every 32 x 32 piece of every tile).
+# Shapes: Y [4112, 4224] 17 x 17 pair tiles (ragged last row and column
+# tiles), dX [4112, 3968] 17 x 16, dW [4224, 3968] 17 x 16; the Wgrad
+# reduction (M = 4112 tokens) ends in a partial K stage.
+# --------------------------------------------------------------------------
+MANY_M, MANY_N, MANY_K = 4112, 4224, 3968
+
+
+def _f64(a):
+    return np.ascontiguousarray(a, dtype=np.float64)
+
+
+@pytest.mark.parametrize("fmt_g", [P.E4M3, P.E5M2], ids=["e4m3", "e5m2_gradients"])
+def test_tensor_linear_many_tiles_per_pair(fmt_g):
+    """Per-tensor scaling (workload C1's recipe), E4M3 throughout or with
+    E5M2 output gradients (the hybrid recipe), as the training step calls it."""
+    M, N, K = MANY_M, MANY_N, MANY_K
+    x, w, dy = _inputs(M, N, K, 7100 + fmt_g)
+    out = run_linear(x, w, dy, P.SCALE_TENSOR, P.E4M3, P.E4M3, fmt_g, step_calls=True)
+    ops = []
+    for t, q, fmt in ((x, out["xq"], P.E4M3), (w, out["wq"], P.E4M3), (dy, out["dyq"], fmt_g)):
+        amax, codes, si = O.quantize_tensor(bits(t), fmt)
+        assert int(host(q.amax)[0]) & 0xFFFF == amax
+        assert np.array_equal(host(q.rowwise.data), codes), "per-tensor codes (several tiles per CTA)"
+        assert np.array_equal(host(q.colwise.data), np.ascontiguousarray(codes.T)), "transposed per-tensor codes"
+        ops.append(O.dequant_tensor(codes, si, fmt))
+    X, Wd, dY = ops
+    rng = np.random.default_rng(7200 + fmt_g)
+    check_gemm_every_tile(out["y"], X, Wd, rng, "per-tensor fprop")
+    check_gemm_every_tile(out["dx"], dY, _f64(Wd.T), rng, "per-tensor dgrad")
+    check_gemm_every_tile(out["dw"], _f64(dY.T), _f64(X.T), rng, "per-tensor wgrad")
+
+
+def test_bf16_linear_many_tiles_per_pair():
+    """The BF16 comparison build (kind::f16) on the same multi-tile shapes."""
+    M, N, K = MANY_M, MANY_N, MANY_K
+    x, w, dy = _inputs(M, N, K, 7300)
+    y = torch.empty((M, N), dtype=torch.bfloat16, device=DEV)
+    dx = torch.empty((M, K), dtype=torch.bfloat16, device=DEV)
+    dw = torch.empty((N, K), dtype=torch.bfloat16, device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    P.puro_bf16_linear_fprop(x, w, y, M, N, K, dev_status=status)
+    P.puro_bf16_linear_dgrad(dy, w.t().contiguous(), dx, M, N, K, dev_status=status)
+    P.puro_bf16_linear_wgrad(dy.t().contiguous(), x.t().contiguous(), dw, M, N, K, dev_status=status)
+    torch.cuda.synchronize()
+    assert P.puro_fp8_get_status(status) == 0
+    X, Wd, dY = (O.bf16_to_double(bits(t)) for t in (x, w, dy))
+    rng = np.random.default_rng(7301)
+    check_gemm_every_tile(y, X, Wd, rng, "bf16 fprop")
+    check_gemm_every_tile(dx, dY, _f64(Wd.T), rng, "bf16 dgrad")
+    check_gemm_every_tile(dw, _f64(dY.T), _f64(X.T), rng, "bf16 wgrad")
+
+
+def test_block_linear_many_tiles_per_pair(tile_n):
+    """The paper's blockwise recipe on the same multi-tile shapes (M a
+    multiple of 128 here), both tile forms, separate (unsplit) calls."""
+    M, N, K = 4096, MANY_N, MANY_K
+    x, w, dy = _inputs(M, N, K, 7400, t3=True)
+    out = run_linear(x, w, dy, P.SCALE_BLOCK)
+    xb, wb, dyb = bits(x), bits(w), bits(dy)
+    X = O.dequant_rows_1x128(*par_quantize_rows_1x128(xb, P.E4M3), P.E4M3)
+    Xt = O.dequant_rows_1x128(*par_quantize_cols_128x1(xb, P.E4M3), P.E4M3)
+    Wd = O.dequant_blocks_128x128(*par_quantize_blocks_128x128(wb, P.E4M3), P.E4M3)
+    dY = O.dequant_rows_1x128(*par_quantize_rows_1x128(dyb, P.E4M3), P.E4M3)
+    dYt = O.dequant_rows_1x128(*par_quantize_cols_128x1(dyb, P.E4M3), P.E4M3)
+    rng = np.random.default_rng(7401 + tile_n)
+    check_gemm_every_tile(out["y"], X, Wd, rng, "block fprop")
+    check_gemm_every_tile(out["dx"], dY, _f64(Wd.T), rng, "block dgrad")
+    check_gemm_every_tile(out["dw"], dYt, Xt, rng, "block wgrad")
+
+
+def test_wgrad_main_grad_unsplit_gate_up_shape():
+    """main_grad += dY^T X into the FP32 [17920, 1536] main-grad of the
+    gate_up projection, unsplit (70 x 6 = 420 pair tiles, 5-6 per pair):
+    the increment against the oracle on every 32 x 32 piece of every tile."""
+    M, N, K = 1024, 17920, 1536
+    x, w, dy = _inputs(M, N, K, 7500, t3=True)
+    xq = P.quantize(x, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT)
+    dyq = P.quantize(dy, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT)
+    assert P.puro_fp8_workspace_size(N, K, M) == 0, "this output is large enough not to split"
+    main0 = W.normal_f32((N, K), 0.05, DEV, 7501)
+    main = main0.clone()
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    P.puro_fp8_linear_wgrad_main_grad(dyq.colwise, xq.colwise, main, dev_status=status)
+    torch.cuda.synchronize()
+    assert P.puro_fp8_get_status(status) == 0
+    rng = np.random.default_rng(7502)
+    from _parity import sample_every
+    rows, cols = sample_every(N, rng), sample_every(K, rng)
+    r_t, c_t = (torch.from_numpy(v).to(DEV) for v in (rows, cols))
+    dYt = O.dequant_rows_1x128(*par_quantize_cols_128x1(bits(dy[:, r_t]), P.E4M3), P.E4M3)
+    Xt = O.dequant_rows_1x128(*par_quantize_cols_128x1(bits(x[:, c_t]), P.E4M3), P.E4M3)
+    ref = O.gemm_tn(dYt, Xt, 8)
+    inc = (main[r_t][:, c_t].double() - main0[r_t][:, c_t].double()).cpu().numpy()
+    ok, ratio = O.within_tolerance(inc, ref)
+    assert ok, f"main-grad increment outside tolerance (worst ratio {ratio:.3g})"

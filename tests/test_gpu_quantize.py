@@ -167,6 +167,18 @@ def test_tensor_quantize(shape, fmt):
     check_tensor_quant(x, q, fmt)
 
 
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("shape", [(32768, 1536), (4112, 3968)])
+def test_tensor_quantize_many_tiles_per_cta(shape, fmt):
+    """The per-tensor quantiser is persistent (two CTAs per SM, 304 on
+    GB300): [32768, 1536] gives each CTA about ten 128 x 128 tiles, so the
+    loop, the double-buffered loads and the reuse of the staging tiles run
+    many times; [4112, 3968] adds ragged last row and column tiles.  Every
+    byte, amax and scale_inv against the oracle."""
+    x = _t3(shape, 160 + shape[1] + fmt, 2.0)
+    check_tensor_quant(x, P.quantize(x, fmt, P.SCALE_TENSOR, P.ROLE_ACT), fmt)
+
+
 def test_tensor_quantize_edge_cases():
     z = torch.zeros((32, 64), dtype=torch.bfloat16, device=DEV)
     q = P.quantize(z, P.E4M3, P.SCALE_TENSOR, P.ROLE_ACT)

@@ -78,21 +78,21 @@ def test_amax_validation(lib):
 def test_quantize_validation(lib):
     q = lib.puro_fp8_quantize
     BLK, TEN, ACT, WGT = P.SCALE_BLOCK, P.SCALE_TENSOR, P.ROLE_ACT, P.ROLE_WEIGHT
-    assert q(A, 128, 128, 7, BLK, ACT, None, A, A, A, A, None) == BAD       # bad format
-    assert q(A, 128, 128, 0, 9, ACT, None, A, A, A, A, None) == BAD         # bad scaling
-    assert q(A, 128, 128, 0, BLK, 5, None, A, A, A, A, None) == BAD         # bad role
-    assert q(A, 130, 128, 0, BLK, ACT, None, A, A, A, A, None) == BAD       # ragged rows in BLOCK
-    assert q(A, 128, 200, 0, BLK, WGT, None, A, A, A, A, None) == BAD       # ragged cols in BLOCK
-    assert q(A, 128, 128, 0, BLK, ACT, A, A, A, A, A, None) == BAD          # amax given in BLOCK
-    assert q(A, 128, 128, 0, BLK, ACT, None, A, A, A, None, None) == BAD    # q_t without scale_t
-    assert q(A, 128, 128, 0, BLK, ACT, None, A + 8, A, None, None, None) == BAD  # misaligned q
-    assert q(A, 128, 128, 0, TEN, ACT, None, A, A, None, None, None) == BAD  # TENSOR needs amax
-    assert q(A, 128, 120, 0, TEN, ACT, A, A, A, None, None, None) == BAD     # TENSOR cols % 16
-    assert q(A, 120, 128, 0, TEN, ACT, A, A, A, A, None, None) == BAD        # TENSOR rows % 16 with q_t
-    assert q(None, 128, 128, 0, BLK, ACT, None, A, A, A, A, None) == BAD     # null input
-    assert q(A, 128, 128, 0, BLK, ACT, None, None, A, None, None, None) == BAD  # null q
+    assert q(A, 128, 128, 7, BLK, ACT, None, A, A, A, A, None, None) == BAD       # bad format
+    assert q(A, 128, 128, 0, 9, ACT, None, A, A, A, A, None, None) == BAD         # bad scaling
+    assert q(A, 128, 128, 0, BLK, 5, None, A, A, A, A, None, None) == BAD         # bad role
+    assert q(A, 130, 128, 0, BLK, ACT, None, A, A, A, A, None, None) == BAD       # ragged rows in BLOCK
+    assert q(A, 128, 200, 0, BLK, WGT, None, A, A, A, A, None, None) == BAD       # ragged cols in BLOCK
+    assert q(A, 128, 128, 0, BLK, ACT, A, A, A, A, A, None, None) == BAD          # amax given in BLOCK
+    assert q(A, 128, 128, 0, BLK, ACT, None, A, A, A, None, None, None) == BAD    # q_t without scale_t
+    assert q(A, 128, 128, 0, BLK, ACT, None, A + 8, A, None, None, None, None) == BAD  # misaligned q
+    assert q(A, 128, 128, 0, TEN, ACT, None, A, A, None, None, None, None) == BAD  # TENSOR needs amax
+    assert q(A, 128, 120, 0, TEN, ACT, A, A, A, None, None, None, None) == BAD     # TENSOR cols % 16
+    assert q(A, 120, 128, 0, TEN, ACT, A, A, A, A, None, None, None) == BAD        # TENSOR rows % 16 with q_t
+    assert q(None, 128, 128, 0, BLK, ACT, None, A, A, A, A, None, None) == BAD     # null input
+    assert q(A, 128, 128, 0, BLK, ACT, None, None, A, None, None, None, None) == BAD  # null q
     # empty BLOCK tensors are a valid no-op that touches nothing
-    assert q(None, 0, 128, 0, BLK, ACT, None, A, A, A, A, None) == P.PURO_OK
+    assert q(None, 0, 128, 0, BLK, ACT, None, A, A, A, A, None, None) == P.PURO_OK
 
 
 def _op(rows, red, scaling=P.SCALE_BLOCK, role=P.ROLE_ACT, fmt=0, data=A, scale=A, reserved=0):
@@ -152,18 +152,18 @@ def test_grouped_weight_quantize_validation(lib):
 
     good = W_(A, 256, 384, A, A, A, A)
     no_t = W_(A, 256, 384, A, A, None, None)
-    assert f(None, 1, P.E4M3, None) == BAD                                   # no table
-    assert f(table(good), -1, P.E4M3, None) == BAD                           # negative count
-    assert f(table(good), 1, 5, None) == BAD                                 # bad format
-    assert f(table(W_(A, 200, 384, A, A, A, A)), 1, P.E4M3, None) == BAD      # rows % 128
-    assert f(table(good, no_t), 2, P.E4M3, None) == BAD                      # mixed transposed copies
-    assert f(table(W_(A, 256, 384, A, A, A, None)), 1, P.E4M3, None) == BAD  # q_t without scale_t
-    assert f(table(W_(A + 2, 256, 384, A, A, A, A)), 1, P.E4M3, None) == BAD  # misaligned input
-    assert f(table(W_(A, 256, 384, None, A, A, A)), 1, P.E4M3, None) == BAD   # no codes buffer
-    assert f(table(good, W_(A, 256, 384, A, A + 8, A, A)), 2, P.E4M3, None) == BAD  # checked before any launch
+    assert f(None, 1, P.E4M3, None, None) == BAD                                   # no table
+    assert f(table(good), -1, P.E4M3, None, None) == BAD                           # negative count
+    assert f(table(good), 1, 5, None, None) == BAD                                 # bad format
+    assert f(table(W_(A, 200, 384, A, A, A, A)), 1, P.E4M3, None, None) == BAD      # rows % 128
+    assert f(table(good, no_t), 2, P.E4M3, None, None) == BAD                      # mixed transposed copies
+    assert f(table(W_(A, 256, 384, A, A, A, None)), 1, P.E4M3, None, None) == BAD  # q_t without scale_t
+    assert f(table(W_(A + 2, 256, 384, A, A, A, A)), 1, P.E4M3, None, None) == BAD  # misaligned input
+    assert f(table(W_(A, 256, 384, None, A, A, A)), 1, P.E4M3, None, None) == BAD   # no codes buffer
+    assert f(table(good, W_(A, 256, 384, A, A + 8, A, A)), 2, P.E4M3, None, None) == BAD  # checked before any launch
     # nothing to do: valid no-ops
-    assert f(None, 0, P.E4M3, None) == P.PURO_OK
-    assert f(table(W_(None, 0, 384, None, None, None, None)), 1, P.E4M3, None) == P.PURO_OK
+    assert f(None, 0, P.E4M3, None, None) == P.PURO_OK
+    assert f(table(W_(None, 0, 384, None, None, None, None)), 1, P.E4M3, None, None) == P.PURO_OK
 
 
 def test_backward_validation(lib):
@@ -179,6 +179,21 @@ def test_backward_validation(lib):
     assert f(None, r(wt), A, r(dyt), r(xt), A, None, 0, None, None) == BAD
     # both empty: a valid no-op
     assert f(r(_op(0, 384)), r(wt), A, r(_op(0, 256)), r(xt), A, None, 0, None, None) == P.PURO_OK
+
+
+def test_noalloc_wgrad_checks_arguments_before_the_scratch_limit(lib):
+    # every call here is answered on the host before any CUDA call
+    f = lib.puro_fp8_linear_wgrad_noalloc
+    r = ctypes.byref
+    big_dyt, big_xt = _op(2048, 32768), _op(1792, 32768)   # a valid split would need 58.7 MB > 40 MiB
+    assert P.puro_fp8_workspace_size(2048, 1792, 32768) > 40 * 1024 * 1024
+    assert f(r(big_dyt), r(big_xt), A, None, None) == P.PURO_ERR_UNSUPPORTED
+    assert f(r(big_dyt), r(_op(1792, 32640)), A, None, None) == BAD          # reduction mismatch
+    assert f(r(_op(2048, 32768, fmt=9)), r(big_xt), A, None, None) == BAD    # bad format
+    assert f(r(big_dyt), r(big_xt), A + 4, None, None) == BAD               # misaligned dW
+    assert f(r(big_dyt), r(_op(1792, 32768, scaling=P.SCALE_TENSOR)), A, None, None) == BAD  # mixed scaling
+    assert f(None, r(big_xt), A, None, None) == BAD
+    assert f(r(_op(0, 32768)), r(big_xt), A, None, None) == P.PURO_OK       # empty output: no-op
 
 
 def test_bf16_gemm_validation(lib):
@@ -240,7 +255,7 @@ def test_fused_rmsnorm_validates_on_the_host(lib):
     def call(rows, cols, **kw):
         a = dict(args, **kw)
         return lib.puro_fp8_quantize_rmsnorm(fake, rows, cols, a["gamma"], a["eps"], a["fmt"], a["rstd"], a["y"],
-                                             a["q"], a["scale"], a["q_t"], a["scale_t"], a["stream"])
+                                             a["q"], a["scale"], a["q_t"], a["scale_t"], None, a["stream"])
 
     assert call(200, 256) == P.PURO_ERR_INVALID_ARG            # rows not a multiple of 128
     assert call(256, 200) == P.PURO_ERR_INVALID_ARG            # cols not a multiple of 128
@@ -256,7 +271,7 @@ def test_fused_swiglu_validates_on_the_host(lib):
     fake = 0x100000  # never dereferenced: every call below is refused before any CUDA call
 
     def call(rows, cols, ld, fmt=P.E4M3, gate=fake, up=fake, y=None, q_t=None, scale_t=None):
-        return lib.puro_fp8_quantize_swiglu(gate, up, rows, cols, ld, fmt, y, fake, fake, q_t, scale_t, None)
+        return lib.puro_fp8_quantize_swiglu(gate, up, rows, cols, ld, fmt, y, fake, fake, q_t, scale_t, None, None)
 
     assert call(200, 256, 512) == P.PURO_ERR_INVALID_ARG            # rows not a multiple of 128
     assert call(256, 200, 400) == P.PURO_ERR_INVALID_ARG            # cols not a multiple of 128

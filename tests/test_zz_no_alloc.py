@@ -5,11 +5,13 @@ backward pass (engine plugins that own every device buffer, latency-critical
 code that cannot pay for cudaMalloc's device-wide synchronisation, fixed
 memory budgets): instead of caller-supplied scratch, its split-reduction
 schedule uses a fixed array inside the library.  This test calls it through
-the C ABI and checks its output against the regular puro_fp8_linear_wgrad
-(given a workspace, so both take the split schedule), on two calls in a row
-with different inputs, within the tolerance the GEMM tests use.  It also
-checks that an oversize request is refused.  The file is named so that
-pytest collects it last.
+the C ABI on two calls in a row with different inputs.  Both calls take the
+same split schedule as the regular puro_fp8_linear_wgrad given a workspace,
+and sum the same FP32 partials in the same fixed order, so each output must
+equal the regular one bit for bit: a wrong offset into the shared array, or
+bytes the previous call left in it, would show.  Each output is also checked
+against the oracle's fp64 dW within the GEMM tolerance.  An oversize request
+must be refused.  The file is named so that pytest collects it last.
 """
 import ctypes
 
@@ -20,6 +22,7 @@ import torch
 import oracle as O
 import paper_2608_27370_gb300 as P
 from paper_2608_27370_gb300 import workloads as W
+from _parity import bits
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda"
@@ -33,12 +36,16 @@ def lib():
 
 
 def _operands(M, N, K, seed):
-    """Quantised Wgrad operands dY^T [N, M] and X^T [K, M] (blockwise E4M3)."""
+    """Quantised Wgrad operands dY^T [N, M] and X^T [K, M] (blockwise E4M3),
+    and the oracle's fp64 dW of the same BF16 inputs."""
     x = W.student_t3_f32((M, K), DEV, seed).to(torch.bfloat16)
     dy = W.normal_bf16((M, N), 1e-3, DEV, seed + 1)
     xq = P.quantize(x, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT)
     dyq = P.quantize(dy, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT)
-    return dyq.colwise, xq.colwise
+    xb, dyb = bits(x), bits(dy)
+    dYt = O.dequant_rows_1x128(*O.quantize_cols_128x1(dyb, P.E4M3), P.E4M3)
+    Xt = O.dequant_rows_1x128(*O.quantize_cols_128x1(xb, P.E4M3), P.E4M3)
+    return dyq.colwise, xq.colwise, O.gemm_tn(dYt, Xt, 8)
 
 
 def _as_f64(t):
@@ -52,7 +59,7 @@ def test_noalloc_wgrad_matches_regular_entry_point_twice(lib):
     stream = torch.cuda.current_stream().cuda_stream
     status = torch.zeros(1, dtype=torch.int32, device=DEV)
     for call, seed in enumerate((71, 93)):
-        dyt, xt = _operands(M, N, K, seed)
+        dyt, xt, dw_ref = _operands(M, N, K, seed)
         ref = torch.empty((N, K), dtype=torch.bfloat16, device=DEV)
         ws = torch.empty(ws_bytes, dtype=torch.uint8, device=DEV)
         P.puro_fp8_linear_wgrad(dyt, xt, ref, workspace=ws)
@@ -63,8 +70,10 @@ def test_noalloc_wgrad_matches_regular_entry_point_twice(lib):
         assert st == P.PURO_OK, f"call {call}: status {st}"
         torch.cuda.synchronize()
         assert P.puro_fp8_get_status(status) == 0
-        ok, ratio = O.within_tolerance(_as_f64(out), _as_f64(ref))
-        assert ok, f"call {call}: outside tolerance of the regular entry point (worst ratio {ratio:.3g})"
+        assert torch.equal(out.view(torch.int16), ref.view(torch.int16)), \
+            f"call {call}: differs from the regular entry point given a workspace"
+        ok, ratio = O.within_tolerance(_as_f64(out), dw_ref)
+        assert ok, f"call {call}: outside tolerance of the oracle (worst ratio {ratio:.3g})"
 
 
 def test_noalloc_wgrad_refuses_oversize_requests(lib):
