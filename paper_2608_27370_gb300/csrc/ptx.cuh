@@ -136,39 +136,6 @@ PURO_DEV void tma_store_2d(const CUtensorMap *map, const void *src, int32_t x, i
                  : "memory");
 }
 
-// ------------------------------------------------- L2 eviction priorities
-// A cache policy (createpolicy) attached to a TMA copy tells L2 how to rank
-// the lines it brings in or writes: evict_first for data streamed once (a
-// read-once input, an output nobody reads next), evict_last for data that is
-// read again soon (the operand every tile row or column of a GEMM re-reads),
-// so a streamed tensor does not push a reused one out.
-PURO_DEV uint64_t l2_policy_evict_first() {
-    uint64_t p;
-    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-    return p;
-}
-PURO_DEV uint64_t l2_policy_evict_last() {
-    uint64_t p;
-    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-    return p;
-}
-
-// tma_load_2d / tma_store_2d with an L2 cache policy.
-PURO_DEV void tma_load_2d_hint(void *dst, const CUtensorMap *map, uint64_t *bar, int32_t x, int32_t y,
-                               uint64_t policy) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-        " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "l"(policy)
-        : "memory");
-}
-PURO_DEV void tma_store_2d_hint(const CUtensorMap *map, const void *src, int32_t x, int32_t y, uint64_t policy) {
-    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group.L2::cache_hint [%0, {%2, %3}], [%1], %4;" ::"l"(
-                     reinterpret_cast<uint64_t>(map)),
-                 "r"(smem_u32(src)), "r"(x), "r"(y), "l"(policy)
-                 : "memory");
-}
-
 // 2-D tiled element-wise add shared -> global (bulk-group completion): each
 // element of the box is added to the global tensor's element (the tensor
 // map's type; f32 adds round to nearest).
@@ -264,16 +231,6 @@ PURO_DEV void tma_load_2d_pair(void *dst, const CUtensorMap *map, uint32_t bar_c
         "cp.async.bulk.tensor.2d.shared::cta.global.tile.mbarrier::complete_tx::bytes.cta_group::2"
         " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar_cluster)
-        : "memory");
-}
-
-// tma_load_2d_pair with an L2 cache policy.
-PURO_DEV void tma_load_2d_pair_hint(void *dst, const CUtensorMap *map, uint32_t bar_cluster, int32_t x, int32_t y,
-                                    uint64_t policy) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cta.global.tile.mbarrier::complete_tx::bytes.cta_group::2.L2::cache_hint"
-        " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar_cluster), "l"(policy)
         : "memory");
 }
 

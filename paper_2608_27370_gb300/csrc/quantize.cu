@@ -654,17 +654,21 @@ __global__ void __launch_bounds__(kQAThreads, 2)
         // ---- A: row groups (a warp holds its eight rows whole) and column partials
         float rmul[8];
         {
+            // each row's maximum in both halves of a word (the halves swapped
+            // and maxed), so one redux gives it without splitting the halves
             uint32_t rmax[8];
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
                 const uint32_t m = __vmaxu2(v[i].x & 0x7FFF7FFFu, v[i].y & 0x7FFF7FFFu);
-                rmax[i] = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
+                rmax[i] = __reduce_max_sync(0xFFFFFFFFu, __vmaxu2(m, __byte_perm(m, 0u, 0x1032)));
             }
+            // lane l takes row (l mod 8)'s maximum by a three-level select
+            const bool b0 = lane & 1, b1 = lane & 2, b2 = lane & 4;
+            const uint32_t s01 = b0 ? rmax[1] : rmax[0], s23 = b0 ? rmax[3] : rmax[2];
+            const uint32_t s45 = b0 ? rmax[5] : rmax[4], s67 = b0 ? rmax[7] : rmax[6];
+            const uint32_t mine = (b2 ? (b1 ? s67 : s45) : (b1 ? s23 : s01)) & 0xFFFFu;
             // lane i < 8 derives row 8br+i's scale; every lane then takes the
             // eight multipliers from those lanes
-            uint32_t mine = rmax[0];
-#pragma unroll
-            for (int i = 1; i < 8; ++i) mine = (lane == i) ? rmax[i] : mine;
             const uint32_t g = e8m0_exponent<FMT>(mine);
             const float mul = mul_of(g);
             if (lane < 8) sm.row_g[8 * br + lane] = static_cast<uint8_t>(g);
@@ -732,52 +736,112 @@ __global__ void __launch_bounds__(kQAThreads, 2)
 
         // ---- C: rowwise codes (row i, 4 columns) and transposed codes
         // (column j, 8 rows) from the block, re-read from shared memory.
+        // Every multiplier of the thread's rows and columns finite: the
+        // common path.  (A NaN multiplier -- a non-finite group -- makes the
+        // sum NaN; large finite ones can only overflow it to infinity.)
+        float4 cmv = make_float4(1.0f, 1.0f, 1.0f, 1.0f);
+        float msum = rmul[0];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) v[i] = *reinterpret_cast<const uint2 *>(in + (8 * br + i) * kQT + 4 * bc);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            const uint64_t m2 = f32x2(rmul[i], rmul[i]);
-            const uint32_t o = quant4<FMT>(bf16_lo(v[i].x), bf16_hi(v[i].x), bf16_lo(v[i].y), bf16_hi(v[i].y), m2,
-                                           isnan(rmul[i]));
-            *reinterpret_cast<uint32_t *>(sm.q_stage + (8 * br + i) * kQT + 4 * bc) = o;  // a warp: one 128-byte row
-        }
+        for (int i = 1; i < 8; ++i) msum += rmul[i];
         if constexpr (HAS_T) {
-            const float4 cmv = *reinterpret_cast<const float4 *>(&sm.col_mul[4 * bc]);
-            const float cmul[4] = {cmv.x, cmv.y, cmv.z, cmv.w};
-            uint2 cc[4];
+            cmv = *reinterpret_cast<const float4 *>(&sm.col_mul[4 * bc]);
+            msum += (cmv.x + cmv.y) + (cmv.z + cmv.w);
+        }
+        if (!isnan(msum)) {
+            // Each row's four values are widened to fp32 once and give both
+            // copies: the rowwise codes (the row's multiplier) and, packed
+            // into one word per row (byte j: column 4bc+j), the transposed
+            // codes (the columns' multipliers).  Eight 4x4 byte transposes
+            // then gather each column's eight codes; the first stage's
+            // selectors already put column (s + rot) mod 4 in output word s,
+            // the rotation that spreads the lanes' stores over all banks.
+            const uint64_t cm01 = f32x2(cmv.x, cmv.y), cm23 = f32x2(cmv.z, cmv.w);
+            uint32_t rw[8];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const uint64_t m2 = f32x2(cmul[j], cmul[j]);
-                const bool nan_col = isnan(cmul[j]);
-                float c[8];
+            for (int i = 0; i < 8; ++i) {
+                const uint2 w = *reinterpret_cast<const uint2 *>(in + (8 * br + i) * kQT + 4 * bc);
+                const uint64_t p0 = f32x2(bf16_lo(w.x), bf16_hi(w.x)), p1 = f32x2(bf16_lo(w.y), bf16_hi(w.y));
+                const uint64_t rr = f32x2(rmul[i], rmul[i]);
+                *reinterpret_cast<uint32_t *>(sm.q_stage + (8 * br + i) * kQT + 4 * bc) =
+                    cvt_f32x2<FMT>(mul_f32x2(p0, rr)) | (cvt_f32x2<FMT>(mul_f32x2(p1, rr)) << 16);
+                if constexpr (HAS_T)
+                    rw[i] = cvt_f32x2<FMT>(mul_f32x2(p0, cm01)) | (cvt_f32x2<FMT>(mul_f32x2(p1, cm23)) << 16);
+            }
+            if constexpr (HAS_T) {
+                const uint32_t rot = static_cast<uint32_t>(bc >> 1) & 3u;
+                const uint32_t a = rot, b = (rot + 1u) & 3u, c = (rot + 2u) & 3u, d = (rot + 3u) & 3u;
+                const uint32_t sel_ab = a | ((4u + a) << 4) | (b << 8) | ((4u + b) << 12);
+                const uint32_t sel_cd = c | ((4u + c) << 4) | (d << 8) | ((4u + d) << 12);
+                uint32_t wt[2][4];  // [rows 0-3 / 4-7][step s]: column (s + rot) mod 4
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const uint32_t w = (j >> 1) ? v[i].y : v[i].x;
-                    c[i] = (j & 1) ? bf16_hi(w) : bf16_lo(w);
+                for (int h = 0; h < 2; ++h) {
+                    const uint32_t x0 = __byte_perm(rw[4 * h], rw[4 * h + 1], sel_ab);
+                    const uint32_t x1 = __byte_perm(rw[4 * h], rw[4 * h + 1], sel_cd);
+                    const uint32_t x2 = __byte_perm(rw[4 * h + 2], rw[4 * h + 3], sel_ab);
+                    const uint32_t x3 = __byte_perm(rw[4 * h + 2], rw[4 * h + 3], sel_cd);
+                    wt[h][0] = __byte_perm(x0, x2, 0x5410);
+                    wt[h][1] = __byte_perm(x0, x2, 0x7632);
+                    wt[h][2] = __byte_perm(x1, x3, 0x5410);
+                    wt[h][3] = __byte_perm(x1, x3, 0x7632);
                 }
-                cc[j].x = quant4<FMT>(c[0], c[1], c[2], c[3], m2, nan_col);
-                cc[j].y = quant4<FMT>(c[4], c[5], c[6], c[7], m2, nan_col);
+#pragma unroll
+                for (int st = 0; st < 4; ++st) {
+                    const int r = 4 * bc + ((st + static_cast<int>(rot)) & 3);  // transposed row (tile column)
+                    *reinterpret_cast<uint2 *>(sm.qt_stage + r * kQT + 16 * ((br >> 1) ^ (r & 7)) + 8 * (br & 1)) =
+                        make_uint2(wt[0][st], wt[1][st]);
+                }
             }
-            // Column j's 8 codes (rows 8br .. 8br+7) go to transposed row
-            // 4bc + j, bytes 8br .. 8br+7, whose 16-byte chunk is
-            // (br / 2) ^ ((4bc + j) % 8) under the 128-byte swizzle.  All 32
-            // lanes of a warp share br, so storing the same j together would
-            // put them in two chunks; lane bc stores column (s + bc / 2) % 4 at
-            // step s, which spreads them over all eight (a rotation of cc).
-            const int rot = (bc >> 1) & 3;
+        } else {
+            // General path (a group of the tile held Inf or NaN): codes one by
+            // one with the NaN handling of quant4, the transposed ones rotated
+            // by register selects.
 #pragma unroll
-            for (int b = 1; b < 4; b <<= 1) {  // cc[s] <- cc[(s + rot) % 4], one rotate-by-b stage per bit
-                const bool on = (rot & b) != 0;
-                uint2 t[4];
+            for (int i = 0; i < 8; ++i) v[i] = *reinterpret_cast<const uint2 *>(in + (8 * br + i) * kQT + 4 * bc);
 #pragma unroll
-                for (int k = 0; k < 4; ++k) t[k] = on ? cc[(k + b) & 3] : cc[k];
-#pragma unroll
-                for (int k = 0; k < 4; ++k) cc[k] = t[k];
+            for (int i = 0; i < 8; ++i) {
+                const uint64_t m2 = f32x2(rmul[i], rmul[i]);
+                const uint32_t o = quant4<FMT>(bf16_lo(v[i].x), bf16_hi(v[i].x), bf16_lo(v[i].y), bf16_hi(v[i].y), m2,
+                                               isnan(rmul[i]));
+                *reinterpret_cast<uint32_t *>(sm.q_stage + (8 * br + i) * kQT + 4 * bc) = o;  // a warp: one 128-byte row
             }
+            if constexpr (HAS_T) {
+                const float4 cmv = *reinterpret_cast<const float4 *>(&sm.col_mul[4 * bc]);
+                const float cmul[4] = {cmv.x, cmv.y, cmv.z, cmv.w};
+                uint2 cc[4];
 #pragma unroll
-            for (int st = 0; st < 4; ++st) {
-                const int r = 4 * bc + ((st + rot) & 3);  // transposed row (tile column)
-                *reinterpret_cast<uint2 *>(sm.qt_stage + r * kQT + 16 * ((br >> 1) ^ (r & 7)) + 8 * (br & 1)) = cc[st];
+                for (int j = 0; j < 4; ++j) {
+                    const uint64_t m2 = f32x2(cmul[j], cmul[j]);
+                    const bool nan_col = isnan(cmul[j]);
+                    float c[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const uint32_t w = (j >> 1) ? v[i].y : v[i].x;
+                        c[i] = (j & 1) ? bf16_hi(w) : bf16_lo(w);
+                    }
+                    cc[j].x = quant4<FMT>(c[0], c[1], c[2], c[3], m2, nan_col);
+                    cc[j].y = quant4<FMT>(c[4], c[5], c[6], c[7], m2, nan_col);
+                }
+                // Column j's 8 codes (rows 8br .. 8br+7) go to transposed row
+                // 4bc + j, bytes 8br .. 8br+7, whose 16-byte chunk is
+                // (br / 2) ^ ((4bc + j) % 8) under the 128-byte swizzle.  All 32
+                // lanes of a warp share br, so storing the same j together would
+                // put them in two chunks; lane bc stores column (s + bc / 2) % 4 at
+                // step s, which spreads them over all eight (a rotation of cc).
+                const int rot = (bc >> 1) & 3;
+#pragma unroll
+                for (int b = 1; b < 4; b <<= 1) {  // cc[s] <- cc[(s + rot) % 4], one rotate-by-b stage per bit
+                    const bool on = (rot & b) != 0;
+                    uint2 t[4];
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) t[k] = on ? cc[(k + b) & 3] : cc[k];
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) cc[k] = t[k];
+                }
+#pragma unroll
+                for (int st = 0; st < 4; ++st) {
+                    const int r = 4 * bc + ((st + rot) & 3);  // transposed row (tile column)
+                    *reinterpret_cast<uint2 *>(sm.qt_stage + r * kQT + 16 * ((br >> 1) ^ (r & 7)) + 8 * (br & 1)) = cc[st];
+                }
             }
         }
 

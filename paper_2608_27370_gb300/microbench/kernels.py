@@ -9,6 +9,8 @@ enough that a full capture ends in seconds).  Not part of the library.
     python -m paper_2608_27370_gb300.microbench.kernels gemm_k1536  # gate_up Fprop, M = 8192, N = 17920, K = 1536
     python -m paper_2608_27370_gb300.microbench.kernels dgrad_quant  # down Dgrad + both FP8 copies of dX, M = 8192
     python -m paper_2608_27370_gb300.microbench.kernels quant    # gate_up output gradient [8192, 17920], both copies
+    python -m paper_2608_27370_gb300.microbench.kernels quant_small  # qkv / o_proj / gate_up input [32768, 1536], both copies
+    python -m paper_2608_27370_gb300.microbench.kernels gemm_oproj   # o_proj Fprop, M = 32768, N = 1536, K = 1536
     python -m paper_2608_27370_gb300.microbench.kernels tensor   # per-tensor scaling: amax, quantise, down Fprop, M = 8192
     python -m paper_2608_27370_gb300.microbench.kernels bf16     # down Fprop on BF16 operands (kind::f16), M = 8192
     python -m paper_2608_27370_gb300.microbench.kernels weight   # one weight's 128x128-block cast: gate_up W [17920, 1536]
@@ -58,8 +60,9 @@ def main(which: str) -> None:
         ws = torch.empty(P.puro_muonh_grouped_workspace_size(mats), dtype=torch.uint8, device=dev)
         for _ in range(2):
             P.puro_muonh_step_grouped(mats, 4.08e-4, sums, ws)
-    elif which in ("gemm", "gemm_k1536"):
-        M, N, K = (8192, 1536, 8960) if which == "gemm" else (8192, 17920, 1536)
+    elif which in ("gemm", "gemm_k1536", "gemm_oproj"):
+        M, N, K = {"gemm": (8192, 1536, 8960), "gemm_k1536": (8192, 17920, 1536),
+                   "gemm_oproj": (32768, 1536, 1536)}[which]
         a = P.quantize(W.normal_bf16((M, K), 1.0, dev, 1), transpose=False)
         b = P.quantize(W.normal_bf16((N, K), 0.02, dev, 2), P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT, transpose=False)
         d = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
@@ -74,8 +77,8 @@ def main(which: str) -> None:
         for _ in range(2):
             P.puro_fp8_linear_dgrad_quantize(dyq.rowwise, wt, P.E4M3, None, q.rowwise.data, q.rowwise.scale,
                                              q.colwise.data, q.colwise.scale)
-    elif which == "quant":
-        dy = W.normal_bf16((8192, 17920), 1e-3, dev, 3)
+    elif which in ("quant", "quant_small"):
+        dy = W.normal_bf16((8192, 17920) if which == "quant" else (32768, 1536), 1e-3, dev, 3)
         q = P.quantize(dy)
         for _ in range(2):
             P.quantize(dy, out=q)
@@ -130,8 +133,8 @@ def main(which: str) -> None:
             P.puro_rmsnorm_bf16(h, g, 1e-6, rstd, y)
             P.puro_swiglu_bf16(gu[:, :6144], gu[:, 6144:], hs)
     else:
-        raise SystemExit(f"unknown kernel {which!r}: swiglu, rmsnorm, muonh, gemm, gemm_k1536, dgrad_quant, quant, "
-                         "tensor, bf16, weight, splitk or unfused")
+        raise SystemExit(f"unknown kernel {which!r}: swiglu, rmsnorm, muonh, gemm, gemm_k1536, gemm_oproj, "
+                         "dgrad_quant, quant, quant_small, tensor, bf16, weight, splitk or unfused")
     torch.cuda.synchronize()
     print("ok", which)
 
