@@ -77,11 +77,6 @@ PURO_DEV uint32_t quant4(float a, float b, float c, float d, uint64_t mul2, bool
     return cvt_f32x2<FMT>(mul_f32x2(f32x2(a, b), mul2)) | (cvt_f32x2<FMT>(mul_f32x2(f32x2(c, d), mul2)) << 16);
 }
 
-// max of the bf16 magnitudes in each 16-bit half, over four words
-PURO_DEV uint32_t max_abs4(uint4 v) {
-    return __vmaxu2(__vmaxu2(v.x & 0x7FFF7FFFu, v.y & 0x7FFF7FFFu), __vmaxu2(v.z & 0x7FFF7FFFu, v.w & 0x7FFF7FFFu));
-}
-
 // Exact 2^(127 - g) as fp32 for g in [0, 247] (always a normal number).
 PURO_DEV float pow2_inv_scale(uint32_t g) { return __uint_as_float((254u - g) << 23); }
 

@@ -282,7 +282,10 @@ cudaError_t launch_swiglu_apply(const uint16_t *gate, const uint16_t *up, int64_
 
 // ------------------------------------------------------ cast kernel
 constexpr int kQT = 128;          // tile edge
-constexpr int kQThreads = 256;
+// Threads of the single-scale cast kernels (weights, per-tensor): thread t
+// owns the 8x4 block of rows 8*(t/32) .. +7 and columns 4*(t%32) .. +3 of
+// the 128x128 tile, the layout of the activation kernel below.
+constexpr int kQThreads = 512;
 
 // Shared memory of one CTA.  Both staging tiles are TMA store sources and
 // so 1024-byte aligned; the transposed tile uses the 128-byte swizzle
@@ -291,7 +294,7 @@ struct QuantSmem {
     alignas(1024) uint8_t q_stage[kQT * kQT];    // rowwise codes, plain rows
     alignas(1024) uint8_t qt_stage[kQT * kQT];   // transposed codes, 128B-swizzled rows
     alignas(128) uint16_t in[2][kQT * kQT];      // bf16 tile, double buffered
-    uint32_t red[8];                             // weight kind: per-warp block maxima
+    uint32_t red[kQThreads / 32];                // weight kind: per-warp block maxima
     uint64_t full[2];                            // TMA tile loads into in[0], in[1]
 };
 
@@ -326,63 +329,72 @@ PURO_DEV void quant_abort(uint64_t *full, int it, bool next_issued, int32_t *sta
 }
 
 
-// Rowwise codes (row i, 8 columns) and transposed codes (column j, 8 rows)
-// of one thread's 8x8 block v (rows 8br .. 8br+7, columns 8bc .. 8bc+7 of a
-// 128x128 tile) into the staging tiles, for a tile with one scale
-// (multiplier m2, twice; nan_all for a non-finite one).
-template <int FMT, bool HAS_T>
-PURO_DEV void tile_codes_to_stage(QuantSmem &sm, const uint4 (&v)[8], int br, int bc, uint64_t m2, bool nan_all) {
+// The transposed codes of one thread's 8x4 block (rows 8br .. 8br+7,
+// columns 4bc .. 4bc+3 of a 128x128 tile) into the transposed staging tile.
+// rw[i] holds row 8br+i's four codes, byte j for column 4bc+j.  Column j's
+// eight codes (rows 8br .. 8br+7) belong in transposed row 4bc + j, bytes
+// 8br .. 8br+7, whose 16-byte chunk is (br / 2) ^ ((4bc + j) % 8) under the
+// 128-byte swizzle.  All 32 lanes of a warp share br, so storing the same j
+// together would put them in two chunks; lane bc stores column
+// (s + bc / 2) % 4 at step s instead, which spreads them over all eight.
+// Two 4x4 byte transposes per four rows gather the columns, and the first
+// stage's selectors (per-lane constants) already put column (s + rot) % 4
+// in output word s, so the rotation costs no instruction.
+PURO_DEV void stage_transposed_8x4(uint8_t *qt_stage, const uint32_t (&rw)[8], int br, int bc) {
+    const uint32_t rot = static_cast<uint32_t>(bc >> 1) & 3u;
+    const uint32_t a = rot, b = (rot + 1u) & 3u, c = (rot + 2u) & 3u, d = (rot + 3u) & 3u;
+    const uint32_t sel_ab = a | ((4u + a) << 4) | (b << 8) | ((4u + b) << 12);
+    const uint32_t sel_cd = c | ((4u + c) << 4) | (d << 8) | ((4u + d) << 12);
+    uint32_t wt[2][4];  // [rows 0-3 / 4-7][step s]: column (s + rot) mod 4
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        uint2 o;
-        o.x = quant4<FMT>(bf16_lo(v[i].x), bf16_hi(v[i].x), bf16_lo(v[i].y), bf16_hi(v[i].y), m2, nan_all);
-        o.y = quant4<FMT>(bf16_lo(v[i].z), bf16_hi(v[i].z), bf16_lo(v[i].w), bf16_hi(v[i].w), m2, nan_all);
-        *reinterpret_cast<uint2 *>(sm.q_stage + (8 * br + i) * kQT + 8 * bc) = o;
+    for (int h = 0; h < 2; ++h) {
+        const uint32_t x0 = __byte_perm(rw[4 * h], rw[4 * h + 1], sel_ab);
+        const uint32_t x1 = __byte_perm(rw[4 * h], rw[4 * h + 1], sel_cd);
+        const uint32_t x2 = __byte_perm(rw[4 * h + 2], rw[4 * h + 3], sel_ab);
+        const uint32_t x3 = __byte_perm(rw[4 * h + 2], rw[4 * h + 3], sel_cd);
+        wt[h][0] = __byte_perm(x0, x2, 0x5410);
+        wt[h][1] = __byte_perm(x0, x2, 0x7632);
+        wt[h][2] = __byte_perm(x1, x3, 0x5410);
+        wt[h][3] = __byte_perm(x1, x3, 0x7632);
     }
-    if constexpr (HAS_T) {
-        // Column j's 8 codes (rows 8br .. 8br+7) go to transposed row
-        // 8bc + j, bytes 8br .. 8br+7.  Lanes of one half-warp share br,
-        // so they would all hit the same swizzled chunk if they stored
-        // the same j together; instead lane bc stores column (s + bc) % 8
-        // at step s, which spreads the 16 lanes over all 32 banks.  The
-        // per-lane order is a barrel rotation of the code array.
-        uint2 cc[8];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            float c[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const uint32_t w = (j >> 1) == 0 ? v[i].x : (j >> 1) == 1 ? v[i].y : (j >> 1) == 2 ? v[i].z : v[i].w;
-                c[i] = (j & 1) ? bf16_hi(w) : bf16_lo(w);
-            }
-            cc[j].x = quant4<FMT>(c[0], c[1], c[2], c[3], m2, nan_all);
-            cc[j].y = quant4<FMT>(c[4], c[5], c[6], c[7], m2, nan_all);
-        }
-        const int rot = bc & 7;
-#pragma unroll
-        for (int b = 1; b < 8; b <<= 1) {  // cc[s] <- cc[(s + rot) % 8], one rotate-by-b stage per bit
-            const bool on = (rot & b) != 0;
-            uint2 t[8];
-#pragma unroll
-            for (int k = 0; k < 8; ++k) t[k] = on ? cc[(k + b) & 7] : cc[k];
-#pragma unroll
-            for (int k = 0; k < 8; ++k) cc[k] = t[k];
-        }
-#pragma unroll
-        for (int st = 0; st < 8; ++st) {
-            const int r = 8 * bc + ((st + rot) & 7);  // transposed row (tile column)
-            *reinterpret_cast<uint2 *>(sm.qt_stage + r * kQT + 16 * ((br >> 1) ^ (r & 7)) + 8 * (br & 1)) = cc[st];
-        }
+    for (int st = 0; st < 4; ++st) {
+        const int r = 4 * bc + ((st + static_cast<int>(rot)) & 3);  // transposed row (tile column)
+        *reinterpret_cast<uint2 *>(qt_stage + r * kQT + 16 * ((br >> 1) ^ (r & 7)) + 8 * (br & 1)) =
+            make_uint2(wt[0][st], wt[1][st]);
     }
 }
 
+// Rowwise and transposed codes of one thread's 8x4 block v (rows 8br ..
+// 8br+7, columns 4bc .. 4bc+3) into the staging tiles, for a tile with one
+// multiplier (m2: it twice; nan_all: a non-finite tile).  With a single
+// scale the transposed codes are the rowwise codes transposed, so each
+// value is converted once.
+template <int FMT, bool HAS_T>
+PURO_DEV void tile_codes_to_stage(QuantSmem &sm, const uint2 (&v)[8], int br, int bc, uint64_t m2, bool nan_all) {
+    uint32_t rw[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        rw[i] = quant4<FMT>(bf16_lo(v[i].x), bf16_hi(v[i].x), bf16_lo(v[i].y), bf16_hi(v[i].y), m2, nan_all);
+        *reinterpret_cast<uint32_t *>(sm.q_stage + (8 * br + i) * kQT + 4 * bc) = rw[i];  // a warp: one 128-byte row
+    }
+    if constexpr (HAS_T) stage_transposed_8x4(sm.qt_stage, rw, br, bc);
+}
+
+// Maximum |bf16| of a thread's 8x4 block in both halves of a word.
+PURO_DEV uint32_t block_max_8x4(const uint2 (&v)[8]) {
+    uint32_t m = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) m = __vmaxu2(m, __vmaxu2(v[i].x & 0x7FFF7FFFu, v[i].y & 0x7FFF7FFFu));
+    return __vmaxu2(m, __byte_perm(m, 0u, 0x1032));
+}
+
 // Weight (128x128 blocks) and per-tensor cast kernel: one scale per tile
-// (the block's or the tensor's), so every thread owns one 8x8 block of the
-// 128x128 tile (rows 8*br .. 8*br+7, columns 8*bc .. 8*bc+7; a warp holds
-// two block rows of 16 blocks) and produces both its rowwise codes (q) and
-// its transposed codes (q_t) from the same registers.  The weight kind
-// reduces the block maximum through the warps (one barrier); the per-tensor
-// kind reads its scale from the device amax.
+// (the block's or the tensor's), so the transposed codes (q_t) are the
+// rowwise codes (q) transposed.  Thread t owns the 8x4 block of rows
+// 8*(t/32) .. +7 and columns 4*(t%32) .. +3.  The weight kind reduces the
+// block maximum through the warps (one barrier); the per-tensor kind reads
+// its scale from the device amax.
 template <int FMT, int KIND, bool HAS_T>
 __global__ void __launch_bounds__(kQThreads, 2)
     quant_tile_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_q,
@@ -395,8 +407,8 @@ __global__ void __launch_bounds__(kQThreads, 2)
     QuantSmem &sm = *reinterpret_cast<QuantSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                    ~static_cast<uintptr_t>(1023));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int br = 2 * warp + (lane >> 4);  // block row: tile rows 8br .. 8br+7
-    const int bc = lane & 15;               // block column: tile columns 8bc .. 8bc+7
+    const int br = warp;  // block row: tile rows 8br .. 8br+7
+    const int bc = lane;  // block column: tile columns 4bc .. 4bc+3
     pdl_wait();
     pdl_launch_dependents();
 
@@ -454,28 +466,24 @@ __global__ void __launch_bounds__(kQThreads, 2)
             }
         }
 
-        // ---- the thread's 8x8 block: v[i] = row 8br+i, columns 8bc .. 8bc+7
+        // ---- the thread's 8x4 block: v[i] = row 8br+i, columns 4bc .. 4bc+3
         const uint16_t *in = sm.in[buf];
-        uint4 v[8];
+        uint2 v[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) v[i] = *reinterpret_cast<const uint4 *>(in + (8 * br + i) * kQT + 8 * bc);
+        for (int i = 0; i < 8; ++i) v[i] = *reinterpret_cast<const uint2 *>(in + (8 * br + i) * kQT + 4 * bc);
 
         // ---- the tile's scale
         float mul = t_mul;
         uint32_t blk_g = 0;
         if constexpr (KIND == kQuantBlockWeight) {
-            uint32_t m = 0;
-#pragma unroll
-            for (int i = 0; i < 8; ++i) m = __vmaxu2(m, max_abs4(v[i]));
-            m = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
+            const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, block_max_8x4(v));
             if (lane == 0) sm.red[warp] = m;
             if (tid == 0) bulk_wait_group_read0();  // staging free (see above)
             if (__syncthreads_or(!landed)) {         // (S2) block maxima written, staging free
                 if (tid == 0) quant_abort(sm.full, it, tile + static_cast<int>(gridDim.x) < ntiles, status);
                 break;
             }
-            m = __reduce_max_sync(0xFFFFFFFFu, sm.red[lane & 7]);
-            blk_g = e8m0_exponent<FMT>(m);
+            blk_g = e8m0_exponent<FMT>(__reduce_max_sync(0xFFFFFFFFu, sm.red[lane & 15]) & 0xFFFFu);
             mul = mul_of(blk_g);
         }
         const uint64_t m2 = f32x2(mul, mul);
@@ -496,7 +504,7 @@ __global__ void __launch_bounds__(kQThreads, 2)
             // writes row i of the transposed operand (k-block r0/128); the
             // block's exponent repeats over its 128 rows.
             const bool col = tid >= kQT;
-            if (!col || HAS_T) {
+            if (tid < 2 * kQT && (!col || HAS_T)) {
                 const int i = tid & (kQT - 1);
                 const int64_t op_rows0 = col ? c0 : r0;
                 const int64_t kb = (col ? r0 : c0) / kQT;
@@ -751,10 +759,8 @@ __global__ void __launch_bounds__(kQAThreads, 2)
             // Each row's four values are widened to fp32 once and give both
             // copies: the rowwise codes (the row's multiplier) and, packed
             // into one word per row (byte j: column 4bc+j), the transposed
-            // codes (the columns' multipliers).  Eight 4x4 byte transposes
-            // then gather each column's eight codes; the first stage's
-            // selectors already put column (s + rot) mod 4 in output word s,
-            // the rotation that spreads the lanes' stores over all banks.
+            // codes (the columns' multipliers), which byte transposes then
+            // gather by column (stage_transposed_8x4).
             const uint64_t cm01 = f32x2(cmv.x, cmv.y), cm23 = f32x2(cmv.z, cmv.w);
             uint32_t rw[8];
 #pragma unroll
@@ -767,30 +773,7 @@ __global__ void __launch_bounds__(kQAThreads, 2)
                 if constexpr (HAS_T)
                     rw[i] = cvt_f32x2<FMT>(mul_f32x2(p0, cm01)) | (cvt_f32x2<FMT>(mul_f32x2(p1, cm23)) << 16);
             }
-            if constexpr (HAS_T) {
-                const uint32_t rot = static_cast<uint32_t>(bc >> 1) & 3u;
-                const uint32_t a = rot, b = (rot + 1u) & 3u, c = (rot + 2u) & 3u, d = (rot + 3u) & 3u;
-                const uint32_t sel_ab = a | ((4u + a) << 4) | (b << 8) | ((4u + b) << 12);
-                const uint32_t sel_cd = c | ((4u + c) << 4) | (d << 8) | ((4u + d) << 12);
-                uint32_t wt[2][4];  // [rows 0-3 / 4-7][step s]: column (s + rot) mod 4
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const uint32_t x0 = __byte_perm(rw[4 * h], rw[4 * h + 1], sel_ab);
-                    const uint32_t x1 = __byte_perm(rw[4 * h], rw[4 * h + 1], sel_cd);
-                    const uint32_t x2 = __byte_perm(rw[4 * h + 2], rw[4 * h + 3], sel_ab);
-                    const uint32_t x3 = __byte_perm(rw[4 * h + 2], rw[4 * h + 3], sel_cd);
-                    wt[h][0] = __byte_perm(x0, x2, 0x5410);
-                    wt[h][1] = __byte_perm(x0, x2, 0x7632);
-                    wt[h][2] = __byte_perm(x1, x3, 0x5410);
-                    wt[h][3] = __byte_perm(x1, x3, 0x7632);
-                }
-#pragma unroll
-                for (int st = 0; st < 4; ++st) {
-                    const int r = 4 * bc + ((st + static_cast<int>(rot)) & 3);  // transposed row (tile column)
-                    *reinterpret_cast<uint2 *>(sm.qt_stage + r * kQT + 16 * ((br >> 1) ^ (r & 7)) + 8 * (br & 1)) =
-                        make_uint2(wt[0][st], wt[1][st]);
-                }
-            }
+            if constexpr (HAS_T) stage_transposed_8x4(sm.qt_stage, rw, br, bc);
         } else {
             // General path (a group of the tile held Inf or NaN): codes one by
             // one with the NaN handling of quant4, the transposed ones rotated
@@ -869,8 +852,8 @@ __global__ void __launch_bounds__(kQThreads, 2) quant_weight_group_kernel(const 
     QuantSmem &sm = *reinterpret_cast<QuantSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                    ~static_cast<uintptr_t>(1023));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int br = 2 * warp + (lane >> 4);  // block row: tile rows 8br .. 8br+7
-    const int bc = lane & 15;               // block column: tile columns 8bc .. 8bc+7
+    const int br = warp;  // block row: tile rows 8br .. 8br+7
+    const int bc = lane;  // block column: tile columns 4bc .. 4bc+3
     pdl_wait();
     pdl_launch_dependents();
     if (tid == 0) {
@@ -910,21 +893,17 @@ __global__ void __launch_bounds__(kQThreads, 2) quant_weight_group_kernel(const 
         const bool landed = tile_landed(&sm.full[buf], static_cast<uint32_t>(it >> 1) & 1u, g.wait_ns);
 
         const uint16_t *in = sm.in[buf];
-        uint4 v[8];
+        uint2 v[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) v[i] = *reinterpret_cast<const uint4 *>(in + (8 * br + i) * kQT + 8 * bc);
-        uint32_t m = 0;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) m = __vmaxu2(m, max_abs4(v[i]));
-        m = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
+        for (int i = 0; i < 8; ++i) v[i] = *reinterpret_cast<const uint2 *>(in + (8 * br + i) * kQT + 4 * bc);
+        const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, block_max_8x4(v));
         if (lane == 0) sm.red[warp] = m;
         if (tid == 0) bulk_wait_group_read0();  // the previous tile's stores have read the staging
         if (__syncthreads_or(!landed)) {         // (S2) block maxima written, staging free
             if (tid == 0) quant_abort(sm.full, it, tile + static_cast<int>(gridDim.x) < ntiles, g.status);
             break;
         }
-        m = __reduce_max_sync(0xFFFFFFFFu, sm.red[lane & 7]);
-        const uint32_t blk_g = e8m0_exponent<FMT>(m);
+        const uint32_t blk_g = e8m0_exponent<FMT>(__reduce_max_sync(0xFFFFFFFFu, sm.red[lane & 15]) & 0xFFFFu);
         const float mul = mul_of(blk_g);
         tile_codes_to_stage<FMT, HAS_T>(sm, v, br, bc, f32x2(mul, mul), isnan(mul));
 
@@ -938,7 +917,7 @@ __global__ void __launch_bounds__(kQThreads, 2) quant_weight_group_kernel(const 
         // scale vectors: thread i < 128 row i of the rowwise copy, 128 + i row
         // i of the transposed copy (the block's exponent over its 128 rows)
         const bool col = tid >= kQT;
-        if (!col || HAS_T) {
+        if (tid < 2 * kQT && (!col || HAS_T)) {
             const int i = tid & (kQT - 1);
             store_scale_vec(col ? g.scale_t[w] : g.scale[w], (col ? c0 : r0) + i, (col ? r0 : c0) / kQT,
                             col ? g.kb_rows[w] : g.tiles_n[w], static_cast<uint8_t>(blk_g));
