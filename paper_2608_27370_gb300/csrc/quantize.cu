@@ -381,6 +381,22 @@ PURO_DEV void tile_codes_to_stage(QuantSmem &sm, const uint2 (&v)[8], int br, in
     if constexpr (HAS_T) stage_transposed_8x4(sm.qt_stage, rw, br, bc);
 }
 
+// Row and column block of a persistent CTA's tiles t, t + step, t + 2 step,
+// ... in a grid of tiles_n column blocks, advanced without a division.
+struct TileWalk {
+    int r, c, dr, dc, n;
+    PURO_DEV TileWalk(int t, int step, int tiles_n)
+        : r(t / tiles_n), c(t % tiles_n), dr(step / tiles_n), dc(step % tiles_n), n(tiles_n) {}
+    PURO_DEV void advance() {
+        r += dr;
+        c += dc;
+        if (c >= n) {
+            c -= n;
+            ++r;
+        }
+    }
+};
+
 // Maximum |bf16| of a thread's 8x4 block in both halves of a word.
 PURO_DEV uint32_t block_max_8x4(const uint2 (&v)[8]) {
     uint32_t m = 0;
@@ -437,19 +453,21 @@ __global__ void __launch_bounds__(kQThreads, 2)
 
     // One TMA load per 128x128 bf16 tile (out-of-range parts read as zero),
     // double buffered: tile it+1 streams in while tile it is processed.
-    auto issue_load = [&](int t, int b) {
+    auto issue_load = [&](const TileWalk &t, int b) {
         mbar_arrive_expect_tx(&sm.full[b], kQT * kQT * 2);
-        tma_load_2d(sm.in[b], &tm_x, &sm.full[b], (t % tiles_n) * kQT, (t / tiles_n) * kQT);
+        tma_load_2d(sm.in[b], &tm_x, &sm.full[b], t.c * kQT, t.r * kQT);
     };
     int tile = blockIdx.x;
-    if (tid == 0 && tile < ntiles) issue_load(tile, 0);
-    for (int it = 0; tile < ntiles; ++it, tile += gridDim.x) {
+    TileWalk cur(tile, gridDim.x, tiles_n), nxt = cur;
+    nxt.advance();
+    if (tid == 0 && tile < ntiles) issue_load(cur, 0);
+    for (int it = 0; tile < ntiles; ++it, tile += gridDim.x, cur = nxt, nxt.advance()) {
         const int buf = it & 1;
-        const int64_t r0 = static_cast<int64_t>(tile / tiles_n) * kQT;
-        const int64_t c0 = static_cast<int64_t>(tile % tiles_n) * kQT;
+        const int64_t r0 = static_cast<int64_t>(cur.r) * kQT;
+        const int64_t c0 = static_cast<int64_t>(cur.c) * kQT;
         if (tid == 0) {
             const int next = tile + gridDim.x;
-            if (next < ntiles) issue_load(next, buf ^ 1);  // its buffer was last read before (S3) of it-1
+            if (next < ntiles) issue_load(nxt, buf ^ 1);  // its buffer was last read before (S3) of it-1
             // The previous tile's TMA stores must have read the staging tiles
             // before they are rewritten: per-tensor mode writes them right
             // after (S1); the weight kind waits just before (S2).
@@ -594,33 +612,35 @@ __global__ void __launch_bounds__(kQAThreads, 2)
     pdl_wait();
     pdl_launch_dependents();
 
-    auto issue_load = [&](int t, int b) {
+    auto issue_load = [&](const TileWalk &t, int b) {
         mbar_arrive_expect_tx(&sm.full[b], kQT * kQT * 2);
-        tma_load_2d(sm.in[b], &tm_x, &sm.full[b], (t % tiles_n) * kQT, (t / tiles_n) * kQT);
+        tma_load_2d(sm.in[b], &tm_x, &sm.full[b], t.c * kQT, t.r * kQT);
     };
     int tile = blockIdx.x;
-    if (tid == 0 && tile < ntiles) issue_load(tile, 0);
+    TileWalk cur(tile, gridDim.x, tiles_n), nxt = cur;  // this tile and the CTA's next one
+    nxt.advance();
+    if (tid == 0 && tile < ntiles) issue_load(cur, 0);
     uint2 un[8];  // kProdSwiGlu: this thread's block of u for the current tile
-    auto load_up = [&](int t) {
-        const int64_t row0 = static_cast<int64_t>(t / tiles_n) * kQT + 8 * br;
-        const int64_t col0 = static_cast<int64_t>(t % tiles_n) * kQT + 4 * bc;
+    auto load_up = [&](const TileWalk &t) {
+        const int64_t row0 = static_cast<int64_t>(t.r) * kQT + 8 * br;
+        const int64_t col0 = static_cast<int64_t>(t.c) * kQT + 4 * bc;
         const uint16_t *p = prod.up + row0 * prod.ld + col0;
 #pragma unroll
         for (int i = 0; i < 8; ++i) un[i] = __ldg(reinterpret_cast<const uint2 *>(p + i * prod.ld));
     };
     if constexpr (PROD == kProdSwiGlu) {
-        if (tile < ntiles) load_up(tile);
+        if (tile < ntiles) load_up(cur);
     }
-    for (int it = 0; tile < ntiles; ++it, tile += gridDim.x) {
+    for (int it = 0; tile < ntiles; ++it, tile += gridDim.x, cur = nxt, nxt.advance()) {
         const int buf = it & 1;
-        const int64_t r0 = static_cast<int64_t>(tile / tiles_n) * kQT;
-        const int64_t c0 = static_cast<int64_t>(tile % tiles_n) * kQT;
+        const int64_t r0 = static_cast<int64_t>(cur.r) * kQT;
+        const int64_t c0 = static_cast<int64_t>(cur.c) * kQT;
         if (tid == 0) {
             const int next = tile + gridDim.x;
             // with a y output, the buffer's last reader was the y store of
             // tile it-1: all but the newest bulk group (its code stores) done
             if (PROD != kProdNone && prod.write_y) bulk_wait_group_read<1>();
-            if (next < ntiles) issue_load(next, buf ^ 1);  // its buffer was last read before (S4) of it-1
+            if (next < ntiles) issue_load(nxt, buf ^ 1);  // its buffer was last read before (S4) of it-1
         }
         // Every thread waits on the tile's barrier itself (which makes the
         // TMA-written tile visible to it); the shared buffers written before
@@ -655,8 +675,7 @@ __global__ void __launch_bounds__(kQAThreads, 2)
                 *reinterpret_cast<uint2 *>(in + (8 * br + i) * kQT + 4 * bc) = v[i];
             }
             if (prod.write_y) fence_proxy_async_smem();
-            const int next = tile + gridDim.x;
-            if (next < ntiles) load_up(next);
+            if (tile + static_cast<int>(gridDim.x) < ntiles) load_up(nxt);
         }
 
         // ---- A: row groups (a warp holds its eight rows whole) and column partials
