@@ -14,6 +14,7 @@ enough that a full capture ends in seconds).  Not part of the library.
     python -m paper_2608_27370_gb300.microbench.kernels tensor   # per-tensor scaling: amax, quantise, down Fprop, M = 8192
     python -m paper_2608_27370_gb300.microbench.kernels bf16     # down Fprop on BF16 operands (kind::f16), M = 8192
     python -m paper_2608_27370_gb300.microbench.kernels weight   # one weight's 128x128-block cast: gate_up W [17920, 1536]
+    python -m paper_2608_27370_gb300.microbench.kernels weights  # one grouped launch: the four weights of eight C5 layers
     python -m paper_2608_27370_gb300.microbench.kernels splitk   # qkv Wgrad at M = 32768: split reduction, BF16 and FP32 main-grad
     python -m paper_2608_27370_gb300.microbench.kernels unfused  # the unfused producers: RMSNorm [32768, 1536], SwiGLU [8192, 6144]
 
@@ -107,6 +108,17 @@ def main(which: str) -> None:
         q = P.quantize(w, P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT)
         for _ in range(2):
             P.quantize(w, P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT, out=q)
+    elif which == "weights":
+        # the step's grouped weight cast: 32 weights (eight C5 layers' qkv,
+        # o_proj, gate_up, down; 1.5 GB of BF16) in one launch, both copies
+        entries = []
+        for layer in range(8):
+            for j, (_, N, K) in enumerate(W.QWEN2_1P5B_LINEARS):
+                w = W.normal_bf16((N, K), 0.02, dev, 100 + 4 * layer + j)
+                entries.append((w, P.quantize(w, P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT)))
+        table = P.weight_table(entries)
+        for _ in range(2):
+            P.puro_fp8_quantize_weights(table, P.E4M3)
     elif which == "splitk":
         # the qkv Wgrad of C5 (dW [2048, 1536], reduction over M = 32768): a
         # 2048 x 1536 output has too few tiles for the SMs, so the reduction
@@ -134,7 +146,7 @@ def main(which: str) -> None:
             P.puro_swiglu_bf16(gu[:, :6144], gu[:, 6144:], hs)
     else:
         raise SystemExit(f"unknown kernel {which!r}: swiglu, rmsnorm, muonh, gemm, gemm_k1536, gemm_oproj, "
-                         "dgrad_quant, quant, quant_small, tensor, bf16, weight, splitk or unfused")
+                         "dgrad_quant, quant, quant_small, tensor, bf16, weight, weights, splitk or unfused")
     torch.cuda.synchronize()
     print("ok", which)
 
