@@ -322,9 +322,10 @@ class LinearStack:
         self.launches_per_step += 1
 
     def _backward_launches(self, N, K):
-        # one grouped launch when neither GEMM splits its reduction, else their own launches
-        dg, wg = self._gemm_launches(self.M, K, N), self._gemm_launches(N, K, self.M)
-        return 1 if dg == 1 and wg == 1 and self.scaling == self.P.SCALE_BLOCK else dg + wg
+        # the library's own plan for puro_fp8_linear_backward with this workspace
+        if self.scaling == self.P.SCALE_BLOCK:
+            return self.P.puro_fp8_linear_backward_launches(self.M, N, K, self.workspace.numel())
+        return self._gemm_launches(self.M, K, N) + self._gemm_launches(N, K, self.M)
 
     def _gemm_launches(self, rows_out, cols_out, red):
         # one GEMM kernel, plus the reduction kernel when the split schedule is taken

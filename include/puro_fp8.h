@@ -289,14 +289,19 @@ puro_status_t puro_fp8_linear_wgrad(const puro_fp8_tensor_t *dy_t, const puro_fp
  * The two are independent (both need only the quantised output gradient),
  * so when both run as unsplit 256-wide block-scaled GEMMs they share one
  * persistent launch: the tiles of the GEMM with the longer reduction first,
- * then the other's, which fill the last round of tiles.  Each output is
- * then bit-identical to the separate call's without a workspace.  Otherwise
- * (per-tensor scaling, a split reduction, the 224-wide tile form, an empty
- * extent) the two GEMMs are launched one after the other, exactly as the
- * separate entry points would.  Arguments as for those entry points; one
- * workspace serves both (its bytes: the larger of the two
- * puro_fp8_workspace_size values).  Both are validated before anything is
- * enqueued.
+ * then the other's.  Where the long tiles do not divide evenly over the CTA
+ * pairs, the pairs with one long tile fewer first take about a long tile's
+ * worth of short ones, so the pairs finish together.  A Wgrad that would
+ * split its reduction with the given workspace joins the Dgrad unsplit in
+ * such a launch when that is modelled faster (it is for every linear of the
+ * Qwen2-1.5B and Qwen3-1.7B shapes at their token counts).  Each output of a
+ * grouped launch is bit-identical to the separate call's without a
+ * workspace.  Otherwise (per-tensor scaling, a split reduction, the
+ * 224-wide tile form, an empty extent) the two GEMMs are launched one after
+ * the other, exactly as the separate entry points would.  Arguments as for
+ * those entry points; one workspace serves both (its bytes: the larger of
+ * the two puro_fp8_workspace_size values).  Both are validated before
+ * anything is enqueued.
  */
 puro_status_t puro_fp8_linear_backward(const puro_fp8_tensor_t *dy, const puro_fp8_tensor_t *w_t, void *dx,
                                        const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t, void *dw,
@@ -386,6 +391,15 @@ puro_status_t puro_fp8_linear_wgrad_main_grad(const puro_fp8_tensor_t *dy_t, con
 #define PURO_NOALLOC_SCRATCH_BYTES (40u * 1024u * 1024u)
 puro_status_t puro_fp8_linear_wgrad_noalloc(const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t, void *dw,
                                             int32_t *dev_status, void *stream);
+
+/*
+ * Kernel launches puro_fp8_linear_backward makes for block-scaled operands
+ * of a linear with M tokens, N output and K input features, given
+ * workspace_bytes of (16-byte aligned) workspace: 1 for a grouped launch,
+ * else one per GEMM plus one per split reduction.  0 for an empty extent.
+ * Host-only, no CUDA call.
+ */
+int32_t puro_fp8_linear_backward_launches(int64_t M, int64_t N, int64_t K, size_t workspace_bytes);
 
 /*
  * Bytes of a PURO_SCALE_BLOCK scale buffer for an operand [rows, red]

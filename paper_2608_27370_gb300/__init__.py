@@ -86,6 +86,7 @@ _SIGNATURES = {
     "puro_fp8_linear_wgrad_main_grad": (_I32, [_P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "puro_fp8_linear_wgrad_noalloc": (_I32, [_P, _P, _P, _P, _P]),
     "puro_fp8_workspace_size": (ctypes.c_size_t, [_I64, _I64, _I64]),
+    "puro_fp8_linear_backward_launches": (_I32, [_I64, _I64, _I64, ctypes.c_size_t]),
     "puro_fp8_scale_bytes": (ctypes.c_size_t, [_I64, _I64]),
     "puro_fp8_get_status": (_I32, [_P, _P, _P]),
     "puro_bf16_linear_fprop": (_I32, [_P, _P, _P, _I64, _I64, _I64, _P, _P]),
@@ -447,6 +448,12 @@ def puro_fp8_linear_wgrad_noalloc(dy_t: FP8Operand, x_t: FP8Operand, dw: torch.T
                                                       _ptr(dw, torch.bfloat16, "dw"),
                                                       _ptr(dev_status, torch.int32, "dev_status"), _stream(stream))
     _check("puro_fp8_linear_wgrad_noalloc", st)
+
+
+def puro_fp8_linear_backward_launches(M: int, N: int, K: int, workspace_bytes: int) -> int:
+    """Kernel launches of puro_fp8_linear_backward for block-scaled operands
+    (M tokens, N out, K in features) given a workspace of that many bytes."""
+    return int(load_library().puro_fp8_linear_backward_launches(M, N, K, workspace_bytes))
 
 
 def puro_fp8_workspace_size(rows_out: int, cols_out: int, red: int) -> int:

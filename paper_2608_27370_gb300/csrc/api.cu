@@ -198,9 +198,41 @@ puro_status_t fp8_gemm(const puro_fp8_tensor_t *a, const puro_fp8_tensor_t *b, v
     return run_fp8_gemm(action, g, m, static_cast<cudaStream_t>(stream));
 }
 
-// Dgrad and Wgrad of one linear: one grouped launch when both are unsplit
-// 256-wide block-scaled GEMMs (the problem with the longer reduction first,
-// so the other's shorter tiles fill the last round), else two.
+// How a linear's backward (Dgrad dX [M, K] over N, Wgrad dW [N, K] over M,
+// block-scaled) runs, given `ws` usable workspace bytes: one grouped launch
+// when both GEMMs are 256-wide and unsplit -- or when the Wgrad would split
+// its reduction but one grouped launch with it unsplit is modelled faster --
+// else each GEMM on its own (a split Wgrad adds its reduction kernel).
+struct BackwardPlan {
+    bool grouped;        // one launch for both
+    bool wgrad_unsplit;  // the Wgrad gives up the split it would take, to join the Dgrad
+    int launches;        // kernel launches
+};
+
+BackwardPlan plan_backward(int64_t M, int64_t N, int64_t K, size_t ws) {
+    auto split_of = [&](int64_t r, int64_t c, int64_t red) {
+        const int sp = choose_splits(r, c, red, false);
+        return (sp > 1 && ws >= splitk_workspace_bytes(r, c, red, false)) ? sp : 1;
+    };
+    auto tile_of = [&](int64_t r, int64_t c, int64_t red) {
+        const int forced = g_tile_n.load();
+        return forced ? forced : choose_tile_n(r, c, red);
+    };
+    BackwardPlan b{};
+    const int sd = split_of(M, K, N), sw = split_of(N, K, M);
+    if (sd == 1 && tile_of(M, K, N) == 256 && tile_of(N, K, M) == 256) {
+        if (sw == 1)
+            b.grouped = true;
+        else
+            b.grouped = b.wgrad_unsplit = grouped_backward_faster(M, N, K, sw);
+    }
+    b.launches = b.grouped ? 1 : (sd > 1 ? 2 : 1) + (sw > 1 ? 2 : 1);
+    return b;
+}
+
+// Dgrad and Wgrad of one linear: one grouped launch when plan_backward says
+// so (the problem with the longer reduction first; the balanced schedule
+// lets the pairs with fewer of its tiles take more of the other's), else two.
 puro_status_t fp8_backward(const puro_fp8_tensor_t *dy, const puro_fp8_tensor_t *w_t, void *dx,
                            const puro_fp8_tensor_t *dy_t, const puro_fp8_tensor_t *x_t, void *dw, void *workspace,
                            size_t workspace_bytes, int32_t *dev_status, void *stream) {
@@ -213,7 +245,12 @@ puro_status_t fp8_backward(const puro_fp8_tensor_t *dy, const puro_fp8_tensor_t 
     GemmAction ad, aw;
     st = prepare_fp8_gemm(dy, w_t, dx, workspace, workspace_bytes, dev_status, false, &gd, &md, &ad);
     if (st != PURO_OK) return st;
-    st = prepare_fp8_gemm(dy_t, x_t, dw, workspace, workspace_bytes, dev_status, false, &gw, &mw, &aw);
+    const size_t ws_usable = (workspace && aligned16(workspace)) ? workspace_bytes : 0;
+    const bool both_block = dy->scaling == PURO_SCALE_BLOCK && dy_t->scaling == PURO_SCALE_BLOCK;
+    const bool unsplit_w = both_block && dy->rows > 0 && dy->red > 0 && w_t->rows > 0 &&
+                           plan_backward(dy->rows, dy->red, w_t->rows, ws_usable).wgrad_unsplit;
+    st = prepare_fp8_gemm(dy_t, x_t, dw, unsplit_w ? nullptr : workspace, unsplit_w ? 0 : workspace_bytes, dev_status,
+                          false, &gw, &mw, &aw);
     if (st != PURO_OK) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const bool grouped = ad == kGemmLaunch && aw == kGemmLaunch && gd.kind == kGemmFP8Block &&
@@ -621,6 +658,11 @@ PURO_API puro_status_t puro_fp8_linear_wgrad_main_grad(const puro_fp8_tensor_t *
                                                        float *main_grad, void *workspace, size_t workspace_bytes,
                                                        int32_t *dev_status, void *stream) {
     return fp8_gemm(dy_t, x_t, main_grad, workspace, workspace_bytes, dev_status, stream, true);
+}
+
+PURO_API int32_t puro_fp8_linear_backward_launches(int64_t M, int64_t N, int64_t K, size_t workspace_bytes) {
+    if (M <= 0 || N <= 0 || K <= 0) return 0;
+    return plan_backward(M, N, K, workspace_bytes).launches;
 }
 
 PURO_API size_t puro_fp8_workspace_size(int64_t rows_out, int64_t cols_out, int64_t red) {

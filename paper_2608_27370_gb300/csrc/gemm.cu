@@ -52,6 +52,7 @@
 // barrier before tensor memory is freed.
 #include <cuda_bf16.h>
 
+#include <algorithm>
 #include <type_traits>
 
 #include "internal.h"
@@ -141,6 +142,9 @@ struct GemmParams {
     int units0;
     int N1, num_m1, num_n1, num_kb1, m_fastest1, kgroups1;
     uint32_t idesc1;
+    // Grouped launch: short (second-problem) units the pairs with one long
+    // unit fewer take first (see PairUnits); 0: plain round-robin.
+    int lead;
 };
 
 // Instruction descriptors (tcgen05.mma), both operands K-major, M = 256
@@ -173,6 +177,44 @@ PURO_DEV void record_timeout(Smem &sm, int32_t *status) {
 struct WorkUnit {
     int m0, n0, kb0, kb1, split;  // m0: first row of the pair tile
     int problem;                  // 0, or 1 for the second problem of a grouped launch
+};
+
+// The work units of one CTA pair, in the order it takes them.  A launch
+// hands them out round-robin over its P pairs: pair p takes units p, p + P,
+// p + 2P, ...  A grouped launch puts the problem with the longer reduction
+// first (units [0, units0)), so its long units go round-robin and the short
+// ones follow in the same global order, which lets the pairs that got one
+// long unit fewer start on the short ones first.  Where there are fewer long
+// units than pairs (a small Wgrad output grouped with its Dgrad), the pairs
+// without one would idle through most of the launch, so they first take
+// `lead` short units among themselves (about one long unit's worth of
+// work), and then every pair goes on round-robin over the rest.  The
+// sequence is a function of (params, pair, P) alone: the producer, the MMA
+// issuer, the helpers and the epilogue of both CTAs walk the same one.
+struct PairUnits {
+    int p, P, units0, u1, plong, pshort, lead, rank, nh, k;
+    PURO_DEV PairUnits(const GemmParams &gp, int pair, int num_pairs)
+        : p(pair), P(num_pairs), units0(gp.units0), u1(gp.num_units - gp.units0), k(0) {
+        plong = units0 % P;                    // pairs [0, plong) take one long unit more
+        pshort = P - plong;
+        rank = (p - plong + P) % P;            // the pair's turn in the short units' round-robin
+        lead = (units0 < P && u1 > 0) ? gp.lead : 0;
+        nh = units0 / P + (p < plong ? 1 : 0);
+    }
+    // The next unit, or -1 when the pair is done.
+    PURO_DEV int next() {
+        if (k < nh) return p + P * k++;
+        int kk = k++ - nh;
+        if (lead > 0 && rank < pshort) {
+            if (kk < lead) {
+                const int j = rank + pshort * kk;
+                return j < u1 ? units0 + j : -1;
+            }
+            kk -= lead;
+        }
+        const int j = pshort * lead + rank + P * kk;
+        return j < u1 ? units0 + j : -1;
+    }
 };
 
 template <int BN>
@@ -267,7 +309,8 @@ PURO_DEV void quant_epilogue(Smem &sm, const GemmParams &p, uint32_t tmem, int w
     const uint32_t sel1 = (lane & 1) ? 0x3715u : 0x6240u;
     const uint32_t sel2 = (lane & 2) ? 0x3276u : 0x5410u;
     int local = 0;
-    for (int u = pair; u < p.num_units; u += num_pairs, ++local) {
+    PairUnits units(p, pair, num_pairs);
+    for (int u = units.next(); u >= 0; u = units.next(), ++local) {
         const WorkUnit wu = work_unit<256>(p, u);
         const int m0 = wu.m0 + kBM * rank;
         const int nq = wu.n0 + 64 * j;  // first column of the quarter
@@ -504,7 +547,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
             uint32_t stage = 0, phase = 0;
             uint32_t issued = 0;  // stage fills started by this thread
             bool aborted = false;
-            for (int u = pair; u < p.num_units && !aborted; u += num_pairs) {
+            PairUnits units(p, pair, num_pairs);
+            for (int u = units.next(); u >= 0 && !aborted; u = units.next()) {
                 const WorkUnit wu = work_unit<BN>(p, u);
                 const int a_row = wu.m0 + kBM * static_cast<int>(rank);
                 const int b_row = wu.n0 + kBNHalf * static_cast<int>(rank);
@@ -568,7 +612,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
         uint32_t gseq = 0;  // groups of four k-blocks started (BN = 224: slot of the scale ring)
         bool aborted = false;
         int local = 0;
-        for (int u = pair; u < p.num_units && !aborted; u += num_pairs, ++local) {
+        PairUnits units(p, pair, num_pairs);
+        for (int u = units.next(); u >= 0 && !aborted; u = units.next(), ++local) {
             const WorkUnit wu = work_unit<BN>(p, u);
             const int buf = local % kAccBufs;
             const uint32_t acc_phase = static_cast<uint32_t>(local / kAccBufs) & 1u;
@@ -663,7 +708,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
         const uint32_t mine = static_cast<uint32_t>(warp - 2);
         uint32_t gseq = 0;
         bool aborted = false;
-        for (int u = pair; u < p.num_units && !aborted; u += num_pairs) {
+        PairUnits units(p, pair, num_pairs);
+        for (int u = units.next(); u >= 0 && !aborted; u = units.next()) {
             const WorkUnit wu = work_unit<BN>(p, u);
             for (int kb = wu.kb0; kb < wu.kb1; kb += kStagesPerGroup, ++gseq) {
                 if ((gseq & 1u) != mine) continue;
@@ -713,7 +759,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(gemm_threads<OUT>(),
         const uint32_t tempty0 = mapa_shared(smem_u32(&sm.tempty[0]), 0);  // the even CTA's
         int local = 0;
         uint32_t pieces = 0;  // BF16 output: 32-column pieces stored, alternating staging halves
-        for (int u = pair; u < p.num_units; u += num_pairs, ++local) {
+        PairUnits units(p, pair, num_pairs);
+        for (int u = units.next(); u >= 0; u = units.next(), ++local) {
             const WorkUnit wu = work_unit<BN>(p, u);
             const int m0 = wu.m0 + kBM * static_cast<int>(rank), n0 = wu.n0;  // this CTA's rows
             const int buf = local % kAccBufs;
@@ -999,6 +1046,7 @@ static GemmParams make_params(const GemmArgs &g, int splits) {
     p.d_bf16 = static_cast<uint16_t *>(g.d_bf16);
     p.q_fmt = g.q_fmt;
     p.units0 = p.num_units;  // one problem unless a grouped launch adds a second
+    p.lead = 0;
     return p;
 }
 
@@ -1063,7 +1111,30 @@ cudaError_t launch_gemm_grouped(const GemmArgs &g0, const GemmMaps &m0, const Ge
     p.kgroups1 = q.kgroups;
     p.idesc1 = q.idesc;
     p.num_units += q.num_units;
+    // the pairs with one long unit fewer first take about a long unit's
+    // worth of short ones (rounded)
+    p.lead = q.num_kb > 0 ? (2 * p.num_kb + q.num_kb) / (2 * q.num_kb) : 0;
     return launch_params<kGemmFP8Block, kGemmOutBF16, 256>(p, g0, m0, m1, s);
+}
+
+// Modelled time, in pipeline stages of one pair, of a linear's Dgrad and
+// Wgrad as one grouped launch with the balanced schedule (the longer
+// reduction's tiles first), against separate launches where the Wgrad
+// splits its reduction into `w_splits` chunks (plus its reduction kernel and
+// launch, about 20 stages).  Host-only, shape-only.
+bool grouped_backward_faster(int64_t M, int64_t N, int64_t K, int w_splits) {
+    const int64_t P = kSplitRefPairs;
+    auto tiles = [](int64_t r, int64_t c) { return ((r + kPairM - 1) / kPairM) * ((c + 255) / 256); };
+    auto stages = [](int64_t red) { return (red + kBKBytes - 1) / kBKBytes; };
+    const int64_t ud = tiles(M, K), ld = stages(N);  // Dgrad: dX [M, K], reduction N
+    const int64_t uw = tiles(N, K), lw = stages(M);  // Wgrad: dW [N, K], reduction M
+    const int64_t u0 = ld >= lw ? ud : uw, l0 = ld >= lw ? ld : lw;
+    const int64_t u1 = ld >= lw ? uw : ud, l1 = ld >= lw ? lw : ld;
+    const int64_t grouped = std::max((u0 + P - 1) / P * l0, (u0 * l0 + u1 * l1 + P - 1) / P + l1);
+    if (w_splits <= 1) return true;  // both unsplit: one launch, no worse than two
+    const int64_t chunk = ((lw + w_splits - 1) / w_splits + kStagesPerGroup - 1) / kStagesPerGroup * kStagesPerGroup;
+    const int64_t separate = (ud + P - 1) / P * ld + (uw * w_splits + P - 1) / P * chunk + 20;
+    return grouped < separate;
 }
 
 cudaError_t launch_gemm(const GemmArgs &g, const GemmMaps &m, cudaStream_t s) {

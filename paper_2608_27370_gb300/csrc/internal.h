@@ -198,6 +198,11 @@ puro_status_t fp8_gemm_validate(const puro_fp8_tensor_t *a, const puro_fp8_tenso
 int choose_splits(int64_t M, int64_t N, int64_t K, bool bf16);
 size_t splitk_workspace_bytes(int64_t M, int64_t N, int64_t K, bool bf16);
 int64_t splitk_rows_per_chunk(int64_t M);  // M rounded up to a whole 256-row pair tile
+// Whether a linear's Dgrad (dX [M, K], reduction N) and Wgrad (dW [N, K],
+// reduction M) are modelled faster as one grouped launch (balanced
+// schedule, Wgrad unsplit) than as two launches with the Wgrad split into
+// w_splits chunks.  Host-only, shape-only.
+bool grouped_backward_faster(int64_t M, int64_t N, int64_t K, int w_splits);
 // Tile width (256 or 224) of an unsplit block-scaled GEMM: modelled waves x
 // per-tile time of the two forms.  Host-only, shape-only.
 int choose_tile_n(int64_t M, int64_t N, int64_t K);

@@ -217,6 +217,36 @@ def test_wgrad_main_grad_zero_reduction_leaves_it_unchanged():
     assert torch.equal(main, before)
 
 
+def test_backward_groups_a_wgrad_that_would_split():
+    """qkv shape at 8192 tokens with a workspace: the Wgrad ([2048, 1536]
+    output, 48 tiles) would split its reduction, but one grouped launch with
+    it unsplit is modelled faster, so both outputs are bit-identical to the
+    separate calls without a workspace, and within tolerance of the oracle."""
+    M, N, K = 8192, 2048, 1536
+    assert P.puro_fp8_workspace_size(N, K, M) > 0, "the Wgrad alone would split"
+    ws_bytes = max(P.puro_fp8_workspace_size(M, K, N), P.puro_fp8_workspace_size(N, K, M))
+    assert P.puro_fp8_linear_backward_launches(M, N, K, ws_bytes) == 1
+    x, w, dy = _inputs(M, N, K, 6500, t3=True)
+    xq = P.quantize(x, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT)
+    wq = P.quantize(w, P.E4M3, P.SCALE_BLOCK, P.ROLE_WEIGHT)
+    dyq = P.quantize(dy, P.E4M3, P.SCALE_BLOCK, P.ROLE_ACT)
+    dx, dw = torch.empty((M, K), dtype=torch.bfloat16, device=DEV), torch.empty((N, K), dtype=torch.bfloat16, device=DEV)
+    dx1, dw1 = torch.empty_like(dx), torch.empty_like(dw)
+    ws = torch.full((ws_bytes,), 0xFF, dtype=torch.uint8, device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    P.puro_fp8_linear_backward(dyq.rowwise, wq.colwise, dx, dyq.colwise, xq.colwise, dw, ws, dev_status=status)
+    P.puro_fp8_linear_dgrad(dyq.rowwise, wq.colwise, dx1)
+    P.puro_fp8_linear_wgrad(dyq.colwise, xq.colwise, dw1)
+    torch.cuda.synchronize()
+    assert P.puro_fp8_get_status(status) == 0
+    assert torch.equal(dx.view(torch.int16), dx1.view(torch.int16))
+    assert torch.equal(dw.view(torch.int16), dw1.view(torch.int16)), "dW is not the unsplit Wgrad's"
+    rng = np.random.default_rng(6501)
+    dYt = O.dequant_rows_1x128(*par_quantize_cols_128x1(bits(dy), P.E4M3), P.E4M3)
+    Xt = O.dequant_rows_1x128(*par_quantize_cols_128x1(bits(x), P.E4M3), P.E4M3)
+    check_gemm_every_tile(dw, dYt, Xt, rng, "grouped wgrad")
+
+
 @pytest.mark.parametrize("M,N,K", [(8192, 4096, 2048),     # both unsplit: one grouped launch
                                    (4096, 2304, 1536),     # ragged last rounds in both
                                    (2048, 1536, 1536)])    # Wgrad small enough to split: two launches

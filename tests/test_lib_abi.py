@@ -196,6 +196,23 @@ def test_noalloc_wgrad_checks_arguments_before_the_scratch_limit(lib):
     assert f(r(_op(0, 32768)), r(big_xt), A, None, None) == P.PURO_OK       # empty output: no-op
 
 
+def test_backward_plan_groups_every_c5_and_c6_linear(lib):
+    # host-only: with the bench's workspace (large enough for any split) the
+    # Dgrad and the Wgrad of every linear share one launch -- the qkv and
+    # o_proj Wgrads, which would split, join their Dgrads unsplit
+    big = 1 << 30
+    for M, shapes in ((32768, [(2048, 1536), (1536, 1536), (17920, 1536), (1536, 8960)]),
+                      (8192, [(4096, 2048), (2048, 2048), (12288, 2048), (2048, 6144)])):
+        for N, K in shapes:
+            assert lib.puro_fp8_linear_backward_launches(M, N, K, big) == 1, (M, N, K)
+            assert lib.puro_fp8_linear_backward_launches(M, N, K, 0) == 1, (M, N, K)
+    assert lib.puro_fp8_linear_backward_launches(0, 2048, 1536, big) == 0
+    # a Dgrad that splits its reduction (2 output tiles, reduction 32768) is
+    # never grouped: its two launches (partials, reduction) plus the Wgrad's
+    assert lib.puro_fp8_linear_backward_launches(512, 32768, 256, big) == 3
+    assert lib.puro_fp8_linear_backward_launches(512, 32768, 256, 0) == 1  # no workspace: both unsplit, grouped
+
+
 def test_bf16_gemm_validation(lib):
     assert lib.puro_bf16_linear_fprop(A, A, A, 12, 16, 16, None, None) == BAD   # M % 8
     assert lib.puro_bf16_linear_fprop(A, A + 2, A, 16, 16, 16, None, None) == BAD
