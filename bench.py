@@ -758,6 +758,85 @@ def paper_model_measure(P, W, torch, device, scaling, steps=5, warmup=3):
     return out
 
 
+def library_context(torch, stack):
+    """Library context, not part of the path: the same twelve GEMMs as
+    bf16_layer_speedup (Fprop, Dgrad and Wgrad of layer 0's four linears,
+    operands already in the layout each GEMM reads, GEMM time only) through
+    torch's wrappers of NVIDIA's libraries: cuBLASLt FP8 (torch._scaled_mm)
+    with E4M3 operands and per-tensor fp32 scales, cuBLASLt MXFP8 with one
+    E8M0 scale per 32 elements of K (the blockwise recipe's arithmetic, each
+    1x128 scale repeated four times) where this torch build accepts it, and
+    cuBLAS BF16 (torch.matmul).  The operand values are the workload's, cast
+    to FP8 by torch; every scale is 1."""
+    f8 = torch.float8_e4m3fn
+    dev = stack.device
+    M = stack.M
+    li0 = stack.inputs[0]
+    ops = []
+    for j, (_, N, K) in enumerate(stack.wl.linears):
+        li = li0[j]
+        x8, w8, dy8 = li.x.to(f8), (li.w * 50.0).to(f8), (li.dy * 1000.0).to(f8)
+        # row-major A [rows, red] and column-major B [red, cols] of each GEMM
+        ops.append(("fprop", x8, w8.t(), li.x, li.w.t(), N, K))
+        ops.append(("dgrad", dy8, w8.t().contiguous().t(), li.dy, li.w, N, K))
+        ops.append(("wgrad", dy8.t().contiguous(), x8.t().contiguous().t(), li.dy.t(), li.x, N, K))
+    one = torch.ones((), dtype=torch.float32, device=dev)
+
+    def mx_scales(rows, red):
+        def up(a, b):
+            return (a + b - 1) // b * b
+        # E8M0 1.0 (byte 127) in the library's blocked layout: its size is
+        # the padded [rows, red / 32] grid (128-row by 4-column blocks)
+        return torch.full((up(rows, 128), up((red + 31) // 32, 4)), 127, dtype=torch.uint8,
+                          device=dev).view(torch.float8_e8m0fnu)
+
+    def timeit(fn, reps=5):
+        for _ in range(2):
+            fn()
+        torch.cuda.synchronize()
+        s = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        s.record()
+        for _ in range(reps):
+            fn()
+        e.record()
+        torch.cuda.synchronize()
+        return s.elapsed_time(e) * 1e-3 / reps
+
+    flops = sum(6.0 * M * N * K for _, N, K in stack.wl.linears)
+    out = {"layer": 0, "note": "NVIDIA libraries through torch, for context; not on the path"}
+
+    def per_tensor():
+        for _, a, b, _, _, _, _ in ops:
+            torch._scaled_mm(a, b, one, one, out_dtype=torch.bfloat16)
+
+    def bf16():
+        for _, _, _, a, b, _, _ in ops:
+            torch.matmul(a, b)
+
+    try:
+        out["cublaslt_fp8_per_tensor_tflops"] = flops / timeit(per_tensor) / 1e12
+    except (RuntimeError, TypeError) as exc:
+        out["cublaslt_fp8_per_tensor_tflops"] = None
+        out["cublaslt_fp8_per_tensor_unavailable"] = str(exc).splitlines()[0][:200]
+    try:
+        mx = [(a, b, mx_scales(a.shape[0], a.shape[1]), mx_scales(b.shape[1], b.shape[0])) for _, a, b, *_ in ops]
+
+        def mxfp8():
+            for a, b, sa, sb in mx:
+                torch._scaled_mm(a, b, sa, sb, out_dtype=torch.bfloat16)
+
+        out["cublaslt_mxfp8_tflops"] = flops / timeit(mxfp8) / 1e12
+        del mx
+    except (RuntimeError, TypeError, AttributeError) as exc:
+        out["cublaslt_mxfp8_tflops"] = None
+        out["cublaslt_mxfp8_unavailable"] = str(exc).splitlines()[0][:200]
+    out["cublas_bf16_tflops"] = flops / timeit(bf16) / 1e12
+    del ops
+    torch.cuda.empty_cache()
+    return out
+
+
 def e2e_measure(P, torch, stack, steps):
     """The same step (the same library calls, through `stack.step`) with
     host-resident inputs: every layer's X and dY are copied from pinned host
@@ -1024,6 +1103,10 @@ def main():
             result["bf16_comparison"] = bf16_layer_speedup(P, torch, stack)
         except (RuntimeError, torch.cuda.OutOfMemoryError) as exc:  # report, do not hide
             result["bf16_comparison"] = {"error": str(exc)}
+        try:
+            result["library_context"] = library_context(torch, stack)
+        except (RuntimeError, torch.cuda.OutOfMemoryError) as exc:
+            result["library_context"] = {"error": str(exc)}
     if rank == 0 and world == 1 and not args.no_paper_model and args.scaling == "block":
         result["e5m2_gradients"] = grad_format_measure(P, torch, stack)
     if not args.no_e2e:
