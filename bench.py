@@ -38,6 +38,10 @@ sys.path.insert(0, ROOT)
 
 METRIC = "FP8 linear fwd+bwd TFLOP/s and % of FP8 peak; quantise HBM GB/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# GB300's nominal figures, reported beside the measured denominators as
+# context: dense FP8 tensor rate and HBM3e bandwidth.
+NOMINAL_FP8_DENSE_TFLOPS = 4500.0
+NOMINAL_HBM_GBS = 7900.0
 FP8_PER_BF16 = 2.0  # nominal dense ratio (4.5 / 2.25 PFLOP/s)
 FP8_FLOP_PER_CLK_SM = 16384  # dense FP8 tensor-pipe rate per SM (a 256x256x32 pair MMA per 128 cycles)
 
@@ -1065,6 +1069,7 @@ def main():
                    "scaling": args.scaling, "l2": "inputs larger than L2 (>=2.4 GB per layer)",
                    "parallelism": f"replicas x{world} (weak scaling, no collective on the path)"},
         "pct_fp8_peak": 100.0 * value / world / fp8_peak_sust,
+        "step_frac_vs_nominal_fp8": value / world / NOMINAL_FP8_DENSE_TFLOPS,
         "tokens_per_s": world * M / step_s,
         "gemm_only_tflops": gemm_tflops,
         "quantize_gbs": quant_gbs,
@@ -1075,14 +1080,18 @@ def main():
                      "peak_source": f"2 x bf16_tflops_sustained ({peak_src}); kernel timed inside a long step",
                      "traffic": captured_traffic("gemm", traffic_wl, stack.gemm_algorithmic_bytes_per_call()),
                      "traffic_note": "DRAM bytes per GEMM launch: DRAM bytes per algorithmic byte from per-kernel ncu captures of one layer's GEMM calls, times the step's average launch",
-                     "timing": "CUDA events around each launch of the last timed step, on the launching stream"},
+                     "timing": "CUDA events around each launch of the last timed step, on the launching stream",
+                     "nominal_peak": NOMINAL_FP8_DENSE_TFLOPS,
+                     "frac_vs_nominal": gemm_tflops / NOMINAL_FP8_DENSE_TFLOPS},
         "roofline_quantize": {"bound": "hbm", "kernel": "quant_act_kernel (X, dY) + quant_weight_group_kernel (W)", "achieved": quant_gbs,
                               "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": quant_gbs / peaks["hbm_gbs"],
                               "peak_source": f"hbm_gbs ({peak_src})",
                               "traffic": captured_traffic("quantize", traffic_wl,
                                                           q["units"] / stack.quantize_kernel_launches_per_step()),
                               "traffic_note": "DRAM bytes per quantiser launch: DRAM bytes per algorithmic byte from per-kernel ncu captures of one layer's quantiser calls, times the step's average launch",
-                              "timing": "CUDA events around each launch of the last timed step, on the launching stream"},
+                              "timing": "CUDA events around each launch of the last timed step, on the launching stream",
+                              "nominal_peak": NOMINAL_HBM_GBS,
+                              "frac_vs_nominal": quant_gbs / NOMINAL_HBM_GBS},
     }
     if args.scaling == "tensor":
         result["roofline"]["kernel"] = "gemm_tn_kernel<FP8 per-tensor>"
