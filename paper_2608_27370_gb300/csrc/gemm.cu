@@ -280,6 +280,31 @@ PURO_DEV uint32_t quant2_cols(float x0, float x1, float m0, float m1) {
     return r;
 }
 
+// 4x4 transpose of 16-byte chunks within each quad of lanes: on entry
+// x[4k .. 4k+3] is chunk k of this lane's row; on exit lane c of the quad
+// holds, in x[4r .. 4r+3], chunk c of the quad's row r.  A warp's store of
+// x[4r .. 4r+3] then writes whole 64-byte row segments (eight rows per
+// instruction) instead of a 16-byte piece of each of 32 rows.
+PURO_DEV void quad_transpose_chunks(uint32_t (&x)[16], int lane) {
+    const int qi = lane & 3;
+#pragma unroll
+    for (int b = 1; b <= 2; b <<= 1) {
+        const bool up = (qi & b) != 0;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            if (k & b) continue;  // chunk pairs (k, k | b): the lower lane sends k | b, the upper k
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+                const uint32_t got = __shfl_xor_sync(0xFFFFFFFFu, sel_u32(up, x[4 * k + w], x[4 * (k | b) + w]), b);
+                if (up)
+                    x[4 * k + w] = got;
+                else
+                    x[4 * (k | b) + w] = got;
+            }
+        }
+    }
+}
+
 // Quantising epilogue (kGemmOutQuant), run by warps 4..19 of both CTAs of
 // a pair.  Warp 4 + 4j + q takes column quarter j (columns 64j .. 64j+63 of
 // every tile; half h = j / 2) and, as its tensor-memory lane quarter q, the
@@ -345,10 +370,21 @@ PURO_DEV void quant_epilogue(Smem &sm, const GemmParams &p, uint32_t tmem, int w
         const bool rows_in = m0 < p.M;  // the CTA's 128 rows
         const int64_t row = static_cast<int64_t>(m0 + 32 * q + lane);
 
-        if (p.d_bf16 && rows_in) {
-            uint4 *dst = reinterpret_cast<uint4 *>(p.d_bf16 + row * p.N + nq);
+        // rows of the quad of lanes this lane stores for (quad_transpose_chunks)
+        const int64_t quad_row = static_cast<int64_t>(m0 + 32 * q + (lane & ~3));
+        const int qc = lane & 3;
+        if (p.d_bf16 && rows_in) {  // the row's 64 BF16 values: two groups of four 16-byte chunks
 #pragma unroll
-            for (int i = 0; i < 8; ++i) dst[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+            for (int h2 = 0; h2 < 2; ++h2) {
+                uint32_t x[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) x[i] = v[16 * h2 + i];
+                quad_transpose_chunks(x, lane);
+#pragma unroll
+                for (int r = 0; r < 4; ++r)
+                    *reinterpret_cast<uint4 *>(p.d_bf16 + (quad_row + r) * p.N + nq + 32 * h2 + 8 * qc) =
+                        make_uint4(x[4 * r], x[4 * r + 1], x[4 * r + 2], x[4 * r + 3]);
+            }
         }
 
         // ---- rowwise copy: the row's 1x128 group is this quarter and its partner
@@ -364,17 +400,20 @@ PURO_DEV void quant_epilogue(Smem &sm, const GemmParams &p, uint32_t tmem, int w
             const uint64_t rm2 = f32x2(rmul, rmul);
             const bool rnan = isnan(rmul);
             if (rows_in) {
-                uint4 *dst = reinterpret_cast<uint4 *>(p.q + row * p.N + nq);
+                uint32_t x[16];  // x[4i .. 4i+3]: codes of columns 16i .. 16i+15 of the quarter
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {  // codes of columns 16i .. 16i+15 of the quarter
-                    uint32_t w[4];
+                for (int i = 0; i < 4; ++i) {
 #pragma unroll
                     for (int k = 0; k < 4; ++k) {
                         const uint32_t a = v[8 * i + 2 * k], b = v[8 * i + 2 * k + 1];
-                        w[k] = quant4<FMT>(bf16_lo(a), bf16_hi(a), bf16_lo(b), bf16_hi(b), rm2, rnan);
+                        x[4 * i + k] = quant4<FMT>(bf16_lo(a), bf16_hi(a), bf16_lo(b), bf16_hi(b), rm2, rnan);
                     }
-                    dst[i] = make_uint4(w[0], w[1], w[2], w[3]);
                 }
+                quad_transpose_chunks(x, lane);
+#pragma unroll
+                for (int r = 0; r < 4; ++r)
+                    *reinterpret_cast<uint4 *>(p.q + (quad_row + r) * p.N + nq + 16 * qc) =
+                        make_uint4(x[4 * r], x[4 * r + 1], x[4 * r + 2], x[4 * r + 3]);
                 if ((j & 1) == 0)  // one scale per row and group
                     store_scale_vec(p.q_scale, row, (wu.n0 + 128 * h) / 128, p.N / 128, static_cast<uint8_t>(g));
             }
