@@ -766,7 +766,8 @@ def library_context(torch, stack):
     """Library context, not part of the path: the same twelve GEMMs as
     bf16_layer_speedup (Fprop, Dgrad and Wgrad of layer 0's four linears,
     operands already in the layout each GEMM reads, GEMM time only) through
-    torch's wrappers of NVIDIA's libraries: cuBLASLt FP8 (torch._scaled_mm)
+    torch's wrappers of NVIDIA's libraries, and ours with per-tensor scales
+    beside them (bf16_layer_speedup has ours blockwise): cuBLASLt FP8 (torch._scaled_mm)
     with E4M3 operands and per-tensor fp32 scales, cuBLASLt MXFP8 with one
     E8M0 scale per 32 elements of K (the blockwise recipe's arithmetic, each
     1x128 scale repeated four times) where this torch build accepts it, and
@@ -818,6 +819,24 @@ def library_context(torch, stack):
         for _, _, _, a, b, _, _ in ops:
             torch.matmul(a, b)
 
+    # ours, the same twelve GEMMs with per-tensor scales (E4M3, scale_inv product in the epilogue)
+    import paper_2608_27370_gb300 as P
+    ours_t = []
+    for j, (_, N, K) in enumerate(stack.wl.linears):
+        li = li0[j]
+        ours_t.append((P.quantize(li.x, P.E4M3, P.SCALE_TENSOR, P.ROLE_ACT),
+                       P.quantize(li.w, P.E4M3, P.SCALE_TENSOR, P.ROLE_WEIGHT),
+                       P.quantize(li.dy, P.E4M3, P.SCALE_TENSOR, P.ROLE_ACT)))
+
+    def ours_per_tensor():
+        for j, (xq, wq, dyq) in enumerate(ours_t):
+            P.puro_fp8_linear_fprop(xq.rowwise, wq.rowwise, stack.y[j])
+        for j, (xq, wq, dyq) in enumerate(ours_t):
+            P.puro_fp8_linear_dgrad(dyq.rowwise, wq.colwise, stack.dx[j], stack.workspace)
+            P.puro_fp8_linear_wgrad(dyq.colwise, xq.colwise, stack.dw[j], stack.workspace)
+
+    out["ours_fp8_per_tensor_tflops"] = flops / timeit(ours_per_tensor) / 1e12
+    del ours_t
     try:
         out["cublaslt_fp8_per_tensor_tflops"] = flops / timeit(per_tensor) / 1e12
     except (RuntimeError, TypeError) as exc:
