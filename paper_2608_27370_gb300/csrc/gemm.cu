@@ -317,7 +317,9 @@ PURO_DEV void quad_transpose_chunks(uint32_t (&x)[16], int lane) {
 // whose warps exchange row maxima at the half's named barrier; 128x1 groups
 // along M -- exactly this CTA's 128 rows, the quarter's four warps -- for
 // the transposed copy).  All outputs leave by plain global stores from
-// registers: a row's 64 codes as four 16-byte stores; the transposed codes
+// registers: a row's 64 codes (and its 64 BF16 values, when asked for)
+// after a transpose of 16-byte chunks within each quad of lanes, so that a
+// store instruction writes eight whole 64-byte row segments; the transposed codes
 // after a 4x4 byte transpose within each quad of lanes, as 4-byte stores
 // that fill a 32-byte sector per column and warp.  The accumulator is
 // released once every quarter is in registers (32 arrivals), so no warp can
